@@ -1,0 +1,367 @@
+#!/usr/bin/env python
+"""Throughput of 8-bit quantized LSTM acoustic-model inference on GB300 (one JSON line on stdout).
+
+A step is one qnn_lstm_forward over one batch of synthetic frames: per-frame activation
+quantization, the integer products of every layer, recovery fused with the gates and the cell
+update, the 8-bit output layer and its softmax. Default workload: 5 LSTM layers of 500 cells,
+40-dimensional input frames, 2000-class 8-bit softmax layer, batch 1, T = 300 frames.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl reference]
+
+N > 1 runs under torchrun: every rank runs its own replica on its own batch (the sequences are
+independent; there is no collective on the data path), and the value is the frames of all ranks
+divided by the slowest rank's time. `--impl reference` times the CPU oracle instead, on a bounded
+sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_1607_04683_gb300 import inputs  # noqa: E402
+
+METRIC = "quantized LSTM frames/sec at batch B; int8 GEMM TOPS as % of GB300 int8 peak"
+DEFAULT_WORKLOAD = inputs.LSTM_5x500_B1.name
+L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(inputs.LSTM_WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_info():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+# ---------------------------------------------------------------------------------------------
+# algorithmic bytes of the dominant kernel (the persistent recurrent kernel), per launch
+# ---------------------------------------------------------------------------------------------
+
+def recurrent_bytes_per_launch(wl: inputs.LstmWorkload) -> int:
+    """One launch runs the T recurrent steps of one layer over B sequences. Unique HBM bytes it
+    must move: the layer's recurrent weight codes once (4H x R, plus P x H for a projection), and
+    per frame of each sequence the recovered input product row (4H fp32) read, the previous
+    output row (R fp32) read and the new output row (R fp32) written."""
+    H, R, P = wl.hidden, wl.R, wl.proj
+    weights = 4 * H * R + (P * H if P > 0 else 0)
+    per_frame = 4 * H * 4 + 2 * R * 4
+    return weights + wl.batch * wl.frames * per_frame
+
+
+def traffic_record(kernel: str, workload: str):
+    """Per-launch DRAM bytes from the committed ncu summary, if taken on the current source."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    src = os.path.join(ROOT, "paper_1607_04683_gb300", "csrc", "lstm.cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        for line in open(path):
+            f = line.split()
+            if len(f) >= 4 and not line.startswith("#") and f[0] == kernel and f[1] == workload and f[3] == sha:
+                return float(f[2])
+    except OSError:
+        pass
+    return None
+
+
+# ---------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+        return False
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------------------
+# CPU oracle timing (reference arm and cpu_baseline)
+# ---------------------------------------------------------------------------------------------
+
+def oracle_frames_per_s(wl, params, x, min_seconds=8.0, max_frames=None, reps_max=5):
+    import oracle
+    d = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    xs = x[:1, : (max_frames or x.shape[1])]
+    frames, t0 = 0, time.perf_counter()
+    for _ in range(reps_max):
+        oracle.lstm_forward(d, params, xs)
+        frames += xs.shape[0] * xs.shape[1]
+        if time.perf_counter() - t0 >= min_seconds:
+            break
+    dt = time.perf_counter() - t0
+    return frames / dt, frames, dt
+
+
+def run_reference(args, wl, rank, world):
+    if rank != 0:
+        return 0
+    params, x = wl.make(batch=1)
+    per_frame_ops = ops_per_frame(wl)
+    # a step: the oracle on the first sequence's first frames, bounded to ~1-3 s
+    sample_frames = max(1, min(wl.frames, int(2.0e9 / max(per_frame_ops, 1))))
+    import oracle
+    d = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    xs = x[:1, :sample_frames]
+    for _ in range(args.warmup):
+        oracle.lstm_forward(d, params, xs)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.lstm_forward(d, params, xs)
+    dt = time.perf_counter() - t0
+    fps = args.steps * sample_frames / dt
+    sample = f"sequence 0, first {sample_frames} frames of {wl.frames}, per step"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": fps, "unit": "frames/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u8", "data": "synthetic",
+        "config": workload_config(wl),
+        "cpu_baseline": {"value": fps, "unit": "frames/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": fps, "unit": "frames/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def ops_per_frame(wl) -> int:
+    """Integer multiply-adds x 2 per frame: every layer's input and recurrent products, the
+    projection, and the output layer."""
+    H, R, P = wl.hidden, wl.R, wl.proj
+    ops = 0
+    for l in range(wl.num_layers):
+        ops += 2 * 4 * H * (wl.layer_in(l) + R) + (2 * P * H if P > 0 else 0)
+    if wl.num_classes > 0:
+        ops += 2 * wl.num_classes * R
+    return ops
+
+
+def workload_config(wl):
+    return {"workload": wl.name, "batch": wl.batch, "frames": wl.frames, "layers": wl.num_layers,
+            "cells": wl.hidden, "proj": wl.proj, "input_dim": wl.input_dim, "classes": wl.num_classes,
+            "output_layer": "8-bit" if wl.output_mode == 1 else ("float" if wl.output_mode == 2 else "none"),
+            "activation_units": "per frame row", "weight_units": "per gate matrix",
+            "l2": "flushed between timed steps (512 MiB write)"}
+
+
+# ---------------------------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------------------------
+
+def run_ours(args, wl, rank, world, local):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_1607_04683_gb300 import build as qbuild, qnn
+
+    if not qbuild.up_to_date():
+        if rank == 0:
+            qbuild.build()
+        if world > 1:
+            dist.barrier()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    params, x = wl.make()
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, torch.from_numpy(params).to(dev))
+    xd = torch.from_numpy(x).to(dev)
+    ycols = wl.num_classes if wl.num_classes > 0 else wl.R
+    yd = torch.empty((wl.batch, wl.frames, ycols), dtype=torch.float32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        model.forward(xd, y=yd)
+    torch.cuda.synchronize()
+    st = qnn.device_status()
+    if st != qnn.QNN_OK:
+        raise RuntimeError(f"device status after warm-up: {st}")
+
+    # ---- timed region: device-resident inputs ----
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    qnn.profile_read()
+    qnn.profile_enable(True)
+    with ClockSampler(local) as clk:
+        barrier()
+        torch.cuda.synchronize()
+        for i in range(args.steps):
+            flush.zero_()
+            evs[i][0].record(stream)
+            model.forward(xd, y=yd)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        barrier()
+    qnn.profile_enable(False)
+    prof = qnn.profile_read()
+    step_ms = [a.elapsed_time(b) for a, b in evs]
+    total_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    frames_per_step = wl.batch * wl.frames
+    value = world * frames_per_step * args.steps / (total_ms / 1e3)
+
+    # ---- end to end: pinned host buffers through the C ABI, copies inside the timed region ----
+    x_host = torch.from_numpy(x).pin_memory()
+    y_host = torch.empty((wl.batch, wl.frames, ycols), dtype=torch.float32).pin_memory()
+    for _ in range(2):
+        model.forward(x_host, y=y_host)
+    torch.cuda.synchronize()
+    e2e_ms = 0.0
+    barrier()
+    for i in range(args.steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        model.forward(x_host, y=y_host)
+        b.record(stream)
+        b.synchronize()
+        e2e_ms += a.elapsed_time(b)
+    barrier()
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = world * frames_per_step * args.steps / (e2e_ms / 1e3)
+    ok = qnn.device_status() == qnn.QNN_OK
+    if not ok:
+        raise RuntimeError("device status reported an error during the timed steps")
+
+    if rank != 0:
+        return 0
+
+    peaks, peak_kind = measured_peaks()
+    kname = max(prof, key=lambda k: prof[k][1])
+    launches, kms = prof[kname]
+    avg_s = kms / launches / 1e3
+    if kname == "lstm_recurrent":
+        alg = recurrent_bytes_per_launch(wl)
+    else:
+        alg = None
+    roofline = None
+    if alg is not None:
+        ach = alg / avg_s / 1e9
+        roofline = {"bound": "hbm", "kernel": kname, "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                    "frac": ach / peaks["hbm_gbs"], "peak_kind": peak_kind,
+                    "traffic": traffic_record(kname, wl.name), "alg_bytes_per_launch": alg,
+                    "avg_launch_ms": avg_s * 1e3, "share_of_step": kms / total_ms if world == 1 else None}
+    line = {
+        "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u8", "data": "synthetic", "config": workload_config(wl),
+        "gpu_launches": sum(v[0] for v in prof.values()),
+        "kernels": {k: {"launches": v[0], "ms": v[1]} for k, v in sorted(prof.items(), key=lambda kv: -kv[1][1])},
+        "int8_tops": ops_per_frame(wl) * frames_per_step * args.steps / (total_ms / 1e3) / 1e12,
+        "roofline": roofline,
+        "e2e": {"value": e2e_value, "unit": "frames/s", "h2d_bytes_per_step": int(x.nbytes),
+                "d2h_bytes_per_step": int(wl.batch * wl.frames * ycols * 4)},
+        "clocks": clk.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        fps, frames, dt = oracle_frames_per_s(wl, params, x, min_seconds=8.0,
+                                              max_frames=max(1, min(wl.frames, int(3.0e9 / ops_per_frame(wl)))))
+        line["cpu_baseline"] = {"value": fps, "unit": "frames/s", "cores": 1, "kind": "oracle",
+                                "sample": f"sequence 0 frames 0..{min(wl.frames, max(1, int(3.0e9 / ops_per_frame(wl))))}"
+                                          f", repeated: {frames} frames in {dt:.1f} s, single thread"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    args = parse()
+    rank, world, local = dist_info()
+    wl = inputs.LSTM_WORKLOADS[args.workload]
+    if world > 1 and args.impl == "ours":
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    try:
+        if args.impl == "reference":
+            return run_reference(args, wl, rank, world)
+        return run_ours(args, wl, rank, world, local)
+    finally:
+        if world > 1 and args.impl == "ours":
+            import torch.distributed as dist
+            if dist.is_initialized():
+                dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

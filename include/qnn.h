@@ -1,0 +1,182 @@
+/*
+ * qnn.h — C ABI of libqnn: 8-bit quantized LSTM acoustic-model inference on one GB300 (sm_103a).
+ *
+ * The method is the one of Alvarez, Prabhavalkar and Bakhtin, "On the efficient representation
+ * and execution of deep acoustic models" (INTERSPEECH 2016):
+ *   - a uniform linear quantizer to 8 bits, S = 255, Q = S / (Vmax - Vmin), with the offset
+ *     rounded consistently: V' = round(Q V) - round(Q Vmin)          (Sec. 3, eq. 2);
+ *   - products of independently quantized matrices in 8-bit integers with 32-bit accumulators,
+ *     recovered as (V_a'' V_b'') / (Q_a Q_b), V'' = V' + round(Q Vmin)  (Sec. 3.1, eq. 1, eq. 3);
+ *   - layers that take fp32 in and give fp32 out: inputs quantized on the fly, weights offline,
+ *     recovered products plus bias through the activation function (Sec. 3.1, Fig. 1);
+ *   - one quantization unit per weight matrix, e.g. per LSTM gate (Sec. 3.1, last paragraph).
+ *
+ * Conventions for every call:
+ *   - Matrices are row-major with an explicit leading dimension in elements.
+ *   - Unless a call says otherwise, pointers are DEVICE pointers on the current CUDA device, and
+ *     the caller owns them. A host pointer where a device pointer is required is rejected with
+ *     QNN_ERR_INVALID_ARG.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream). Calls are asynchronous on it:
+ *     argument errors are returned at once; errors found by the GPU (non-finite inputs, a
+ *     persistent-kernel wait that timed out) are recorded in a device status word and returned
+ *     by qnn_device_status().
+ *   - There is no CPU fallback: without a usable CUDA device every compute call returns
+ *     QNN_ERR_CUDA.
+ */
+#ifndef QNN_H
+#define QNN_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    QNN_OK = 0,
+    QNN_ERR_INVALID_ARG = 1,  /* bad size, stride, pointer kind or enum value */
+    QNN_ERR_NONFINITE = 2,    /* a quantization unit held NaN or +-Inf (no range exists, Sec. 3) */
+    QNN_ERR_K_TOO_LARGE = 3,  /* K > 33025: K * 255^2 would overflow the 32-bit accumulator */
+    QNN_ERR_CUDA = 4,         /* a CUDA runtime call failed, or no device */
+    QNN_ERR_TIMEOUT = 5,      /* a grid-wide wait in a persistent kernel gave up (bounded spin) */
+    QNN_ERR_NO_COOP = 6,      /* the persistent grid cannot be co-resident on this device */
+    QNN_ERR_NO_MEMORY = 7,    /* device allocation failed */
+} qnn_status;
+
+typedef enum { QNN_PER_MATRIX = 0, QNN_PER_ROW = 1 } qnn_granularity;
+
+/* Output layer of an LSTM model: none (the top layer's outputs are returned), 8-bit
+ * ("quant-all" of Sec. 5), or float ("quant" of Sec. 5: all layers but the softmax quantized). */
+typedef enum { QNN_OUT_NONE = 0, QNN_OUT_QUANT = 1, QNN_OUT_FLOAT = 2 } qnn_output_mode;
+
+/* Largest reduction length for which 8-bit codes cannot overflow a 32-bit accumulator:
+ * K * 255 * 255 <= 2^31 - 1. */
+#define QNN_K_MAX 33025
+
+/* Quantization parameters of one unit (16 bytes). vmin/vmax: the exact fp32 range of the unit;
+ * Q: the fp32 scale S / (vmax - vmin), S = 255 (Sec. 3); z: round(Q vmin), the rounded offset of
+ * eq. (2). Code of v: clamp(round(Q v) - z, 0, 255). Recovery (eq. 3): (code + z) / Q.
+ * Readings where the paper is silent: Q is raised by single ulps until the range maximum reaches
+ * code 255; codes are clamped to [0, 255]; a unit with vmax == vmin, or with |Q vmin| or
+ * |Q vmax| >= 2^22, uses Q = 255 / max(|vmin|, |vmax|) (Q = 1 if all values are 0). */
+typedef struct {
+    float vmin;
+    float vmax;
+    float Q;
+    int32_t z;
+} qnn_qparams;
+
+/* Human-readable name of a status code (static string). */
+const char *qnn_status_string(qnn_status s);
+
+/* Waits for `stream`, then returns and clears the device status word of the current device:
+ * QNN_OK, QNN_ERR_NONFINITE or QNN_ERR_TIMEOUT (the first error recorded since the last call), or
+ * QNN_ERR_CUDA if the stream itself failed. */
+qnn_status qnn_device_status(void *stream);
+
+/*
+ * qnn_quantize — Sec. 3 "Quantizing" and eq. (2): fp32 -> 8-bit codes, on the fly.
+ *   x          [rows x cols] fp32, leading dimension ldx >= cols.
+ *   granularity QNN_PER_MATRIX: one unit for the whole matrix (one params entry);
+ *              QNN_PER_ROW: one unit per row (rows params entries).
+ *   codes      [rows x cols] uint8 out, leading dimension ldc >= cols.
+ *   params     out: 1 or `rows` entries.
+ *   code_sums  out, nullable: [rows] int32, sum of each row's codes (used by the offset terms of
+ *              eq. 1).
+ * Non-finite values: the unit's codes are unspecified and QNN_ERR_NONFINITE is recorded.
+ * Per-matrix quantization allocates a small library-owned scratch buffer on first use.
+ */
+qnn_status qnn_quantize(const float *x, int64_t rows, int64_t cols, int64_t ldx, int granularity,
+                        uint8_t *codes, int64_t ldc, qnn_qparams *params, int32_t *code_sums, void *stream);
+
+/*
+ * qnn_qmatmul — eq. (1) with eq. (2)'s offsets, recovered to fp32 (Fig. 1: y = R(Mult(Q(X), W')) + B).
+ *   A     [M x K] uint8 activation codes (lda >= K); pa: 1 (ga = QNN_PER_MATRIX) or M
+ *         (ga = QNN_PER_ROW) params; rsA [M] int32 row code sums of A.
+ *   W     [N x K] uint8 weight codes (ldw >= K): the rows split into n_blocks equal blocks
+ *         (N % n_blocks == 0), block b quantized with pw[b] (e.g. one block per LSTM gate);
+ *         csW [N] int32 row code sums of W.
+ *   bias  [N] fp32, nullable.
+ *   Y     [M x N] fp32 out (ldy >= N): Y[m,n] = S / (Qa Qw) + bias[n], with the exact integer
+ *         S = sum_k (A[m,k] + za)(W[n,k] + zw) = acc + zw*rsA[m] + za*csW[n] + K*za*zw and
+ *         the fp32 operations (float)S, Qa*Qw, divide, add, each rounded once.
+ *   acc_out [M x N] int32 out, nullable: acc[m,n] = sum_k A[m,k] W[n,k] (the 32-bit accumulator).
+ * 1 <= K <= QNN_K_MAX.
+ */
+qnn_status qnn_qmatmul(const uint8_t *A, int64_t lda, const qnn_qparams *pa, int ga, const int32_t *rsA,
+                       int64_t M, int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw,
+                       int64_t n_blocks, const int32_t *csW, int64_t N, const float *bias, float *Y,
+                       int64_t ldy, int32_t *acc_out, void *stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * Quantized LSTM / LSTMP stack (Sec. 4 model family) with an optional softmax output layer.
+ * ------------------------------------------------------------------------------------------- */
+
+typedef struct {
+    int32_t num_layers;  /* L >= 1 */
+    int32_t input_dim;   /* I, features per frame */
+    int32_t hidden;      /* H, LSTM cells per layer */
+    int32_t proj;        /* P, recurrent projection units after each layer; 0 = none */
+    int32_t num_classes; /* C, softmax outputs; 0 = no output layer */
+    int32_t output_mode; /* qnn_output_mode; must be QNN_OUT_NONE iff num_classes == 0 */
+} qnn_lstm_desc;
+
+typedef struct qnn_lstm_model qnn_lstm_model;
+
+/* Number of fp32 values in the packed parameter buffer. Layout, layer by layer, with
+ * Ik = I for the first layer and R = (P > 0 ? P : H) otherwise, gates in the order [i, f, g, o]:
+ *   Wx[4][H][Ik], Wh[4][H][R], b[4][H], then Wp[P][H] if P > 0;
+ * after the last layer, if C > 0: Wo[C][R], bo[C]. Returns -1 on an invalid descriptor. */
+int64_t qnn_lstm_param_count(const qnn_lstm_desc *d);
+
+/* Quantizes the weights offline (Sec. 3.1: one unit per gate matrix, per projection and per
+ * output matrix) and keeps device copies in the model. `params` (host or device) is read during
+ * the call only. The call is synchronous. *out receives the model (destroy with
+ * qnn_lstm_model_destroy). */
+qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float *params, qnn_lstm_model **out);
+
+void qnn_lstm_model_destroy(qnn_lstm_model *m);
+
+/* Copies the model's weight codes (host buffer, qnn_lstm_param_count bytes; the packed layout
+ * with every bias slot zero) and the parameters of each unit in order (4 Wx, 4 Wh, Wp per layer,
+ * then Wo; host buffer of at least 9 L + 1 entries) and their count. Synchronous. */
+qnn_status qnn_lstm_model_weights(const qnn_lstm_model *m, uint8_t *codes_host, qnn_qparams *params_host,
+                                  int64_t *n_units);
+
+/*
+ * qnn_lstm_forward — inference over B independent sequences of T frames.
+ *   x        [B][T][I] fp32 frames.
+ *   y        [B][T][C] softmax outputs if the model has an output layer, else [B][T][R] top-layer
+ *            outputs.
+ *   h_state  [L][B][R], c_state [L][B][H], nullable: initial state in, final state out (a
+ *            stream can therefore be processed in chunks); NULL means a zero initial state and
+ *            the final state is not returned.
+ *   h_all    [L][B][T][R], nullable: every layer's output at every frame (diagnostics).
+ * x, y, h_state, c_state and h_all may each be host or device memory: host buffers are copied
+ * to or from device memory on `stream` inside the call (pinned host memory keeps the copies
+ * asynchronous). Activations are quantized per row (one frame of one sequence), weights per
+ * gate matrix. The model keeps a device workspace sized for the largest B*T seen; calls on one
+ * model must not overlap in time.
+ */
+qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
+                            float *c_state, float *h_all, void *stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * Kernel timing (diagnostics and benchmarks; no counterpart in the paper).
+ * ------------------------------------------------------------------------------------------- */
+
+/* While enabled, every kernel launch the library makes is bracketed by two CUDA events on the
+ * launching stream (process-wide switch, off by default). */
+qnn_status qnn_profile_enable(int on);
+
+/* Waits for the recorded events, then returns per kernel name (static strings) the number of
+ * launches and their summed device time in milliseconds since the last read, and resets the
+ * totals. Up to `capacity` entries are written to the (nullable) host arrays; *count receives
+ * the number of distinct kernels. */
+qnn_status qnn_profile_read(int capacity, const char **names, double *total_ms, int64_t *launches, int *count);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QNN_H */

@@ -221,7 +221,7 @@ def lstm_quantize_weights(d: LstmDesc, params: np.ndarray):
     """Offline weight codes in packed order (u8) and one params entry per unit."""
     params = np.ascontiguousarray(params, np.float32)
     n = lstm_param_count(d)
-    codes = np.empty(n, np.uint8)
+    codes = np.zeros(n, np.uint8)
     qp = np.zeros(9 * d.num_layers + 1, QPARAMS_DTYPE)
     nu = C.c_int64(0)
     _check(lib().orc_lstm_quantize_weights(C.byref(d), _ptr(params), _ptr(codes), _ptr(qp), C.byref(nu)))

@@ -477,8 +477,9 @@ int orc_lstm_forward(const orc_lstm_desc *d, const float *params, const float *x
     return st;
 }
 
-/* Weight quantization alone (step a1), for parity of the offline codes: writes every unit's
- * codes in the packed order of the parameters (gate matrices, Wp, Wo) and their parameters. */
+/* Weight quantization alone (offline step), for parity of the offline codes: writes every unit's
+ * codes at the offsets of the packed parameter layout (bias slots untouched) and the parameters
+ * of each unit in order (4 Wx, 4 Wh, Wp per layer, then Wo). */
 int orc_lstm_quantize_weights(const orc_lstm_desc *d, const float *params, uint8_t *codes, orc_qparams *qp,
                               int64_t *n_units)
 {
@@ -499,6 +500,7 @@ int orc_lstm_quantize_weights(const orc_lstm_desc *d, const float *params, uint8
             off += H * R;
         }
         q += 4 * H * R + 4 * H;
+        off += 4 * H; /* bias slot: no codes */
         if (P > 0 && !st) {
             st = orc_quantize(q, P, H, H, ORC_PER_MATRIX, codes + off, H, &qp[u], NULL);
             ++u;

@@ -1,0 +1,125 @@
+// qnn_device.cuh — device arithmetic shared by the libqnn kernels: the quantizer's parameter
+// rule (Sec. 3, eq. 2), code and recovery (eq. 2, eq. 3), the recovered offset-applied product
+// (eq. 1), the pinned fp32 exponential and the LSTM gate functions.
+//
+// Every fp32 operation that can decide a code is written with an explicit round-to-nearest
+// intrinsic (__fmul_rn, __fadd_rn, __fdiv_rn, __fmaf_rn) so that the compiler can neither fuse
+// nor reorder it: the same inputs give the same bits on every run and every launch shape.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/qnn.h"
+
+namespace qnn {
+
+constexpr float kScale = 255.0f;          // S for 8 bits (Sec. 3)
+constexpr float kDegenerateLim = 4194304.0f;  // 2^22: |Q v| beyond this leaves no fractional bit
+
+// Device status word (library-owned, one per device): keeps the first error a kernel finds
+// (QNN_ERR_NONFINITE, QNN_ERR_TIMEOUT) until qnn_device_status() reads and clears it.
+__device__ __forceinline__ void record_status(int *status, int st) { atomicCAS(status, 0, st); }
+
+// Sec. 3: Q = S / (vmax - vmin); eq. (2): z = round(Q vmin). Q is raised one ulp at a time until
+// round(Q vmax) - z reaches S, so the range maximum gets the top code. Degenerate units (no
+// range, or a range so narrow that Q v has no fractional bits left) use Q = S / max|v|.
+__device__ __forceinline__ qnn_qparams params_from_range(float vmin, float vmax) {
+    qnn_qparams p;
+    p.vmin = vmin;
+    p.vmax = vmax;
+    float R = __fsub_rn(vmax, vmin);
+    float Q = (R > 0.0f) ? __fdiv_rn(kScale, R) : 0.0f;
+    bool degenerate = !(R > 0.0f) || !isfinite(Q) || !(fabsf(__fmul_rn(Q, vmin)) < kDegenerateLim) ||
+                      !(fabsf(__fmul_rn(Q, vmax)) < kDegenerateLim);
+    if (degenerate) {
+        float amax = fmaxf(fabsf(vmin), fabsf(vmax));
+        Q = (amax > 0.0f) ? __fdiv_rn(kScale, amax) : 1.0f;
+        p.Q = Q;
+        p.z = __float2int_rn(__fmul_rn(Q, vmin));
+        return p;
+    }
+    int z = __float2int_rn(__fmul_rn(Q, vmin));
+    for (int it = 0; it < 64; ++it) {
+        int top = __float2int_rn(__fmul_rn(Q, vmax)) - z;
+        if (top >= 255) break;
+        Q = __int_as_float(__float_as_int(Q) + 1);
+        z = __float2int_rn(__fmul_rn(Q, vmin));
+    }
+    p.Q = Q;
+    p.z = z;
+    return p;
+}
+
+// Eq. (2): code = clamp(round(Q v) - round(Q vmin), 0, S).
+__device__ __forceinline__ uint32_t quant_code(float v, float Q, int z) {
+    int c = __float2int_rn(__fmul_rn(Q, v)) - z;
+    c = c < 0 ? 0 : c;
+    c = c > 255 ? 255 : c;
+    return (uint32_t)c;
+}
+
+// Eq. (1) recovery of the exact offset-applied product S: S / (Qa Qw), each op rounded once.
+__device__ __forceinline__ float recover_product(long long S, float Qa, float Qw) {
+    return __fdiv_rn(__ll2float_rn(S), __fmul_rn(Qa, Qw));
+}
+
+// S = acc + zw*rsA + za*csW + K*za*zw: eq. (1)'s sum of (a' + za)(w' + zw) expanded so that the
+// inner loop multiplies raw codes only.
+__device__ __forceinline__ long long offset_product(int acc, int za, int zw, int rsA, int csW, int K) {
+    return (long long)acc + (long long)zw * rsA + (long long)za * csW + (long long)K * za * zw;
+}
+
+// Pinned fp32 exponential: Cody-Waite reduction x = n ln2 + r (n = round(x log2 e), ln 2 split
+// into a 16-significant-bit head and its remainder), e^r by its degree-7 Taylor polynomial in
+// Horner form with fused multiply-adds, times 2^n assembled from exponent bits. x is clamped to
+// [-87, 88] so every result is a finite normal number.
+__device__ __forceinline__ float pexp(float x) {
+    x = x < -87.0f ? -87.0f : x;
+    x = x > 88.0f ? 88.0f : x;
+    float nf = rintf(__fmul_rn(x, 1.44269504088896341f));
+    int n = (int)nf;
+    float r = __fmaf_rn(-nf, 0.693145751953125f, x);
+    r = __fmaf_rn(-nf, 1.428606820309417232e-06f, r);
+    float p = 1.984126984126984127e-04f;
+    p = __fmaf_rn(p, r, 1.388888888888888889e-03f);
+    p = __fmaf_rn(p, r, 8.333333333333333333e-03f);
+    p = __fmaf_rn(p, r, 4.166666666666666667e-02f);
+    p = __fmaf_rn(p, r, 1.666666666666666667e-01f);
+    p = __fmaf_rn(p, r, 0.5f);
+    p = __fmaf_rn(p, r, 1.0f);
+    p = __fmaf_rn(p, r, 1.0f);
+    return __fmul_rn(p, __int_as_float((n + 127) << 23));
+}
+
+__device__ __forceinline__ float psigmoid(float x) { return __fdiv_rn(1.0f, __fadd_rn(1.0f, pexp(-x))); }
+
+__device__ __forceinline__ float ptanh(float x) {
+    return __fsub_rn(1.0f, __fdiv_rn(2.0f, __fadd_rn(pexp(__fmul_rn(2.0f, x)), 1.0f)));
+}
+
+// LSTM cell (no peepholes, gates [i, f, g, o]): c' = f c + i g; m = o tanh(c').
+__device__ __forceinline__ void lstm_cell(float pi, float pf, float pg, float po, float &c, float &m) {
+    float ig = psigmoid(pi), fg = psigmoid(pf), gg = ptanh(pg), og = psigmoid(po);
+    c = __fadd_rn(__fmul_rn(fg, c), __fmul_rn(ig, gg));
+    m = __fmul_rn(og, ptanh(c));
+}
+
+// Warp-wide reductions.
+__device__ __forceinline__ float warp_min(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ int warp_sum(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+}  // namespace qnn

@@ -1,0 +1,63 @@
+"""CPU-side checks of the boundary: the library builds for sm_103a, loads without a GPU and exports
+every symbol include/qnn.h declares; host-side argument checks that never reach a kernel."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def qlib():
+    from paper_1607_04683_gb300 import build, qnn
+    build.build()
+    return qnn.lib()
+
+
+def declared_functions():
+    hdr = open(os.path.join(ROOT, "include", "qnn.h")).read()
+    hdr = re.sub(r"/\*.*?\*/", "", hdr, flags=re.S)
+    return sorted(set(re.findall(r"\b(qnn_[a-z0-9_]+)\s*\(", hdr)))
+
+
+def test_every_declared_symbol_is_exported(qlib):
+    from paper_1607_04683_gb300 import qnn
+    names = declared_functions()
+    assert names, "no declarations found"
+    for n in names:
+        assert hasattr(qlib, n), n
+    assert sorted(qnn.EXPORTS) == names
+
+
+def test_status_strings(qlib):
+    for s in range(8):
+        assert qlib.qnn_status_string(s).decode().startswith("QNN_")
+
+
+def test_param_count_matches_oracle_layout(qlib):
+    import oracle
+    from paper_1607_04683_gb300 import inputs, qnn
+    for wl in inputs.LSTM_WORKLOADS.values():
+        d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes)
+        od = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes)
+        assert qnn.qnn_lstm_param_count(d) == oracle.lstm_param_count(od) == wl.param_count()
+    bad = qnn.lstm_desc(0, 4, 4)
+    assert qnn.qnn_lstm_param_count(bad) == -1
+    bad = qnn.LstmDesc(1, 4, 4, 0, 5, qnn.OUT_NONE)  # classes without an output layer mode
+    assert qnn.qnn_lstm_param_count(bad) == -1
+
+
+def test_argument_errors_need_no_gpu(qlib):
+    from paper_1607_04683_gb300 import qnn
+    # invalid sizes are rejected before any pointer or device is touched
+    assert qlib.qnn_quantize(None, 4, 0, 4, 0, None, 4, None, None, None) == qnn.QNN_ERR_INVALID_ARG
+    assert qlib.qnn_quantize(None, 4, 8, 4, 0, None, 8, None, None, None) == qnn.QNN_ERR_INVALID_ARG
+    assert qlib.qnn_quantize(None, 4, 8, 8, 7, None, 8, None, None, None) == qnn.QNN_ERR_INVALID_ARG
+    assert qlib.qnn_qmatmul(None, 40000, None, 0, None, 1, 40000, None, 40000, None, 1, None, 1, None, None, 1, None,
+                            None) == qnn.QNN_ERR_K_TOO_LARGE
+    assert qlib.qnn_qmatmul(None, 8, None, 0, None, 1, 8, None, 8, None, 3, None, 4, None, None, 4, None,
+                            None) == qnn.QNN_ERR_INVALID_ARG
+    h = C.c_void_p()
+    assert qlib.qnn_lstm_model_create(C.byref(qnn.lstm_desc(0, 1, 1)), None, C.byref(h)) == qnn.QNN_ERR_INVALID_ARG

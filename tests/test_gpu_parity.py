@@ -1,0 +1,328 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the same seeded inputs.
+
+Bar: codes, parameters, code sums and int32 accumulators bit-exact; every LSTM layer output
+bit-exact (the whole recurrence is the same sequence of fp32 operations on both sides, so any
+difference would be a bug); softmax outputs within 1e-4 absolute (their sums run in a different
+order on the GPU).
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_1607_04683_gb300 import inputs
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+SOFTMAX_TOL = 1e-4
+
+
+@pytest.fixture(scope="module")
+def qnn():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_1607_04683_gb300 import build, qnn as q
+    build.build()
+    q.lib()
+    torch.cuda.set_device(0)
+    assert q.device_status() == q.QNN_OK
+    return q
+
+
+def gpu(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def rng(seed):
+    return np.random.Generator(np.random.PCG64(seed))
+
+
+# ------------------------------------------------------------------------------------------
+# qnn_quantize
+# ------------------------------------------------------------------------------------------
+
+QUANT_SHAPES = [(1, 1), (1, 3), (3, 5), (7, 40), (9, 128), (33, 500), (300, 40), (17, 1000), (5, 8192), (1025, 77)]
+
+
+@pytest.mark.parametrize("rows,cols", QUANT_SHAPES)
+@pytest.mark.parametrize("gran", [0, 1])
+def test_quantize_bit_exact(qnn, rows, cols, gran):
+    r = rng(rows * 1000 + cols)
+    x = (r.normal(0.3, 1.7, (rows, cols)) * r.uniform(0.01, 10, (rows, 1))).astype(np.float32)
+    codes, params, sums = qnn.qnn_quantize(gpu(x), gran)
+    assert qnn.device_status() == qnn.QNN_OK
+    c_ref, p_ref, s_ref = oracle.quantize(x, gran)
+    assert np.array_equal(codes.cpu().numpy(), c_ref)
+    assert np.array_equal(sums.cpu().numpy(), s_ref)
+    p = qnn.params_view(params)
+    for f in ("vmin", "vmax", "Q", "z"):
+        assert np.array_equal(p[f], p_ref[f]), f
+
+
+def test_quantize_strided_and_degenerate_rows(qnn):
+    r = rng(5)
+    big = r.normal(0, 1, (64, 203)).astype(np.float32)
+    big[3] = 0.0
+    big[7] = -2.5
+    big[11, :] = 1e-3
+    big[11, 5] = np.nextafter(np.float32(1e-3), np.float32(1))
+    view = gpu(big)[:, 3:190]  # row stride 203, unaligned start
+    codes, params, sums = qnn.qnn_quantize(view, qnn.PER_ROW)
+    c_ref, p_ref, s_ref = oracle.quantize(np.ascontiguousarray(big[:, 3:190]), oracle.PER_ROW)
+    assert np.array_equal(codes.cpu().numpy(), c_ref)
+    assert np.array_equal(sums.cpu().numpy(), s_ref)
+    p = qnn.params_view(params)
+    for f in ("vmin", "vmax", "Q", "z"):
+        assert np.array_equal(p[f], p_ref[f]), f
+
+
+def test_quantize_large_matrix_per_matrix(qnn):
+    # config-4 size activation: 16384 x 8192, per-matrix unit; codes checked on sampled rows.
+    shape = inputs.QmatmulShape(16384, 8192, 8192)
+    W, A = inputs.make_qmatmul_operands(shape)
+    Ag = gpu(A)
+    codes, params, sums = qnn.qnn_quantize(Ag, qnn.PER_MATRIX)
+    p = qnn.params_view(params)[0]
+    assert p["vmin"] == A.min() and p["vmax"] == A.max()
+    ref = oracle.params_from_range(float(A.min()), float(A.max()))
+    assert p["Q"] == np.float32(ref["Q"]) and p["z"] == ref["z"]
+    rows = rng(1).choice(shape.M, 64, replace=False)
+    cs = codes[torch.from_numpy(rows).cuda()].cpu().numpy()
+    for i, row in enumerate(rows):
+        exp = np.array([oracle.code(float(v), ref) for v in A[row, ::97]], np.uint8)
+        assert np.array_equal(cs[i, ::97], exp)
+        assert sums[int(row)].item() == int(cs[i].astype(np.int64).sum())
+
+
+def test_quantize_nonfinite_reported(qnn):
+    x = np.ones((4, 33), np.float32)
+    x[2, 7] = np.nan
+    qnn.qnn_quantize(gpu(x), qnn.PER_ROW)
+    assert qnn.device_status() == qnn.QNN_ERR_NONFINITE
+    assert qnn.device_status() == qnn.QNN_OK  # cleared by the read
+    x[2, 7] = np.inf
+    qnn.qnn_quantize(gpu(x), qnn.PER_MATRIX)
+    assert qnn.device_status() == qnn.QNN_ERR_NONFINITE
+
+
+def test_quantize_rejects_host_pointers(qnn):
+    import ctypes as C
+    x = np.ones((2, 8), np.float32)
+    codes = np.zeros((2, 8), np.uint8)
+    prm = np.zeros(2, qnn.QPARAMS_DTYPE)
+    st = qnn.lib().qnn_quantize(x.ctypes.data_as(C.c_void_p), 2, 8, 8, 1, codes.ctypes.data_as(C.c_void_p), 8,
+                                prm.ctypes.data_as(C.c_void_p), None, None)
+    assert st == qnn.QNN_ERR_INVALID_ARG
+
+
+# ------------------------------------------------------------------------------------------
+# qnn_qmatmul
+# ------------------------------------------------------------------------------------------
+
+def _operands(M, N, K, ga, seed, n_blocks=1):
+    r = rng(seed)
+    A = r.normal(0.2, 1.0, (M, K)).astype(np.float32)
+    Wf = [r.uniform(-s, s, (N // n_blocks, K)).astype(np.float32) for s in np.linspace(0.05, 0.5, n_blocks)]
+    ca, pa, ra = oracle.quantize(A, ga)
+    parts = [oracle.quantize(w, oracle.PER_MATRIX) for w in Wf]
+    cw = np.concatenate([p[0] for p in parts])
+    pw = np.concatenate([p[1] for p in parts])
+    cs = np.concatenate([p[2] for p in parts])
+    bias = r.normal(0, 1, N).astype(np.float32)
+    return ca, pa, ra, cw, pw, cs, bias
+
+
+MM_SHAPES = [(1, 8, 1), (1, 4, 40), (3, 5, 7), (16, 64, 64), (130, 130, 100), (257, 260, 500), (300, 2000, 40),
+             (64, 96, 1000), (200, 136, 2048)]
+
+
+@pytest.mark.parametrize("M,N,K", MM_SHAPES)
+@pytest.mark.parametrize("ga", [0, 1])
+def test_qmatmul_bit_exact(qnn, M, N, K, ga):
+    nb = 4 if N % 4 == 0 else 1
+    ca, pa, ra, cw, pw, cs, bias = _operands(M, N, K, ga, M * 7 + N * 3 + K, nb)
+    Y, acc = qnn.qnn_qmatmul(gpu(ca), qnn.params_tensor(pa), ga, gpu(ra), gpu(cw), qnn.params_tensor(pw), gpu(cs),
+                             n_blocks=nb, bias=gpu(bias), want_acc=True)
+    ref = oracle.qmatmul(ca, pa, ga, cw, pw, n_blocks=nb, bias=bias)
+    assert np.array_equal(acc.cpu().numpy(), ref["acc"])
+    assert np.array_equal(Y.cpu().numpy(), ref["y"])
+
+
+def test_qmatmul_unaligned_leading_dims(qnn):
+    M, N, K = 37, 45, 99
+    ca, pa, ra, cw, pw, cs, _ = _operands(M, N, K, 1, 11)
+    Abig = np.zeros((M, K + 5), np.uint8)
+    Abig[:, 2:2 + K] = ca
+    Ag = gpu(Abig)[:, 2:2 + K]
+    Y, acc = qnn.qnn_qmatmul(Ag, qnn.params_tensor(pa), 1, gpu(ra), gpu(cw), qnn.params_tensor(pw), gpu(cs),
+                             want_acc=True)
+    ref = oracle.qmatmul(ca, pa, 1, cw, pw)
+    assert np.array_equal(acc.cpu().numpy(), ref["acc"]) and np.array_equal(Y.cpu().numpy(), ref["y"])
+
+
+def test_qmatmul_k_max_all_255(qnn):
+    K = oracle.K_MAX
+    a = np.full((2, K), 255, np.uint8)
+    p = np.zeros(1, qnn.QPARAMS_DTYPE)
+    p[0] = (0.0, 1.0, 255.0, 0)
+    rs = np.full(2, 255 * K, np.int32)
+    Y, acc = qnn.qnn_qmatmul(gpu(a), qnn.params_tensor(p), 0, gpu(rs), gpu(a), qnn.params_tensor(p), gpu(rs),
+                             want_acc=True)
+    assert int(acc[0, 0].item()) == K * 65025 == 2147450625
+    with pytest.raises(qnn.QnnError) as e:
+        b = np.full((1, K + 1), 1, np.uint8)
+        qnn.qnn_qmatmul(gpu(b), qnn.params_tensor(p), 0, gpu(rs[:1]), gpu(b), qnn.params_tensor(p), gpu(rs[:1]))
+    assert e.value.status == qnn.QNN_ERR_K_TOO_LARGE
+
+
+@pytest.mark.parametrize("KN", [512, 2048, 8192])
+def test_qmatmul_sweep_full_size_sampled(qnn, KN):
+    # The standalone sweep's largest M at each K = N, fp32 in: quantize both operands on the GPU
+    # (per matrix), product; compared on a sample of rows and columns the oracle computes.
+    shape = inputs.QmatmulShape(16384, KN, KN)
+    W, A = inputs.make_qmatmul_operands(shape)
+    ca, pa, ra = qnn.qnn_quantize(gpu(A), qnn.PER_MATRIX)
+    cw, pw, cs = qnn.qnn_quantize(gpu(W), qnn.PER_MATRIX)
+    Y, acc = qnn.qnn_qmatmul(ca, pa, 0, ra, cw, pw, cs, want_acc=True)
+    r = rng(KN)
+    rows = np.sort(r.choice(shape.M, 48, replace=False))
+    cols = np.sort(r.choice(shape.N, 48, replace=False))
+    c_a, p_a, _ = oracle.quantize(A, oracle.PER_MATRIX)
+    c_w, p_w, _ = oracle.quantize(W, oracle.PER_MATRIX)
+    assert np.array_equal(qnn.params_view(pa), p_a) and np.array_equal(qnn.params_view(pw), p_w)
+    ref = oracle.qmatmul(c_a[rows], p_a, 0, c_w[cols], p_w)
+    ri, ci = torch.from_numpy(rows).cuda(), torch.from_numpy(cols).cuda()
+    assert np.array_equal(acc[ri][:, ci].cpu().numpy(), ref["acc"])
+    assert np.array_equal(Y[ri][:, ci].cpu().numpy(), ref["y"])
+
+
+# ------------------------------------------------------------------------------------------
+# qnn_lstm_forward
+# ------------------------------------------------------------------------------------------
+
+def _small(name="t", L=2, I=7, H=9, P=0, C=0, B=2, T=6, seed=5, mode=None, fb=1.0, w=0.5, mu=0.0):
+    return inputs.LstmWorkload(name, seed=seed, num_layers=L, input_dim=I, hidden=H, proj=P, num_classes=C,
+                               batch=B, frames=T, w_range=w, forget_bias=fb, seq_mean_range=mu,
+                               output_mode=(mode if mode is not None else (1 if C > 0 else 0)))
+
+
+def _gpu_forward(qnn, wl, params, x, h_all=True, h0=None, c0=None):
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, gpu(params))
+    B, T, _ = x.shape
+    ha = torch.empty((wl.num_layers, B, T, wl.R), dtype=torch.float32, device="cuda") if h_all else None
+    hs = gpu(h0) if h0 is not None else torch.zeros((wl.num_layers, B, wl.R), dtype=torch.float32, device="cuda")
+    cs = gpu(c0) if c0 is not None else torch.zeros((wl.num_layers, B, wl.hidden), dtype=torch.float32, device="cuda")
+    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha)
+    assert qnn.device_status() == qnn.QNN_OK
+    out = {"y": y.cpu().numpy(), "h": hs.cpu().numpy(), "c": cs.cpu().numpy(), "model": model}
+    if h_all:
+        out["h_all"] = ha.cpu().numpy()
+    return out
+
+
+def _compare(got, ref, wl):
+    if "h_all" in got and "h_all" in ref:
+        for l in range(wl.num_layers):
+            assert np.array_equal(got["h_all"][l], ref["h_all"][l]), f"layer {l} outputs differ"
+    assert np.array_equal(got["h"], ref["h"]) and np.array_equal(got["c"], ref["c"])
+    if wl.num_classes > 0:
+        assert np.max(np.abs(got["y"] - ref["y"])) <= SOFTMAX_TOL
+    else:
+        assert np.array_equal(got["y"], ref["y"])
+
+
+def _oracle(wl, params, x, **kw):
+    d = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    return oracle.lstm_forward(d, params, x, **kw)
+
+
+SMALL_CASES = [dict(), dict(L=1, I=3, H=4, B=1, T=9), dict(L=3, H=16, C=11, B=3), dict(L=2, H=33, I=40, C=5, B=17, T=4),
+               dict(L=2, I=6, H=10, P=4, C=7, B=2, T=5), dict(L=2, I=80, H=130, P=48, C=70, B=20, T=6),
+               dict(L=2, H=12, C=5, mode=2), dict(L=1, I=40, H=500, B=70, T=3, C=2000, w=0.08),
+               dict(L=3, I=5, H=8, B=65, T=3, mu=0.5)]
+
+
+@pytest.mark.parametrize("cfg", SMALL_CASES)
+def test_lstm_small_bit_exact(qnn, cfg):
+    wl = _small(**cfg)
+    params, x = wl.make()
+    got = _gpu_forward(qnn, wl, params, x)
+    ref = _oracle(wl, params, x, want_h_all=True)
+    _compare(got, ref, wl)
+
+
+def test_lstm_weight_codes_bit_exact(qnn):
+    wl = _small(L=2, I=40, H=37, P=12, C=9)
+    params, _ = wl.make()
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes)
+    model = qnn.LstmModel(d, gpu(params))
+    codes, prm = model.weights()
+    c_ref, p_ref = oracle.lstm_quantize_weights(oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj,
+                                                            wl.num_classes), params)
+    assert np.array_equal(codes, c_ref)
+    assert np.array_equal(prm.view(np.int32), p_ref.view(np.int32))
+
+
+def test_lstm_streaming_state_and_host_buffers(qnn):
+    wl = _small(L=3, H=20, C=6, B=4, T=12)
+    params, x = wl.make()
+    full = _gpu_forward(qnn, wl, params, x)
+    a = _gpu_forward(qnn, wl, params, x[:, :5])
+    b = _gpu_forward(qnn, wl, params, x[:, 5:], h0=a["h"], c0=a["c"])
+    assert np.array_equal(np.concatenate([a["h_all"], b["h_all"]], 2), full["h_all"])
+    assert np.array_equal(b["h"], full["h"]) and np.array_equal(b["c"], full["c"])
+    # host (numpy) buffers through the same call
+    y_host = full["model"].forward(x)
+    assert np.array_equal(y_host, full["y"])
+
+
+def test_lstm_nonfinite_input_reported(qnn):
+    wl = _small(L=1, H=8, B=1, T=3)
+    params, x = wl.make()
+    x[0, 1, 2] = np.nan
+    d = qnn.lstm_desc(1, wl.input_dim, wl.hidden)
+    model = qnn.LstmModel(d, gpu(params))
+    model.forward(gpu(x))
+    assert qnn.device_status() == qnn.QNN_ERR_NONFINITE
+
+
+def test_config_small_1x128_full(qnn):
+    wl = inputs.SMALL_1x128
+    params, x = wl.make()
+    got = _gpu_forward(qnn, wl, params, x)
+    ref = _oracle(wl, params, x, want_h_all=True)
+    _compare(got, ref, wl)
+
+
+def test_config_5x500_b1_full(qnn):
+    # the benchmarked workload, whole: 5 x 500 cells, 2000 classes, T = 300, batch 1
+    wl = inputs.LSTM_5x500_B1
+    params, x = wl.make()
+    got = _gpu_forward(qnn, wl, params, x)
+    ref = _oracle(wl, params, x, want_h_all=True)
+    _compare(got, ref, wl)
+
+
+def test_config_5x500_b256_sampled(qnn):
+    # batch 256 x 500 frames on the GPU; the oracle recomputes two whole sequences (per-row
+    # quantization makes every sequence independent of the others).
+    wl = inputs.LSTM_5x500_B256
+    params, x = wl.make()
+    got = _gpu_forward(qnn, wl, params, x, h_all=False)
+    for b in (0, 173):
+        ref = _oracle(wl, params, x[b:b + 1])
+        assert np.array_equal(got["h"][:, b], ref["h"][:, 0]) and np.array_equal(got["c"][:, b], ref["c"][:, 0])
+        assert np.max(np.abs(got["y"][b] - ref["y"][0])) <= SOFTMAX_TOL
+
+
+def test_config_lstmp_2048_b1024_sampled(qnn):
+    # the large projected model at full batch, a 24-frame prefix (outputs are causal in time);
+    # the oracle recomputes one sequence.
+    wl = inputs.LSTMP_5x2048P512_B1024
+    params, x = wl.make(frames=24)
+    got = _gpu_forward(qnn, wl, params, x, h_all=False)
+    b = 611
+    ref = _oracle(wl, params, x[b:b + 1])
+    assert np.array_equal(got["h"][:, b], ref["h"][:, 0]) and np.array_equal(got["c"][:, b], ref["c"][:, 0])
+    assert np.max(np.abs(got["y"][b] - ref["y"][0])) <= SOFTMAX_TOL
