@@ -42,6 +42,8 @@ def parse():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(inputs.LSTM_WORKLOADS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true", help="standalone quantized matmul sweep instead")
+    ap.add_argument("--shape", default="", help="with --sweep: one shape M,N,K only")
     return ap.parse_args()
 
 
@@ -343,8 +345,69 @@ def run_ours(args, wl, rank, world, local):
     return 0
 
 
+def run_sweep(args):
+    """Standalone quantized matmul sweep (K = N in {512, 2048, 8192}, M in {1, 16, 256, 4096,
+    16384}, per-matrix units): one JSON line per shape with the product's TOPS (codes in, fp32
+    out), the fp32-in rate including the activation quantizer, and the quantizer's GB/s. L2 is
+    flushed before every timed repetition."""
+    import torch
+
+    from paper_1607_04683_gb300 import build as qbuild, qnn
+    qbuild.build()
+    torch.cuda.set_device(0)
+    peaks, peak_kind = measured_peaks()
+    imma = qnn.measure_peak(0)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    reps = max(3, args.steps)
+
+    def timed(fn):
+        ts = []
+        for _ in range(reps + 1):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            ts.append(a.elapsed_time(b))
+        return statistics.median(ts[1:]) / 1e3
+
+    shapes = inputs.QMATMUL_SWEEP
+    if args.shape:
+        M, N, K = (int(v) for v in args.shape.split(","))
+        shapes = [inputs.QmatmulShape(M, N, K)]
+    for shape in shapes:
+        W, A = inputs.make_qmatmul_operands(shape)
+        Ag, Wg = torch.from_numpy(A).cuda(), torch.from_numpy(W).cuda()
+        cw, pw, cs = qnn.qnn_quantize(Wg, qnn.PER_MATRIX)
+        ca, pa, ra = qnn.qnn_quantize(Ag, qnn.PER_MATRIX)
+        Y = torch.empty((shape.M, shape.N), dtype=torch.float32, device="cuda")
+        t_mm = timed(lambda: qnn.qnn_qmatmul(ca, pa, 0, ra, cw, pw, cs, out=Y))
+        t_q = timed(lambda: qnn.qnn_quantize(Ag, qnn.PER_MATRIX))
+
+        def both():
+            c, p, r = qnn.qnn_quantize(Ag, qnn.PER_MATRIX)
+            qnn.qnn_qmatmul(c, p, 0, r, cw, pw, cs, out=Y)
+        t_all = timed(both)
+        ops = 2.0 * shape.M * shape.N * shape.K
+        mm_bytes = shape.M * shape.K + shape.N * shape.K + 4 * shape.M * shape.N
+        print(json.dumps({
+            "sweep": "qmatmul", "M": shape.M, "N": shape.N, "K": shape.K,
+            "qmatmul_tops": ops / t_mm / 1e12, "qmatmul_ms": t_mm * 1e3,
+            "frac_of_measured_mma_u8_peak": ops / t_mm / 1e12 / imma, "mma_u8_peak_tops": imma,
+            "qmatmul_gbs": mm_bytes / t_mm / 1e9,
+            "fp32_in_tops": ops / t_all / 1e12, "quantize_ms": t_q * 1e3,
+            "quantize_gbs_alg": 5.0 * shape.M * shape.K / t_q / 1e9, "hbm_peak_gbs": peaks["hbm_gbs"],
+            "peak_kind": peak_kind, "l2": "flushed"}), flush=True)
+        del Ag, Wg, cw, ca, Y
+        torch.cuda.empty_cache()
+    return 0
+
+
 def main():
     args = parse()
+    if args.sweep:
+        return run_sweep(args)
     rank, world, local = dist_info()
     wl = inputs.LSTM_WORKLOADS[args.workload]
     if world > 1 and args.impl == "ours":

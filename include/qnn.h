@@ -175,6 +175,12 @@ qnn_status qnn_profile_enable(int on);
  * the number of distinct kernels. */
 qnn_status qnn_profile_read(int capacity, const char **names, double *total_ms, int64_t *launches, int *count);
 
+/* Measures the peak rate of an integer datapath on the current device, in tera-operations per
+ * second (a multiply-add counts as two operations): kind 0 = the warp-level integer tensor-core
+ * MMA (mma.sync m16n8k32 u8 x u8 -> s32) the products use, kind 1 = dp4a on the CUDA cores.
+ * Register-only loops on every SM; synchronous; the best of three timed runs. */
+qnn_status qnn_measure_peak(int kind, double *tops);
+
 #ifdef __cplusplus
 }
 #endif

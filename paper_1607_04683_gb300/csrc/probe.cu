@@ -1,0 +1,88 @@
+// probe.cu — peak-rate microbenchmarks of the integer datapaths the library uses, so that
+// throughput can be reported against the measured rate of this GPU rather than a datasheet.
+//
+//   kind 0: mma.sync m16n8k32 u8 x u8 -> s32 (warp-level integer tensor-core MMA)
+//   kind 1: dp4a (four 8-bit products summed into a 32-bit integer, on the CUDA cores)
+//
+// Every warp runs eight independent accumulator chains from registers (no memory traffic in the
+// loop); the result is written once so the work cannot be removed by the compiler.
+#include "qnn_host.h"
+
+namespace qnn {
+namespace {
+
+constexpr int kChains = 8;
+
+__global__ void __launch_bounds__(256) mma_u8_peak_kernel(int iters, int *sink) {
+    uint32_t a[4] = {0x01020304u ^ threadIdx.x, 0x05060708u, 0x090a0b0cu, 0x0d0e0f10u};
+    uint32_t b0 = 0x11121314u ^ blockIdx.x, b1 = 0x15161718u;
+    int acc[kChains][4] = {};
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+        for (int c = 0; c < kChains; ++c)
+            asm volatile(
+                "mma.sync.aligned.m16n8k32.row.col.s32.u8.u8.s32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                "{%0,%1,%2,%3};\n"
+                : "+r"(acc[c][0]), "+r"(acc[c][1]), "+r"(acc[c][2]), "+r"(acc[c][3])
+                : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+    }
+    int s = 0;
+#pragma unroll
+    for (int c = 0; c < kChains; ++c) s += acc[c][0] + acc[c][1] + acc[c][2] + acc[c][3];
+    if (s == 0x7fffffff) sink[0] = s;
+}
+
+__global__ void __launch_bounds__(256) dp4a_peak_kernel(int iters, int *sink) {
+    int acc[kChains];
+    const int a = 0x01020304 ^ threadIdx.x, b = 0x05060708 ^ blockIdx.x;
+#pragma unroll
+    for (int c = 0; c < kChains; ++c) acc[c] = c;
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+        for (int c = 0; c < kChains; ++c) acc[c] = __dp4a((unsigned)a, (unsigned)b, (unsigned)acc[c]);
+    }
+    int s = 0;
+#pragma unroll
+    for (int c = 0; c < kChains; ++c) s += acc[c];
+    if (s == 0x7fffffff) sink[0] = s;
+}
+
+}  // namespace
+}  // namespace qnn
+
+using namespace qnn;
+
+// Measures the peak rate of an integer datapath in tera-operations per second (one multiply-add
+// counts as two operations). Synchronous; allocates a 4-byte sink. kind: 0 = mma.sync u8, 1 = dp4a.
+extern "C" qnn_status qnn_measure_peak(int kind, double *tops) {
+    if (!tops || kind < 0 || kind > 1) return QNN_ERR_INVALID_ARG;
+    int *sink = nullptr;
+    QNN_CUDA_TRY(cudaMalloc(&sink, sizeof(int)));
+    const int blocks = sm_count() * 4;
+    const int iters = kind == 0 ? 4096 : 16384;
+    cudaEvent_t e0, e1;
+    QNN_CUDA_TRY(cudaEventCreate(&e0));
+    QNN_CUDA_TRY(cudaEventCreate(&e1));
+    double best = 0.0;
+    for (int rep = 0; rep < 4; ++rep) {
+        QNN_CUDA_TRY(cudaEventRecord(e0));
+        if (kind == 0)
+            mma_u8_peak_kernel<<<blocks, 256>>>(iters, sink);
+        else
+            dp4a_peak_kernel<<<blocks, 256>>>(iters, sink);
+        QNN_CUDA_TRY(cudaEventRecord(e1));
+        QNN_CUDA_TRY(cudaEventSynchronize(e1));
+        float ms = 0.0f;
+        QNN_CUDA_TRY(cudaEventElapsedTime(&ms, e0, e1));
+        const double warps = (double)blocks * 8.0;
+        const double ops = kind == 0 ? warps * iters * kChains * (2.0 * 16 * 8 * 32)
+                                     : (double)blocks * 256.0 * iters * kChains * 8.0;
+        const double r = ops / (ms * 1e-3) / 1e12;
+        if (rep > 0 && r > best) best = r;
+    }
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    cudaFree(sink);
+    *tops = best;
+    return QNN_OK;
+}

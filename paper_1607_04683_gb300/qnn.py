@@ -32,7 +32,7 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 # Every symbol the header declares (checked by the CPU test that loads the library).
 EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmul", "qnn_lstm_param_count",
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
-           "qnn_profile_enable", "qnn_profile_read")
+           "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak")
 
 
 class QnnError(RuntimeError):
@@ -80,12 +80,21 @@ def lib():
         L.qnn_profile_enable.restype = i32
         L.qnn_profile_read.argtypes = [i32, P, P, P, C.POINTER(i32)]
         L.qnn_profile_read.restype = i32
+        L.qnn_measure_peak.argtypes = [i32, C.POINTER(C.c_double)]
+        L.qnn_measure_peak.restype = i32
         _lib = L
     return _lib
 
 
 def profile_enable(on: bool = True):
     _check(lib().qnn_profile_enable(1 if on else 0), "qnn_profile_enable")
+
+
+def measure_peak(kind: int) -> float:
+    """Measured peak TOPS of an integer datapath: 0 = mma.sync u8 tensor-core MMA, 1 = dp4a."""
+    v = C.c_double(0.0)
+    _check(lib().qnn_measure_peak(kind, C.byref(v)), "qnn_measure_peak")
+    return v.value
 
 
 def profile_read() -> dict:
