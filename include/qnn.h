@@ -161,6 +161,30 @@ qnn_status qnn_lstm_model_weights(const qnn_lstm_model *m, uint8_t *codes_host, 
 qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
                             float *c_state, float *h_all, void *stream);
 
+/*
+ * qnn_quantize_matrix_static — qnn_quantize with QNN_PER_MATRIX, allocating nothing.
+ * The paper has no counterpart: this is an interface for callers that cannot allocate device
+ * memory inside a library call (a fixed pre-reserved memory budget, device memory owned by the
+ * caller's own allocator or pool, or a latency-critical stream where the device-wide
+ * synchronization of cudaMalloc/cudaFree is not acceptable). Same results as qnn_quantize with
+ * QNN_PER_MATRIX (codes, params[0], code_sums) for finite inputs.
+ *   x, codes, params, code_sums: as for qnn_quantize (device memory, caller-owned); params has
+ *     one entry.
+ *   status   device int, nullable, caller-owned: QNN_ERR_NONFINITE is written into it (if it is
+ *     still 0) when the matrix holds NaN or +-Inf; the codes are then unspecified.
+ * Limits: rows <= 524288 (its scratch holds one partial range per 32 rows); larger inputs return
+ * QNN_ERR_INVALID_ARG before anything runs.
+ * Scratch: a 128 KiB + 256 B static device array inside the library, held on every GPU that loads
+ * the library until the process exits and shared by all calls. Calls that overlap in time on the
+ * GPU (unordered streams) race on it; ordered calls are safe (each call clears the completion
+ * counter on its stream before its kernels run). The first call on each device resolves the
+ * array's device address (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture. Calls no cudaMalloc or cudaFree.
+ */
+qnn_status qnn_quantize_matrix_static(const float *x, int64_t rows, int64_t cols, int64_t ldx, uint8_t *codes,
+                                      int64_t ldc, qnn_qparams *params, int32_t *code_sums, int *status,
+                                      void *stream);
+
 /* ---------------------------------------------------------------------------------------------
  * Kernel timing (diagnostics and benchmarks; no counterpart in the paper).
  * ------------------------------------------------------------------------------------------- */

@@ -32,7 +32,7 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 # Every symbol the header declares (checked by the CPU test that loads the library).
 EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmul", "qnn_lstm_param_count",
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
-           "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak")
+           "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static")
 
 
 class QnnError(RuntimeError):
@@ -82,6 +82,8 @@ def lib():
         L.qnn_profile_read.restype = i32
         L.qnn_measure_peak.argtypes = [i32, C.POINTER(C.c_double)]
         L.qnn_measure_peak.restype = i32
+        L.qnn_quantize_matrix_static.argtypes = [P, i64, i64, i64, P, i64, P, P, P, P]
+        L.qnn_quantize_matrix_static.restype = i32
         _lib = L
     return _lib
 
