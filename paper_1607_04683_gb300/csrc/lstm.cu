@@ -17,6 +17,7 @@
 #include <cstring>
 #include <vector>
 
+#include "lstm_model.h"
 #include "qnn_device.cuh"
 #include "qnn_host.h"
 
@@ -408,39 +409,6 @@ using namespace qnn;
 
 namespace {
 
-struct QUnitDev {  // one quantized weight matrix (or the four gate matrices of one kind)
-    uint8_t *codes = nullptr;  // [rows][ld]
-    int32_t *sums = nullptr;   // [rows]
-    qnn_qparams *params = nullptr;  // [n_units]
-    int64_t rows = 0, cols = 0, ld = 0;
-    int n_units = 0;
-};
-
-struct LayerDev {
-    QUnitDev wx, wh, wp;
-    float *bias = nullptr;  // [4H]
-    int64_t kin = 0;
-};
-
-}  // namespace
-
-struct qnn_lstm_model {
-    qnn_lstm_desc d{};
-    int64_t L = 0, I = 0, H = 0, P = 0, C = 0, R = 0;
-    int device = 0;
-    void *weights = nullptr;
-    std::vector<LayerDev> layers;
-    QUnitDev wo;
-    float *wo_f = nullptr, *bo = nullptr;
-    // forward workspace
-    void *ws = nullptr;
-    size_t ws_bytes = 0;
-    // host mirror of the unit parameters (filled at creation)
-    std::vector<qnn_qparams> host_params;
-};
-
-namespace {
-
 bool valid_desc(const qnn_lstm_desc *d) {
     if (!d || d->num_layers < 1 || d->input_dim < 1 || d->hidden < 1 || d->proj < 0 || d->num_classes < 0) return false;
     if ((d->num_classes == 0) != (d->output_mode == QNN_OUT_NONE)) return false;
@@ -493,6 +461,7 @@ extern "C" void qnn_lstm_model_destroy(qnn_lstm_model *m) {
     cudaDeviceSynchronize();
     cudaFree(m->weights);
     cudaFree(m->ws);
+    cudaFree(m->sws);
     cudaSetDevice(prev);
     delete m;
 }
@@ -699,6 +668,12 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const bool x_dev = is_device_ptr(x), y_dev = is_device_ptr(y);
     const bool hs_dev = h_state && is_device_ptr(h_state), cs_dev = c_state && is_device_ptr(c_state);
     const bool ha_dev = h_all && is_device_ptr(h_all);
+    if (path_choice() != PathChoice::kLayerwise) {
+        bool used = false;
+        QNN_TRY(small_path_forward(m, x, B, T, y, h_state, c_state, h_all, st, &used));
+        if (used) return QNN_OK;
+        if (path_choice() == PathChoice::kSmall) return QNN_ERR_INVALID_ARG;
+    }
     const FwdPlan plan = plan_recurrent(m, B);
 
     // workspace layout

@@ -326,3 +326,41 @@ def test_config_lstmp_2048_b1024_sampled(qnn):
     ref = _oracle(wl, params, x[b:b + 1])
     assert np.array_equal(got["h"][:, b], ref["h"][:, 0]) and np.array_equal(got["c"][:, b], ref["c"][:, 0])
     assert np.max(np.abs(got["y"][b] - ref["y"][0])) <= SOFTMAX_TOL
+
+
+# ------------------------------------------------------------------------------------------
+# The two forward paths: batch-of-few cluster pipeline and layer-by-layer
+# ------------------------------------------------------------------------------------------
+
+PATH_CASES = [dict(L=1, I=40, H=128, B=1, T=20), dict(L=3, I=40, H=100, C=37, B=2, T=9),
+              dict(L=2, I=13, H=500, C=2000, B=4, T=5, w=0.08), dict(L=5, I=40, H=33, C=3, B=3, T=4)]
+
+
+@pytest.mark.parametrize("cfg", PATH_CASES)
+def test_small_and_layerwise_paths_agree(qnn, cfg, monkeypatch):
+    wl = _small(**cfg)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x, want_h_all=True)
+    outs = {}
+    for path in ("small", "layerwise"):
+        monkeypatch.setenv("QNN_LSTM_PATH", path)
+        qnn.profile_read()
+        qnn.profile_enable(True)
+        got = _gpu_forward(qnn, wl, params, x)
+        qnn.profile_enable(False)
+        kernels = qnn.profile_read()
+        assert ("lstm_small" in kernels) == (path == "small"), kernels
+        _compare(got, ref, wl)
+        outs[path] = got
+    assert np.array_equal(outs["small"]["y"], outs["layerwise"]["y"])
+
+
+def test_benchmarked_workload_takes_the_small_path(qnn, monkeypatch):
+    monkeypatch.delenv("QNN_LSTM_PATH", raising=False)
+    wl = inputs.LSTM_5x500_B1
+    params, x = wl.make(frames=8)
+    qnn.profile_read()
+    qnn.profile_enable(True)
+    _gpu_forward(qnn, wl, params, x, h_all=False)
+    qnn.profile_enable(False)
+    assert "lstm_small" in qnn.profile_read()
