@@ -2,24 +2,31 @@
 // launch, organised as a dataflow pipeline of thread-block clusters (no grid-wide barrier).
 //
 // Roles. Each LSTM layer is one cluster of CS blocks (CS = ceil(H / 32) <= 16); block r of the
-// cluster owns cells [32 r, 32 r + 32): all four gate rows of its cells in Wx and Wh, held in
-// registers (warp w: cells 2w, 2w+1, i.e. 8 gate rows; lane l: bytes [16 l, 16 l + 16) of every
-// row, so K <= 512). The softmax layer's 8-bit product runs in further clusters, 128 rows of Wo
-// per block. Every block has 16 compute warps and one loader warp.
-//
-// Per frame t, in every layer block:
-//   X  the loader warp has put the layer's input row for frame t (x_t, or the previous layer's
-//      h_t) into a shared-memory ring; each compute warp quantizes it (one unit per row, eq. 2),
-//      multiplies with its Wx rows (dp4a, u8 x u8 -> s32), reduces across the warp and recovers
-//      the product plus bias (eq. 1, eq. 3, Fig. 1).
-//   H  it waits until all blocks of the cluster have delivered h_{t-1} into its shared memory
-//      (distributed shared memory stores + remote mbarrier arrivals), quantizes h_{t-1}, multiplies
-//      with its Wh rows, adds, applies the gates and the cell update (c stays in registers) and
-//      sends its two new h values to every block of the cluster; it also writes them to global
-//      memory tagged with the launch's epoch, where the next layer's loader polls for them.
-// Layers therefore run one frame apart, and the recurrence of a layer only waits on its own
-// cluster. Every wait is bounded in time (QNN_ERR_TIMEOUT, then every block leaves its loop and
-// meets its cluster at the final cluster barrier).
+// cluster owns cells [32 r, 32 r + 32): the 128 gate rows (cell c, gate g -> local row 4 c + g)
+// of Wx and Wh. The softmax layer's 8-bit product runs in further clusters, 128 rows of Wo per
+// block. A block has three kinds of warps:
+//   8 product warps   16 local rows each; Wh (or Wo) rows in registers, lane l holding bytes
+//                     [16 l, 16 l + 16) of each row (so K <= 512), Wx rows in shared memory.
+//   4 epilogue warps  one thread per (cell, gate): recovery, bias, gate nonlinearity, and in the
+//                     first lane of each quad the cell update (c stays in that register).
+//   1 loader warp     brings each frame's input row into a shared-memory ring: x_t for the first
+//                     layer, otherwise the previous layer's h_t, polled from global memory where
+//                     it is written tagged with the launch's epoch; it also finds the row's range.
+// Per frame t of a layer block:
+//   X  the product warps quantize the input row cooperatively (two values per thread, eq. 2 with
+//      the loader's range), multiply with Wx (dp4a, u8 x u8 -> s32, reduced across the warp) and
+//      hand the int32 sums to the epilogue warps (mbarrier).
+//   H  they wait until every block of the cluster has delivered its 32 values of h_{t-1} and their
+//      range (distributed shared memory stores + one remote mbarrier arrival per block), quantize
+//      h_{t-1} cooperatively, multiply with Wh and hand the sums over.
+//   E  the epilogue warps apply eq. 1's offsets, recover, add the bias, apply the gates and the
+//      cell update, then send the block's 32 new h values and their range to every block of the
+//      cluster, and write them tagged to global memory for the next layer.
+// A layer's recurrence only waits on its own cluster; consecutive layers run one frame apart. Every
+// wait is bounded in time: one that gives up records QNN_ERR_TIMEOUT and raises an abort flag,
+// after which all waits return at once, so every block runs its loop to the end (outputs then
+// meaningless) and meets its cluster at the final cluster barrier; no block exits while a peer
+// may still write into its shared memory.
 #include <cfloat>
 #include <cstdlib>
 #include <cstring>
@@ -31,15 +38,21 @@
 namespace qnn {
 namespace {
 
-constexpr int kSW = 16;                     // compute warps per block
-constexpr int kSThreads = (kSW + 1) * 32;   // plus one loader warp
-constexpr int kRing = 4;                    // input ring depth (frames)
-constexpr int kMaxB = 4;                    // batch limit of this path
-constexpr int kMaxK = 512;                  // 16 bytes of every weight row per lane
-constexpr int kCellsPerBlock = 2 * kSW;     // 32
-constexpr int kOutRowsPerBlock = 8 * kSW;   // 128
+constexpr int kPW = 8;                        // product warps
+constexpr int kEW = 4;                        // epilogue warps
+constexpr int kPT = kPW * 32;                 // product threads (256)
+constexpr int kET = kEW * 32;                 // epilogue threads (128)
+constexpr int kLoaderWarp = kPW + kEW;        // warp 12
+constexpr int kSThreads = (kPW + kEW + 1) * 32;  // 416
+constexpr int kRing = 4;                      // input ring depth (frames)
+constexpr int kMaxB = 4;                      // batch limit of this path
+constexpr int kMaxK = 512;                    // 16 bytes of every weight row per lane
+constexpr int kRows = 128;                    // local rows per block
+constexpr int kCellsPerBlock = kRows / 4;     // 32
+constexpr int kMaxCS = 16;
 constexpr int kMaxLayers = 8;
 constexpr unsigned long long kWaitNs = 2000000000ull;
+constexpr int kSpinCheck = 512;               // polls between checks of the clock and the abort flag
 
 struct SmallLayer {
     const uint8_t *wx;
@@ -72,6 +85,32 @@ struct SmallArgs {
     int L, I, H, R, C, B, T, CS;
 };
 
+// ---- shared memory layout ---------------------------------------------------------------------
+
+struct RowMeta {  // quantized activation row: offset, scale, code sum
+    int za;
+    float Qa;
+    int rs;
+    int pad;
+};
+
+struct Smem {
+    float hbuf[2][kMaxB][kMaxK];        // h_{t} of the whole layer, by frame parity (cluster writes)
+    float2 hmm[2][kMaxB][kMaxCS];       // per source block: range of its 32 values
+    float ring[kRing][kMaxB][kMaxK];    // input rows (loader writes)
+    float2 ring_mm[kRing][kMaxB];       // their ranges
+    int ring_bad[kRing][kMaxB];         // non-finite flag
+    uint8_t codes_x[kMaxB][kMaxK];      // quantized input rows of the current frame
+    uint8_t codes_h[kMaxB][kMaxK];      // quantized h_{t-1}
+    int acc_x[2][kMaxB][kRows];         // int32 sums, by frame parity
+    int acc_h[2][kMaxB][kRows];
+    RowMeta meta_x[2][kMaxB], meta_h[2][kMaxB];
+    float hloc[2][kMaxB][kCellsPerBlock];  // this block's new h values
+    float2 emm[2][kMaxB][kEW];           // epilogue warps' ranges
+    uint8_t wx[kRows][kMaxK];            // Wx rows of this block (local row order)
+    unsigned long long bar_full[kRing], bar_empty[kRing], bar_h[2], bar_ax[2], bar_ah[2];
+};
+
 // ---- PTX helpers --------------------------------------------------------------------------------
 
 __device__ __forceinline__ uint32_t saddr(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
@@ -81,16 +120,13 @@ __device__ __forceinline__ unsigned long long now_ns() {
     asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
     return t;
 }
-
 __device__ __forceinline__ void mbar_init(uint32_t bar, unsigned count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
-
-__device__ __forceinline__ void mbar_arrive_local(uint32_t bar) {
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}" ::"r"(bar) : "memory");
 }
-
-__device__ __forceinline__ bool mbar_try_local(uint32_t bar, unsigned parity) {
+__device__ __forceinline__ bool mbar_try(uint32_t bar, unsigned parity) {
     uint32_t ok;
     asm volatile(
         "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
@@ -99,7 +135,6 @@ __device__ __forceinline__ bool mbar_try_local(uint32_t bar, unsigned parity) {
         : "memory");
     return ok != 0;
 }
-
 __device__ __forceinline__ bool mbar_try_cluster(uint32_t bar, unsigned parity) {
     uint32_t ok;
     asm volatile(
@@ -110,46 +145,52 @@ __device__ __forceinline__ bool mbar_try_cluster(uint32_t bar, unsigned parity) 
         : "memory");
     return ok != 0;
 }
-
 __device__ __forceinline__ uint32_t map_rank(uint32_t local, uint32_t rank) {
     uint32_t r;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
     return r;
 }
-
-__device__ __forceinline__ void st_cluster_f32x2(uint32_t raddr, float a, float b) {
+__device__ __forceinline__ void st_cluster_v4(uint32_t raddr, float4 v) {
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(raddr), "f"(v.x), "f"(v.y), "f"(v.z),
+                 "f"(v.w)
+                 : "memory");
+}
+__device__ __forceinline__ void st_cluster_v2(uint32_t raddr, float a, float b) {
     asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(raddr), "f"(a), "f"(b) : "memory");
 }
-
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t raddr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(raddr) : "memory");
 }
-
 __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-
 __device__ __forceinline__ uint32_t cluster_rank() {
     uint32_t r;
     asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
     return r;
 }
-
 __device__ __forceinline__ unsigned long long ld_tag(const unsigned long long *p) {
     unsigned long long v;
     asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
     return v;
 }
-
 __device__ __forceinline__ void st_tag(unsigned long long *p, unsigned long long v) {
     asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
+__device__ __forceinline__ void named_bar(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
 
-// Bounded wait helpers: false when the wait gave up (timeout recorded) or another block aborted.
-struct Waiter {
+// Bounded waits. A wait that gives up records QNN_ERR_TIMEOUT and raises the abort flag; every
+// later wait then returns within kSpinCheck polls. Waits never make a warp leave its loop, so all
+// warps keep executing the same sequence of named barriers and the launch always runs to its end.
+struct Deadline {
     const SmallArgs *a;
     unsigned long long t0;
+    int spins;
     __device__ bool expired() {
+        if (++spins < kSpinCheck) return false;
+        spins = 0;
         if (*(volatile int *)a->abort_flag) return true;
         if (now_ns() - t0 > kWaitNs) {
             record_status(a->status, QNN_ERR_TIMEOUT);
@@ -160,165 +201,83 @@ struct Waiter {
     }
 };
 
-// Warp-uniform results: every lane of the warp gets the same answer.
-__device__ __forceinline__ bool wait_local(const SmallArgs &a, uint32_t bar, unsigned parity) {
-    bool ok = true;
-    if (!mbar_try_local(bar, parity)) {
-        Waiter w{&a, now_ns()};
-        while (!mbar_try_local(bar, parity))
-            if (w.expired()) {
-                ok = false;
-                break;
-            }
-    }
-    return __all_sync(0xffffffffu, ok);
+__device__ __forceinline__ void wait_cta(const SmallArgs &a, uint32_t bar, unsigned parity) {
+    if (mbar_try(bar, parity)) return;
+    Deadline d{&a, now_ns(), 0};
+    while (!mbar_try(bar, parity))
+        if (d.expired()) return;
 }
 
-__device__ __forceinline__ bool wait_cluster(const SmallArgs &a, uint32_t bar, unsigned parity) {
-    bool ok = true;
-    if (!mbar_try_cluster(bar, parity)) {
-        Waiter w{&a, now_ns()};
-        while (!mbar_try_cluster(bar, parity))
-            if (w.expired()) {
-                ok = false;
-                break;
-            }
-    }
-    return __all_sync(0xffffffffu, ok);
+__device__ __forceinline__ void wait_cluster(const SmallArgs &a, uint32_t bar, unsigned parity) {
+    if (mbar_try_cluster(bar, parity)) return;
+    Deadline d{&a, now_ns(), 0};
+    while (!mbar_try_cluster(bar, parity))
+        if (d.expired()) return;
 }
 
-// ---- per-warp quantization of one row held in shared memory ------------------------------------
+// ---- product warps ------------------------------------------------------------------------------
 
-struct RowQ {
-    uint32_t code[4];  // codes of bytes [16 lane, 16 lane + 16), zero past len
-    int za, rs;
-    float Qa;
-};
-
-// Row of `len` fp32 values in shared memory; every lane of the warp gets the unit's parameters
-// (eq. 2), its 16 codes and the row code sum.
-__device__ __forceinline__ RowQ quantize_row_warp(const float *row, int len, const SmallArgs &a) {
-    const int lane = threadIdx.x & 31;
-    const int k0 = lane * 16;
-    float mn = FLT_MAX, mx = -FLT_MAX;
-    bool bad = false;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int k = k0 + 4 * q;
-        if (k < len) {
-            float4 v = *reinterpret_cast<const float4 *>(row + k);
-            float e[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-                if (k + i < len) {
-                    bad |= !isfinite(e[i]);
-                    mn = fminf(mn, e[i]);
-                    mx = fmaxf(mx, e[i]);
-                }
-        }
-    }
-    mn = warp_min(mn);
-    mx = warp_max(mx);
-    if (__any_sync(0xffffffffu, bad)) {
-        if (lane == 0) record_status(a.status, QNN_ERR_NONFINITE);
-        mn = 0.0f;
-        mx = 0.0f;
-    }
-    const qnn_qparams p = params_from_range(mn, mx);
-    RowQ r;
-    int s = 0;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int k = k0 + 4 * q;
-        uint32_t w = 0;
-        if (k < len) {
-            float4 v = *reinterpret_cast<const float4 *>(row + k);
-            float e[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-                if (k + i < len) {
-                    uint32_t c = quant_code(e[i], p.Q, p.z);
-                    s += (int)c;
-                    w |= c << (8 * i);
-                }
-        }
-        r.code[q] = w;
-    }
-    r.rs = warp_sum(s);
-    r.za = p.z;
-    r.Qa = p.Q;
-    return r;
-}
-
-// Eight row partial dot products (8 rows x 16 bytes of this lane), reduced across the warp so that
-// lane l ends with the full sum of row ((l >> 2) & 7).
-__device__ __forceinline__ int dot8_reduce(const uint32_t (&w)[8][4], const RowQ &q) {
-    int v[8];
-#pragma unroll
-    for (int r = 0; r < 8; ++r) {
-        unsigned acc = 0;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) acc = __dp4a(w[r][i], q.code[i], acc);  // u8 x u8 summed into u32
-        v[r] = (int)acc;
-    }
-    const int lane = threadIdx.x & 31;
-    const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4;
-    int u[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int send = b4 ? v[i] : v[i + 4];
-        const int keep = b4 ? v[i + 4] : v[i];
-        u[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
-    }
-    int x2[2];
+// Codes of two values per product thread (k = tid, tid + 256 < len) into `codes` (eq. 2 with the
+// unit's range already known). Zero past len.
+__device__ __forceinline__ void code_row(const float *row, int len, const qnn_qparams &p, uint8_t *codes, int tid) {
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
-        const int send = b3 ? u[i] : u[i + 2];
-        const int keep = b3 ? u[i + 2] : u[i];
-        x2[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+        const int k = tid + i * kPT;
+        codes[k] = k < len ? (uint8_t)quant_code(row[k], p.Q, p.z) : (uint8_t)0;
     }
-    const int send = b2 ? x2[0] : x2[1];
-    const int keep = b2 ? x2[1] : x2[0];
-    int s = keep + __shfl_xor_sync(0xffffffffu, send, 4);
-    s += __shfl_xor_sync(0xffffffffu, s, 2);
-    s += __shfl_xor_sync(0xffffffffu, s, 1);
-    return s;
 }
 
-__device__ __forceinline__ void load_rows(uint32_t (&w)[8][4], const uint8_t *base, int ld, int H, int kind,
-                                          int first, int valid_rows, int lane) {
-    // kind 0: gate rows of two cells (row r -> gate r & 3 of cell first + (r >> 2)), rows g*H + j
-    // kind 1: plain rows first + r
+// Sixteen row partial dot products of this lane (16 rows x 16 bytes), summed across the warp so
+// that lane l ends with the full sum of local row ((l >> 1) & 15). Also returns the row code sum.
+__device__ __forceinline__ int dot16(const uint32_t (&w)[16][4], const uint8_t *codes, int &rs) {
+    const int lane = threadIdx.x & 31;
+    const uint4 cv = *reinterpret_cast<const uint4 *>(codes + lane * 16);
+    const uint32_t c[4] = {cv.x, cv.y, cv.z, cv.w};
+    unsigned bs = 0;
 #pragma unroll
-    for (int r = 0; r < 8; ++r) {
-        int64_t row;
-        bool ok;
-        if (kind == 0) {
-            const int j = first + (r >> 2);
-            ok = j < H && (r >> 2) < valid_rows;
-            row = (int64_t)(r & 3) * H + j;
-        } else {
-            ok = r < valid_rows;
-            row = first + r;
+    for (int i = 0; i < 4; ++i) bs = __dp4a(c[i], 0x01010101u, bs);
+    rs = warp_sum((int)bs);
+    int v[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+        unsigned acc = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc = __dp4a(w[r][i], c[i], acc);
+        v[r] = (int)acc;
+    }
+#pragma unroll
+    for (int s = 4; s >= 1; --s) {  // halve the live rows at each exchange: 8, 4, 2, 1
+        const int half = 1 << (s - 1);
+        const bool up = (lane >> s) & 1;
+#pragma unroll
+        for (int i = 0; i < half; ++i) {
+            const int send = up ? v[i] : v[i + half];
+            const int keep = up ? v[i + half] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 1 << s);
         }
+    }
+    return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
+}
+
+// Loads 16 local rows into registers; local row lr maps to a global row through row_of(lr)
+// (negative: absent, zero codes).
+template <typename RowOf>
+__device__ __forceinline__ void load_rows16(uint32_t (&w)[16][4], const uint8_t *base, int ld, int first, RowOf row_of) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+        const int64_t row = row_of(first + r);
         uint4 v = make_uint4(0, 0, 0, 0);
-        if (ok && lane * 16 < ld) v = *reinterpret_cast<const uint4 *>(base + row * ld + lane * 16);
-        w[r][0] = v.x;
-        w[r][1] = v.y;
-        w[r][2] = v.z;
-        w[r][3] = v.w;
+        if (row >= 0 && lane * 16 < ld) v = *reinterpret_cast<const uint4 *>(base + row * ld + lane * 16);
+        w[r][0] = v.x, w[r][1] = v.y, w[r][2] = v.z, w[r][3] = v.w;
     }
 }
 
 __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_constant__ SmallArgs a) {
-    extern __shared__ __align__(128) uint8_t smem[];
-    float *hbuf = reinterpret_cast<float *>(smem);                 // [2][kMaxB][kMaxK]
-    float *ring = hbuf + 2 * kMaxB * kMaxK;                        // [kRing][kMaxB][kMaxK]
-    uint8_t *swx = reinterpret_cast<uint8_t *>(ring + kRing * kMaxB * kMaxK);  // [8 kSW][kMaxK] Wx rows
-    uint64_t *bars = reinterpret_cast<uint64_t *>(swx + 8 * kSW * kMaxK);
-    const uint32_t full0 = saddr(bars), empty0 = saddr(bars + kRing), hbar0 = saddr(bars + 2 * kRing);
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    Smem &S = *reinterpret_cast<Smem *>(smem_raw);
 
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
     const int CS = a.CS;
     const int cid = blockIdx.x / CS;
     const uint32_t rank = cluster_rank();
@@ -326,41 +285,74 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
     const int l = cid;
     const int B = a.B, T = a.T, H = a.H, R = a.R;
     const int kin = is_layer ? a.layer[l].kin : R;
+    const int j0 = (int)rank * kCellsPerBlock;
 
-    if (threadIdx.x == 0) {
+    const uint32_t full0 = saddr(&S.bar_full[0]), empty0 = saddr(&S.bar_empty[0]);
+    const uint32_t hbar0 = saddr(&S.bar_h[0]), axb0 = saddr(&S.bar_ax[0]), ahb0 = saddr(&S.bar_ah[0]);
+
+    if (tid == 0) {
         for (int i = 0; i < kRing; ++i) {
             mbar_init(full0 + 8 * i, 32);
-            mbar_init(empty0 + 8 * i, kSW);
+            mbar_init(empty0 + 8 * i, 1);
         }
-        mbar_init(hbar0, CS * kSW);
-        mbar_init(hbar0 + 8, CS * kSW);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(hbar0 + 8 * i, CS);
+            mbar_init(axb0 + 8 * i, kPT);
+            mbar_init(ahb0 + 8 * i, kPT);
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    // initial state h_{-1} of this layer into hbuf[1]
     if (is_layer) {
-        for (int i = threadIdx.x; i < B * kMaxK; i += kSThreads) {
+        // h_{-1} of the whole layer into hbuf[1]; its range into every source slot of hmm[1]
+        for (int i = tid; i < B * kMaxK; i += kSThreads) {
             const int b = i / kMaxK, k = i % kMaxK;
-            hbuf[(1 * kMaxB + b) * kMaxK + k] = k < R ? a.h0[((int64_t)l * B + b) * R + k] : 0.0f;
+            S.hbuf[1][b][k] = k < R ? a.h0[((int64_t)l * B + b) * R + k] : 0.0f;
+        }
+        __syncthreads();
+        if (warp < B) {
+            float mn = FLT_MAX, mx = -FLT_MAX;
+            for (int k = lane; k < R; k += 32) {
+                mn = fminf(mn, S.hbuf[1][warp][k]);
+                mx = fmaxf(mx, S.hbuf[1][warp][k]);
+            }
+            mn = warp_min(mn);
+            mx = warp_max(mx);
+            if (lane < kMaxCS) S.hmm[1][warp][lane] = make_float2(mn, mx);
+        }
+        // Wx rows of this block, local row 4c + g <- global row g H + j0 + c
+        const SmallLayer &ly = a.layer[l];
+        for (int i = tid; i < kRows * (kMaxK / 16); i += kSThreads) {
+            const int lr = i / (kMaxK / 16), ch = i % (kMaxK / 16);
+            const int j = j0 + lr / 4, g = lr % 4;
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (j < H && ch * 16 < ly.ldx)
+                v = *reinterpret_cast<const uint4 *>(ly.wx + ((int64_t)g * H + j) * ly.ldx + ch * 16);
+            *reinterpret_cast<uint4 *>(&S.wx[lr][ch * 16]) = v;
         }
     }
     __syncthreads();
     cluster_sync();
 
-    bool ok = true;
-    if (warp == kSW) {
-        // ---------------- loader warp ----------------
-        const float *xin = a.x;
+    if (warp == kLoaderWarp) {
+        // ---------------- loader ----------------
         const unsigned long long *src = nullptr;
         if (!(is_layer && l == 0)) src = a.hx + (int64_t)(is_layer ? l - 1 : a.L - 1) * B * T * R;
-        for (int t = 0; t < T && ok; ++t) {
+        for (int t = 0; t < T; ++t) {
             const int slot = t % kRing;
-            if (t >= kRing) ok = wait_local(a, empty0 + 8 * slot, ((t / kRing) - 1) & 1);
-            if (!ok) break;
-            for (int b = 0; b < B && ok; ++b) {
-                float *dst = ring + ((int64_t)slot * kMaxB + b) * kMaxK;
+            if (t >= kRing) wait_cta(a, empty0 + 8 * slot, ((t / kRing) - 1) & 1);
+            for (int b = 0; b < B; ++b) {
+                float *dst = S.ring[slot][b];
+                float mn = FLT_MAX, mx = -FLT_MAX;
+                bool bad = false;
                 if (src == nullptr) {
-                    const float *xr = xin + ((int64_t)b * T + t) * a.I;
-                    for (int k = lane; k < kin; k += 32) dst[k] = xr[k];
+                    const float *xr = a.x + ((int64_t)b * T + t) * a.I;
+                    for (int k = lane; k < kin; k += 32) {
+                        const float v = xr[k];
+                        dst[k] = v;
+                        bad |= !isfinite(v);
+                        mn = fminf(mn, v);
+                        mx = fmaxf(mx, v);
+                    }
                 } else {
                     const unsigned long long *hr = src + ((int64_t)b * T + t) * R;
                     unsigned long long v[16];
@@ -369,172 +361,230 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                         const int k = lane + 32 * i;
                         v[i] = k < kin ? ld_tag(hr + k) : ((unsigned long long)a.epoch << 32);
                     }
-                    Waiter wt{&a, now_ns()};
+                    Deadline d{&a, now_ns(), 0};
                     while (true) {
                         bool ready = true;
 #pragma unroll
                         for (int i = 0; i < 16; ++i) ready &= (unsigned)(v[i] >> 32) == a.epoch;
                         if (__all_sync(0xffffffffu, ready)) break;
-                        if (wt.expired()) {
-                            ok = false;
-                            break;
-                        }
+                        if (__any_sync(0xffffffffu, d.expired())) break;
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             const int k = lane + 32 * i;
                             if (k < kin && (unsigned)(v[i] >> 32) != a.epoch) v[i] = ld_tag(hr + k);
                         }
                     }
-                    ok = __all_sync(0xffffffffu, ok);
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
                         const int k = lane + 32 * i;
-                        if (k < kin) dst[k] = __uint_as_float((unsigned)(v[i] & 0xffffffffu));
+                        if (k < kin) {
+                            const float f = __uint_as_float((unsigned)(v[i] & 0xffffffffu));
+                            dst[k] = f;
+                            bad |= !isfinite(f);
+                            mn = fminf(mn, f);
+                            mx = fmaxf(mx, f);
+                        }
+                    }
+                }
+                mn = warp_min(mn);
+                mx = warp_max(mx);
+                bad = __any_sync(0xffffffffu, bad);
+                if (lane == 0) {
+                    S.ring_mm[slot][b] = make_float2(mn, mx);
+                    S.ring_bad[slot][b] = bad ? 1 : 0;
+                }
+            }
+            mbar_arrive(full0 + 8 * slot);
+        }
+    } else if (warp < kPW) {
+        // ---------------- product warps ----------------
+        const int lr0 = warp * 16;  // local rows lr0 .. lr0 + 15
+        uint32_t wr[16][4];
+        if (is_layer) {
+            const SmallLayer &ly = a.layer[l];
+            load_rows16(wr, ly.wh, ly.ldh, lr0, [&](int lr) -> int64_t {
+                const int j = j0 + lr / 4;
+                return j < H ? (int64_t)(lr % 4) * H + j : -1;
+            });
+        } else {
+            const int nb = ((cid - a.L) * CS + (int)rank) * kRows;
+            load_rows16(wr, a.wo, a.ldo, lr0, [&](int lr) -> int64_t { return nb + lr < a.C ? nb + lr : -1; });
+        }
+        // output-layer epilogue constants (product lanes hold row lr0 + ((lane >> 1) & 15))
+        int o_cs = 0, o_n = -1;
+        float o_b = 0.0f;
+        if (!is_layer) {
+            const int n = ((cid - a.L) * CS + (int)rank) * kRows + lr0 + ((lane >> 1) & 15);
+            if (n < a.C) {
+                o_n = n;
+                o_cs = a.wo_sum[n];
+                o_b = a.bo[n];
+            }
+        }
+        // X phase of frame t: ring -> codes -> products (layer: Wx sums to the epilogue; output
+        // layer: logits).
+        auto x_phase = [&](int t) {
+            const int slot = t % kRing, par = t & 1;
+            wait_cta(a, full0 + 8 * slot, (t / kRing) & 1);
+            for (int b = 0; b < B; ++b) {
+                const float2 mm = S.ring_mm[slot][b];
+                float mn = mm.x, mx = mm.y;
+                if (S.ring_bad[slot][b]) {
+                    if (tid == 0) record_status(a.status, QNN_ERR_NONFINITE);
+                    mn = 0.0f;
+                    mx = 0.0f;
+                }
+                const qnn_qparams p = params_from_range(mn, mx);
+                code_row(S.ring[slot][b], kin, p, S.codes_x[b], tid);
+                if (tid == 0) S.meta_x[par][b] = RowMeta{p.z, p.Q, 0, 0};
+            }
+            named_bar(1, kPT);
+            if (tid == 0) mbar_arrive(empty0 + 8 * slot);
+            for (int b = 0; b < B; ++b) {
+                int rs;
+                int s;
+                if (is_layer) {
+                    uint32_t wx16[16][4];
+#pragma unroll
+                    for (int r = 0; r < 16; ++r) {
+                        const uint4 v = *reinterpret_cast<const uint4 *>(&S.wx[lr0 + r][lane * 16]);
+                        wx16[r][0] = v.x, wx16[r][1] = v.y, wx16[r][2] = v.z, wx16[r][3] = v.w;
+                    }
+                    s = dot16(wx16, S.codes_x[b], rs);
+                    if ((lane & 1) == 0) S.acc_x[par][b][lr0 + ((lane >> 1) & 15)] = s;
+                    if (tid == 0) S.meta_x[par][b].rs = rs;
+                } else {
+                    s = dot16(wr, S.codes_x[b], rs);
+                    if ((lane & 1) == 0 && o_n >= 0) {
+                        const RowMeta mt = S.meta_x[par][b];
+                        const qnn_qparams po = a.wo_p[0];
+                        const long long Sv = offset_product(s, mt.za, po.z, rs, o_cs, R);
+                        a.logits[((int64_t)b * T + t) * a.C + o_n] = __fadd_rn(recover_product(Sv, mt.Qa, po.Q), o_b);
                     }
                 }
             }
-            mbar_arrive_local(full0 + 8 * slot);
+            if (is_layer) mbar_arrive(axb0 + 8 * par);
+        };
+        if (!is_layer) {
+            for (int t = 0; t < T; ++t) {
+                x_phase(t);
+                named_bar(1, kPT);  // codes_x is rewritten next frame
+            }
+        } else {
+            if (T > 0) x_phase(0);
+            for (int t = 0; t < T; ++t) {
+                const int par = t & 1, pb = (t - 1) & 1;
+                if (t > 0) wait_cluster(a, hbar0 + 8 * pb, ((t - 1) >> 1) & 1);
+                // H phase: quantize h_{t-1} cooperatively, product with Wh
+                for (int b = 0; b < B; ++b) {
+                    float mn = FLT_MAX, mx = -FLT_MAX;
+#pragma unroll
+                    for (int s2 = 0; s2 < kMaxCS; ++s2)
+                        if (s2 < CS) {
+                            const float2 mm = S.hmm[pb][b][s2];
+                            mn = fminf(mn, mm.x);
+                            mx = fmaxf(mx, mm.y);
+                        }
+                    const qnn_qparams p = params_from_range(mn, mx);
+                    code_row(S.hbuf[pb][b], R, p, S.codes_h[b], tid);
+                    if (tid == 0) S.meta_h[par][b] = RowMeta{p.z, p.Q, 0, 0};
+                }
+                named_bar(1, kPT);
+                for (int b = 0; b < B; ++b) {
+                    int rs;
+                    const int s = dot16(wr, S.codes_h[b], rs);
+                    if ((lane & 1) == 0) S.acc_h[par][b][lr0 + ((lane >> 1) & 15)] = s;
+                    if (tid == 0) S.meta_h[par][b].rs = rs;
+                }
+                mbar_arrive(ahb0 + 8 * par);
+                // X phase of the next frame overlaps the cluster exchange of this one
+                if (t + 1 < T) x_phase(t + 1);
+            }
         }
     } else if (is_layer) {
-        // ---------------- LSTM layer compute warp ----------------
+        // ---------------- epilogue warps ----------------
         const SmallLayer &ly = a.layer[l];
-        const int j0 = (int)rank * kCellsPerBlock;
-        const int cell0 = j0 + 2 * warp;  // this warp's cells: cell0, cell0 + 1
-        // Wh rows (the recurrent critical path) in registers, Wx rows in shared memory
-        uint32_t whr[8][4];
-        load_rows(whr, ly.wh, ly.ldh, H, 0, cell0, 2, lane);
-        {
-            uint32_t tmp[8][4];
-            load_rows(tmp, ly.wx, ly.ldx, H, 0, cell0, 2, lane);
-            uint8_t *mine = swx + (size_t)warp * 8 * kMaxK;
-#pragma unroll
-            for (int r = 0; r < 8; ++r)
-                *reinterpret_cast<uint4 *>(mine + r * kMaxK + lane * 16) =
-                    make_uint4(tmp[r][0], tmp[r][1], tmp[r][2], tmp[r][3]);
-            __syncwarp();
-        }
-        const uint8_t *wx_rows = swx + (size_t)warp * 8 * kMaxK;
-        const int e = (lane >> 4) & 1, g = (lane >> 2) & 3;
-        const int j = cell0 + e;
+        const int et = tid - kPT;            // 0..127: local row 4c + g
+        const int cl = et >> 2, g = et & 3;  // cell within the block, gate
+        const int j = j0 + cl;
         const bool jv = j < H;
         const int64_t n = (int64_t)g * H + (jv ? j : 0);
         const int csx = jv ? ly.wx_sum[n] : 0, csh = jv ? ly.wh_sum[n] : 0;
         const float bias = jv ? ly.bias[n] : 0.0f;
         const qnn_qparams px = ly.wx_p[g], ph = ly.wh_p[g];
-        float c[kMaxB], yxb[kMaxB], hlast[kMaxB];
+        const int ew = warp - kPW;
+        const bool tag_out = (l < a.L - 1) || (a.C > 0);
+        float c[kMaxB], hl[kMaxB];
 #pragma unroll
         for (int b = 0; b < kMaxB; ++b) {
             c[b] = (b < B && jv) ? a.c0[((int64_t)l * B + b) * H + j] : 0.0f;
-            hlast[b] = 0.0f;
-            yxb[b] = 0.0f;
+            hl[b] = 0.0f;
         }
-        const bool tag_out = (l < a.L - 1) || (a.C > 0);
-        const uint32_t my_hbuf = saddr(hbuf);
-        for (int t = 0; t < T && ok; ++t) {
-            // X: input product of frame t
-            const int slot = t % kRing;
-            ok = wait_local(a, full0 + 8 * slot, (t / kRing) & 1);
-            if (!ok) break;
+        const uint32_t hbuf_l = saddr(&S.hbuf[0][0][0]), hmm_l = saddr(&S.hmm[0][0][0]);
+        for (int t = 0; t < T; ++t) {
+            const int par = t & 1;
+            wait_cta(a, axb0 + 8 * par, (t >> 1) & 1);
+            float yx[kMaxB];
 #pragma unroll
             for (int b = 0; b < kMaxB; ++b) {
                 if (b >= B) break;
-                const RowQ q = quantize_row_warp(ring + ((int64_t)slot * kMaxB + b) * kMaxK, kin, a);
-                uint32_t wx8[8][4];
-#pragma unroll
-                for (int r = 0; r < 8; ++r) {
-                    const uint4 v = *reinterpret_cast<const uint4 *>(wx_rows + r * kMaxK + lane * 16);
-                    wx8[r][0] = v.x, wx8[r][1] = v.y, wx8[r][2] = v.z, wx8[r][3] = v.w;
-                }
-                const int s = dot8_reduce(wx8, q);
-                const long long S = offset_product(s, q.za, px.z, q.rs, csx, kin);
-                yxb[b] = __fadd_rn(recover_product(S, q.Qa, px.Q), bias);
+                const RowMeta mt = S.meta_x[par][b];
+                const long long Sv = offset_product(S.acc_x[par][b][et], mt.za, px.z, mt.rs, csx, ly.kin);
+                yx[b] = __fadd_rn(recover_product(Sv, mt.Qa, px.Q), bias);
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive_local(empty0 + 8 * slot);
-            // H: wait for h_{t-1} from the whole cluster (h_{-1} was preloaded)
-            const int pb = (t - 1) & 1;
-            if (t > 0) {
-                ok = wait_cluster(a, hbar0 + 8 * pb, ((t - 1) >> 1) & 1);
-                if (!ok) break;
-            }
-            float hv[kMaxB];
+            wait_cta(a, ahb0 + 8 * par, (t >> 1) & 1);
 #pragma unroll
             for (int b = 0; b < kMaxB; ++b) {
-                hv[b] = 0.0f;
                 if (b >= B) break;
-                const RowQ q = quantize_row_warp(hbuf + ((int64_t)pb * kMaxB + b) * kMaxK, R, a);
-                const int s = dot8_reduce(whr, q);
-                const long long S = offset_product(s, q.za, ph.z, q.rs, csh, R);
-                const float pre = __fadd_rn(yxb[b], recover_product(S, q.Qa, ph.Q));
-                const int base = lane & 16;
-                const float pi = __shfl_sync(0xffffffffu, pre, base + 0);
-                const float pf = __shfl_sync(0xffffffffu, pre, base + 4);
-                const float pg = __shfl_sync(0xffffffffu, pre, base + 8);
-                const float po = __shfl_sync(0xffffffffu, pre, base + 12);
+                const RowMeta mt = S.meta_h[par][b];
+                const long long Sv = offset_product(S.acc_h[par][b][et], mt.za, ph.z, mt.rs, csh, R);
+                const float pre = __fadd_rn(yx[b], recover_product(Sv, mt.Qa, ph.Q));
+                const int q0 = lane & ~3;
+                const float pi = __shfl_sync(0xffffffffu, pre, q0 + 0);
+                const float pf = __shfl_sync(0xffffffffu, pre, q0 + 1);
+                const float pg = __shfl_sync(0xffffffffu, pre, q0 + 2);
+                const float po = __shfl_sync(0xffffffffu, pre, q0 + 3);
                 float m;
                 lstm_cell(pi, pf, pg, po, c[b], m);
-                hv[b] = jv ? m : 0.0f;
-                hlast[b] = hv[b];
-            }
-            // send h_t: lane d < CS delivers both cells' values to block d of the cluster
-            const int cb = t & 1;
-#pragma unroll
-            for (int b = 0; b < kMaxB; ++b) {
-                if (b >= B) break;
-                const float v0 = __shfl_sync(0xffffffffu, hv[b], 0);
-                const float v1 = __shfl_sync(0xffffffffu, hv[b], 16);
-                if (lane < CS && cell0 < H) {
-                    const uint32_t raddr =
-                        map_rank(my_hbuf + 4u * (uint32_t)(((cb * kMaxB + b) * kMaxK) + cell0), (uint32_t)lane);
-                    st_cluster_f32x2(raddr, v0, v1);
-                }
-                // outputs to global: lanes 0 and 16 own cell0 and cell0 + 1
-                if ((lane & 15) == 0 && jv) {
+                const float h = jv ? m : 0.0f;
+                hl[b] = h;
+                if (g == 0) S.hloc[par][b][cl] = h;
+                const float mn = warp_min(jv ? h : FLT_MAX), mx = warp_max(jv ? h : -FLT_MAX);
+                if (lane == 0) S.emm[par][b][ew] = make_float2(mn, mx);
+                if (g == 0 && jv) {
                     const int64_t o = (((int64_t)l * B + b) * T + t) * R + j;
-                    if (tag_out)
-                        st_tag(a.hx + o, ((unsigned long long)a.epoch << 32) | __float_as_uint(hv[b]));
-                    if (a.h_all) a.h_all[o] = hv[b];
-                    if (a.ytop && l == a.L - 1) a.ytop[((int64_t)b * T + t) * R + j] = hv[b];
+                    if (tag_out) st_tag(a.hx + o, ((unsigned long long)a.epoch << 32) | __float_as_uint(h));
+                    if (a.h_all) a.h_all[o] = h;
+                    if (a.ytop && l == a.L - 1) a.ytop[((int64_t)b * T + t) * R + j] = h;
                 }
             }
-            if (lane < CS) mbar_arrive_remote(map_rank(hbar0 + 8 * cb, (uint32_t)lane));
+            named_bar(2, kET);
+            // the first epilogue warp sends this block's 32 values and their range to every block
+            if (ew == 0 && lane < CS) {
+                for (int b = 0; b < B; ++b) {
+                    float mn = FLT_MAX, mx = -FLT_MAX;
+#pragma unroll
+                    for (int w = 0; w < kEW; ++w) {
+                        const float2 mm = S.emm[par][b][w];
+                        mn = fminf(mn, mm.x);
+                        mx = fmaxf(mx, mm.y);
+                    }
+                    const uint32_t dst = map_rank(hbuf_l + 4u * (uint32_t)((par * kMaxB + b) * kMaxK + j0), lane);
+#pragma unroll
+                    for (int q = 0; q < kCellsPerBlock / 4; ++q)
+                        st_cluster_v4(dst + 16u * q, *reinterpret_cast<const float4 *>(&S.hloc[par][b][4 * q]));
+                    st_cluster_v2(map_rank(hmm_l + 8u * (uint32_t)((par * kMaxB + b) * kMaxCS + rank), lane), mn, mx);
+                }
+                mbar_arrive_remote(map_rank(hbar0 + 8 * par, lane));
+            }
         }
-        if (ok && (lane & 15) == 0 && jv) {
+        if (g == 0 && jv) {
 #pragma unroll
             for (int b = 0; b < kMaxB; ++b) {
                 if (b >= B) break;
-                if (a.h_fin) a.h_fin[((int64_t)l * B + b) * R + j] = hlast[b];
+                if (a.h_fin) a.h_fin[((int64_t)l * B + b) * R + j] = hl[b];
                 if (a.c_fin) a.c_fin[((int64_t)l * B + b) * H + j] = c[b];
             }
-        }
-    } else {
-        // ---------------- output layer compute warp ----------------
-        const int ob = (cid - a.L) * CS + (int)rank;
-        const int n0 = ob * kOutRowsPerBlock + warp * 8;
-        const int nv = a.C - n0 < 8 ? (a.C - n0 < 0 ? 0 : a.C - n0) : 8;
-        uint32_t wor[8][4];
-        load_rows(wor, a.wo, a.ldo, 0, 1, n0, nv, lane);
-        const int r = (lane >> 2) & 7;
-        const int n = n0 + r;
-        const bool nvld = r < nv;
-        const int cso = nvld ? a.wo_sum[n] : 0;
-        const float bo = nvld ? a.bo[n] : 0.0f;
-        const qnn_qparams po = a.wo_p[0];
-        for (int t = 0; t < T && ok; ++t) {
-            const int slot = t % kRing;
-            ok = wait_local(a, full0 + 8 * slot, (t / kRing) & 1);
-            if (!ok) break;
-#pragma unroll
-            for (int b = 0; b < kMaxB; ++b) {
-                if (b >= B) break;
-                const RowQ q = quantize_row_warp(ring + ((int64_t)slot * kMaxB + b) * kMaxK, R, a);
-                const int s = dot8_reduce(wor, q);
-                const long long S = offset_product(s, q.za, po.z, q.rs, cso, R);
-                const float y = __fadd_rn(recover_product(S, q.Qa, po.Q), bo);
-                if ((lane & 3) == 0 && nvld) a.logits[((int64_t)b * T + t) * a.C + n] = y;
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive_local(empty0 + 8 * slot);
         }
     }
     __syncwarp();
@@ -558,15 +608,14 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
                               float *c_state, float *h_all, cudaStream_t st, bool *used) {
     *used = false;
     const int64_t L = m->L, I = m->I, H = m->H, C = m->C, R = m->R;
-    if (m->P != 0 || B > kMaxB || L > kMaxLayers || I > kMaxK || R > kMaxK || H > kCellsPerBlock * 16) return QNN_OK;
+    if (m->P != 0 || B > kMaxB || L > kMaxLayers || I > kMaxK || R > kMaxK || H > kCellsPerBlock * kMaxCS) return QNN_OK;
     if (C > 0 && m->d.output_mode != QNN_OUT_QUANT) return QNN_OK;
     if (T > (int64_t)INT32_MAX / 4) return QNN_OK;
     const int CS = (int)((H + kCellsPerBlock - 1) / kCellsPerBlock);
-    const int out_blocks = C > 0 ? (int)((C + kOutRowsPerBlock - 1) / kOutRowsPerBlock) : 0;
+    const int out_blocks = C > 0 ? (int)((C + kRows - 1) / kRows) : 0;
     const int out_clusters = (out_blocks + CS - 1) / CS;
     const int clusters = (int)L + out_clusters;
-    const size_t smem = sizeof(float) * (2 + kRing) * kMaxB * kMaxK + (size_t)8 * kSW * kMaxK +
-                        sizeof(uint64_t) * (2 * kRing + 2);
+    const size_t smem = sizeof(Smem);
 
     int dev = 0;
     QNN_CUDA_TRY(cudaGetDevice(&dev));
@@ -594,7 +643,7 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
     }
     if (max_clusters < clusters) return QNN_OK;  // cannot be co-resident: layer-by-layer path
 
-    // workspace: staging, tagged layer outputs, logits, zero state
+    // workspace: staging, tagged layer outputs, logits, state
     const bool x_dev = is_device_ptr(x), y_dev = is_device_ptr(y);
     const bool hs_dev = h_state && is_device_ptr(h_state), cs_dev = c_state && is_device_ptr(c_state);
     const bool ha_dev = h_all && is_device_ptr(h_all);
