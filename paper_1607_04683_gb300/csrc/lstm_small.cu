@@ -38,12 +38,14 @@
 namespace qnn {
 namespace {
 
-constexpr int kPW = 8;                        // product warps
+constexpr int kPW = 16;                       // product warps
 constexpr int kEW = 4;                        // epilogue warps
-constexpr int kPT = kPW * 32;                 // product threads (256)
+constexpr int kPT = kPW * 32;                 // product threads (512)
 constexpr int kET = kEW * 32;                 // epilogue threads (128)
-constexpr int kLoaderWarp = kPW + kEW;        // warp 12
-constexpr int kSThreads = (kPW + kEW + 1) * 32;  // 416
+constexpr int kLoaderWarp = kPW + kEW;        // warp 20
+constexpr int kSThreads = (kPW + kEW + 1) * 32;  // 672
+constexpr int kRowsPW = 8;                    // local rows per product warp
+constexpr int kRowShift = 2;                  // after the warp reduction lane l holds row (l >> 2) & 7
 constexpr int kRing = 4;                      // input ring depth (frames)
 constexpr int kMaxB = 4;                      // batch limit of this path
 constexpr int kMaxK = 512;                    // 16 bytes of every weight row per lane
@@ -53,6 +55,11 @@ constexpr int kMaxCS = 16;
 constexpr int kMaxLayers = 8;
 constexpr unsigned long long kWaitNs = 2000000000ull;
 constexpr int kSpinCheck = 512;               // polls between checks of the clock and the abort flag
+constexpr int kHBytes = kCellsPerBlock * 4 + 8;  // one block's h values of one row and their range
+// Product warps start the next frame's input product only after the epilogue has finished its
+// gate arithmetic (instead of right after handing over the recurrent sums), so that the two do
+// not compete for issue slots on the recurrent critical path.
+constexpr bool kXAfterEpilogue = true;
 
 struct SmallLayer {
     const uint8_t *wx;
@@ -108,7 +115,7 @@ struct Smem {
     float hloc[2][kMaxB][kCellsPerBlock];  // this block's new h values
     float2 emm[2][kMaxB][kEW];           // epilogue warps' ranges
     uint8_t wx[kRows][kMaxK];            // Wx rows of this block (local row order)
-    unsigned long long bar_full[kRing], bar_empty[kRing], bar_h[2], bar_ax[2], bar_ah[2];
+    unsigned long long bar_full[kRing], bar_empty[kRing], bar_h[2], bar_ax[2], bar_ah[2], bar_ep[2];
 };
 
 // ---- PTX helpers --------------------------------------------------------------------------------
@@ -150,16 +157,23 @@ __device__ __forceinline__ uint32_t map_rank(uint32_t local, uint32_t rank) {
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
     return r;
 }
-__device__ __forceinline__ void st_cluster_v4(uint32_t raddr, float4 v) {
-    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(raddr), "f"(v.x), "f"(v.y), "f"(v.z),
-                 "f"(v.w)
+// Asynchronous stores into a peer block's shared memory; each completes `bytes` of the peer's
+// mbarrier transaction count when its data has landed (no fence needed by the sender).
+__device__ __forceinline__ void st_async_v4(uint32_t raddr, float4 v, uint32_t rbar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                     raddr),
+                 "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
                  : "memory");
 }
-__device__ __forceinline__ void st_cluster_v2(uint32_t raddr, float a, float b) {
-    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(raddr), "f"(a), "f"(b) : "memory");
+__device__ __forceinline__ void st_async_v2(uint32_t raddr, float a, float b, uint32_t rbar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(raddr),
+                 "f"(a), "f"(b), "r"(rbar)
+                 : "memory");
 }
-__device__ __forceinline__ void mbar_arrive_remote(uint32_t raddr) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(raddr) : "memory");
+// Arrive on a local mbarrier and add `bytes` to the transaction count its phase waits for.
+__device__ __forceinline__ void mbar_arrive_expect(uint32_t bar, uint32_t bytes) {
+    asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}" ::"r"(bar), "r"(bytes)
+                 : "memory");
 }
 __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
@@ -217,19 +231,22 @@ __device__ __forceinline__ void wait_cluster(const SmallArgs &a, uint32_t bar, u
 
 // ---- product warps ------------------------------------------------------------------------------
 
-// Codes of two values per product thread (k = tid, tid + 256 < len) into `codes` (eq. 2 with the
-// unit's range already known). Zero past len.
+// Code of one value per product thread (k = tid < len) into `codes` (eq. 2 with the unit's range
+// already known). Zero past len.
 __device__ __forceinline__ void code_row(const float *row, int len, const qnn_qparams &p, uint8_t *codes, int tid) {
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kMaxK / kPT; ++i) {
         const int k = tid + i * kPT;
         codes[k] = k < len ? (uint8_t)quant_code(row[k], p.Q, p.z) : (uint8_t)0;
     }
 }
 
-// Sixteen row partial dot products of this lane (16 rows x 16 bytes), summed across the warp so
-// that lane l ends with the full sum of local row ((l >> 1) & 15). Also returns the row code sum.
-__device__ __forceinline__ int dot16(const uint32_t (&w)[16][4], const uint8_t *codes, int &rs) {
+// Eight row partial dot products of this lane (8 rows x 16 bytes), summed across the warp so that
+// lane l ends with the full sum of local row ((l >> 2) & 7). Also returns the row code sum.
+// `row(r)` yields this lane's 16 bytes of local row r (from registers or shared memory; a row is
+// fetched only when it is multiplied, so shared-memory rows never occupy registers all at once).
+template <typename RowBytes>
+__device__ __forceinline__ int dot8(RowBytes row, const uint8_t *codes, int &rs) {
     const int lane = threadIdx.x & 31;
     const uint4 cv = *reinterpret_cast<const uint4 *>(codes + lane * 16);
     const uint32_t c[4] = {cv.x, cv.y, cv.z, cv.w};
@@ -237,35 +254,41 @@ __device__ __forceinline__ int dot16(const uint32_t (&w)[16][4], const uint8_t *
 #pragma unroll
     for (int i = 0; i < 4; ++i) bs = __dp4a(c[i], 0x01010101u, bs);
     rs = warp_sum((int)bs);
-    int v[16];
+    int v[kRowsPW];
 #pragma unroll
-    for (int r = 0; r < 16; ++r) {
-        unsigned acc = 0;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) acc = __dp4a(w[r][i], c[i], acc);
+    for (int r = 0; r < kRowsPW; ++r) {
+        const uint4 w = row(r);
+        unsigned acc = __dp4a(w.x, c[0], 0u);
+        acc = __dp4a(w.y, c[1], acc);
+        acc = __dp4a(w.z, c[2], acc);
+        acc = __dp4a(w.w, c[3], acc);
         v[r] = (int)acc;
     }
 #pragma unroll
-    for (int s = 4; s >= 1; --s) {  // halve the live rows at each exchange: 8, 4, 2, 1
-        const int half = 1 << (s - 1);
-        const bool up = (lane >> s) & 1;
+    for (int s = 4; s >= 2; --s) {  // halve the live rows at each exchange: 4, 2, 1
+        const int half = kRowsPW >> (5 - s);
+        // choose with bit masks, not a conditional: a select between two array elements can be
+        // compiled into an indexed access, which would put v[] in local memory
+        const int up = -((lane >> s) & 1);
 #pragma unroll
         for (int i = 0; i < half; ++i) {
-            const int send = up ? v[i] : v[i + half];
-            const int keep = up ? v[i + half] : v[i];
+            const int send = (v[i] & up) | (v[i + half] & ~up);
+            const int keep = (v[i + half] & up) | (v[i] & ~up);
             v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 1 << s);
         }
     }
-    return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
+    int s = v[0] + __shfl_xor_sync(0xffffffffu, v[0], 2);
+    return s + __shfl_xor_sync(0xffffffffu, s, 1);
 }
 
-// Loads 16 local rows into registers; local row lr maps to a global row through row_of(lr)
-// (negative: absent, zero codes).
+// Loads a product warp's local rows into registers; local row lr maps to a global row through
+// row_of(lr) (negative: absent, zero codes).
 template <typename RowOf>
-__device__ __forceinline__ void load_rows16(uint32_t (&w)[16][4], const uint8_t *base, int ld, int first, RowOf row_of) {
+__device__ __forceinline__ void load_rows(uint32_t (&w)[kRowsPW][4], const uint8_t *base, int ld, int first,
+                                          RowOf row_of) {
     const int lane = threadIdx.x & 31;
 #pragma unroll
-    for (int r = 0; r < 16; ++r) {
+    for (int r = 0; r < kRowsPW; ++r) {
         const int64_t row = row_of(first + r);
         uint4 v = make_uint4(0, 0, 0, 0);
         if (row >= 0 && lane * 16 < ld) v = *reinterpret_cast<const uint4 *>(base + row * ld + lane * 16);
@@ -296,11 +319,16 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
             mbar_init(empty0 + 8 * i, 1);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(hbar0 + 8 * i, CS);
-            mbar_init(axb0 + 8 * i, kPT);
-            mbar_init(ahb0 + 8 * i, kPT);
+            mbar_init(hbar0 + 8 * i, 1);  // one local arrival (with the expected bytes) per phase
+            mbar_init(axb0 + 8 * i, kPW);
+            mbar_init(ahb0 + 8 * i, kPW);
+            mbar_init(saddr(&S.bar_ep[i]), kEW);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        if (is_layer) {  // frames 0 and 1: every block of the cluster sends B x (32 values + range)
+            mbar_arrive_expect(hbar0, (uint32_t)(CS * B * kHBytes));
+            mbar_arrive_expect(hbar0 + 8, (uint32_t)(CS * B * kHBytes));
+        }
     }
     if (is_layer) {
         // h_{-1} of the whole layer into hbuf[1]; its range into every source slot of hmm[1]
@@ -398,23 +426,25 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
         }
     } else if (warp < kPW) {
         // ---------------- product warps ----------------
-        const int lr0 = warp * 16;  // local rows lr0 .. lr0 + 15
-        uint32_t wr[16][4];
+        const int lr0 = warp * kRowsPW;  // local rows lr0 .. lr0 + 7
+        const int my_row = lr0 + ((lane >> kRowShift) & (kRowsPW - 1));  // row this lane ends with
+        const bool row_writer = (lane & ((1 << kRowShift) - 1)) == 0;
+        uint32_t wr[kRowsPW][4];
         if (is_layer) {
             const SmallLayer &ly = a.layer[l];
-            load_rows16(wr, ly.wh, ly.ldh, lr0, [&](int lr) -> int64_t {
+            load_rows(wr, ly.wh, ly.ldh, lr0, [&](int lr) -> int64_t {
                 const int j = j0 + lr / 4;
                 return j < H ? (int64_t)(lr % 4) * H + j : -1;
             });
         } else {
             const int nb = ((cid - a.L) * CS + (int)rank) * kRows;
-            load_rows16(wr, a.wo, a.ldo, lr0, [&](int lr) -> int64_t { return nb + lr < a.C ? nb + lr : -1; });
+            load_rows(wr, a.wo, a.ldo, lr0, [&](int lr) -> int64_t { return nb + lr < a.C ? nb + lr : -1; });
         }
-        // output-layer epilogue constants (product lanes hold row lr0 + ((lane >> 1) & 15))
+        // output-layer epilogue constants of my_row
         int o_cs = 0, o_n = -1;
         float o_b = 0.0f;
         if (!is_layer) {
-            const int n = ((cid - a.L) * CS + (int)rank) * kRows + lr0 + ((lane >> 1) & 15);
+            const int n = ((cid - a.L) * CS + (int)rank) * kRows + my_row;
             if (n < a.C) {
                 o_n = n;
                 o_cs = a.wo_sum[n];
@@ -444,18 +474,14 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 int rs;
                 int s;
                 if (is_layer) {
-                    uint32_t wx16[16][4];
-#pragma unroll
-                    for (int r = 0; r < 16; ++r) {
-                        const uint4 v = *reinterpret_cast<const uint4 *>(&S.wx[lr0 + r][lane * 16]);
-                        wx16[r][0] = v.x, wx16[r][1] = v.y, wx16[r][2] = v.z, wx16[r][3] = v.w;
-                    }
-                    s = dot16(wx16, S.codes_x[b], rs);
-                    if ((lane & 1) == 0) S.acc_x[par][b][lr0 + ((lane >> 1) & 15)] = s;
+                    s = dot8([&](int r) { return *reinterpret_cast<const uint4 *>(&S.wx[lr0 + r][lane * 16]); },
+                              S.codes_x[b], rs);
+                    if (row_writer) S.acc_x[par][b][my_row] = s;
                     if (tid == 0) S.meta_x[par][b].rs = rs;
                 } else {
-                    s = dot16(wr, S.codes_x[b], rs);
-                    if ((lane & 1) == 0 && o_n >= 0) {
+                    s = dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
+                              S.codes_x[b], rs);
+                    if (row_writer && o_n >= 0) {
                         const RowMeta mt = S.meta_x[par][b];
                         const qnn_qparams po = a.wo_p[0];
                         const long long Sv = offset_product(s, mt.za, po.z, rs, o_cs, R);
@@ -463,7 +489,10 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                     }
                 }
             }
-            if (is_layer) mbar_arrive(axb0 + 8 * par);
+            if (is_layer) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(axb0 + 8 * par);
+            }
         };
         if (!is_layer) {
             for (int t = 0; t < T; ++t) {
@@ -474,7 +503,11 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
             if (T > 0) x_phase(0);
             for (int t = 0; t < T; ++t) {
                 const int par = t & 1, pb = (t - 1) & 1;
-                if (t > 0) wait_cluster(a, hbar0 + 8 * pb, ((t - 1) >> 1) & 1);
+                if (t > 0) {
+                    wait_cluster(a, hbar0 + 8 * pb, ((t - 1) >> 1) & 1);
+                    // re-arm this buffer's barrier for frame t + 1 (its senders need our frame t first)
+                    if (tid == 0 && t + 1 < T) mbar_arrive_expect(hbar0 + 8 * pb, (uint32_t)(CS * B * kHBytes));
+                }
                 // H phase: quantize h_{t-1} cooperatively, product with Wh
                 for (int b = 0; b < B; ++b) {
                     float mn = FLT_MAX, mx = -FLT_MAX;
@@ -492,12 +525,16 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 named_bar(1, kPT);
                 for (int b = 0; b < B; ++b) {
                     int rs;
-                    const int s = dot16(wr, S.codes_h[b], rs);
-                    if ((lane & 1) == 0) S.acc_h[par][b][lr0 + ((lane >> 1) & 15)] = s;
+                    const int s =
+                        dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
+                              S.codes_h[b], rs);
+                    if (row_writer) S.acc_h[par][b][my_row] = s;
                     if (tid == 0) S.meta_h[par][b].rs = rs;
                 }
-                mbar_arrive(ahb0 + 8 * par);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(ahb0 + 8 * par);
                 // X phase of the next frame overlaps the cluster exchange of this one
+                if (kXAfterEpilogue) wait_cta(a, saddr(&S.bar_ep[par]), (t >> 1) & 1);
                 if (t + 1 < T) x_phase(t + 1);
             }
         }
@@ -549,7 +586,13 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 const float h = jv ? m : 0.0f;
                 hl[b] = h;
                 if (g == 0) S.hloc[par][b][cl] = h;
-                const float mn = warp_min(jv ? h : FLT_MAX), mx = warp_max(jv ? h : -FLT_MAX);
+                // range of the warp's 8 cells (the four lanes of a quad hold the same value)
+                float mn = jv ? h : FLT_MAX, mx = jv ? h : -FLT_MAX;
+#pragma unroll
+                for (int o = 4; o < 32; o <<= 1) {
+                    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+                    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+                }
                 if (lane == 0) S.emm[par][b][ew] = make_float2(mn, mx);
                 if (g == 0 && jv) {
                     const int64_t o = (((int64_t)l * B + b) * T + t) * R + j;
@@ -558,9 +601,14 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                     if (a.ytop && l == a.L - 1) a.ytop[((int64_t)b * T + t) * R + j] = h;
                 }
             }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(saddr(&S.bar_ep[par]));  // gate arithmetic of frame t done
             named_bar(2, kET);
             // the first epilogue warp sends this block's 32 values and their range to every block
-            if (ew == 0 && lane < CS) {
+            // of the cluster (lane d -> block d); the stores complete on the peer's barrier. The
+            // last frame's values are not sent: no block waits for them (nothing is in flight at exit).
+            if (ew == 0 && lane < CS && t + 1 < T) {
+                const uint32_t rbar = map_rank(hbar0 + 8 * par, lane);
                 for (int b = 0; b < B; ++b) {
                     float mn = FLT_MAX, mx = -FLT_MAX;
 #pragma unroll
@@ -572,10 +620,10 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                     const uint32_t dst = map_rank(hbuf_l + 4u * (uint32_t)((par * kMaxB + b) * kMaxK + j0), lane);
 #pragma unroll
                     for (int q = 0; q < kCellsPerBlock / 4; ++q)
-                        st_cluster_v4(dst + 16u * q, *reinterpret_cast<const float4 *>(&S.hloc[par][b][4 * q]));
-                    st_cluster_v2(map_rank(hmm_l + 8u * (uint32_t)((par * kMaxB + b) * kMaxCS + rank), lane), mn, mx);
+                        st_async_v4(dst + 16u * q, *reinterpret_cast<const float4 *>(&S.hloc[par][b][4 * q]), rbar);
+                    st_async_v2(map_rank(hmm_l + 8u * (uint32_t)((par * kMaxB + b) * kMaxCS + rank), lane), mn, mx,
+                                rbar);
                 }
-                mbar_arrive_remote(map_rank(hbar0 + 8 * par, lane));
             }
         }
         if (g == 0 && jv) {
@@ -588,6 +636,10 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
         }
     }
     __syncwarp();
+    // After an aborted run some waits returned early; give peer stores still in flight time to
+    // land (they take microseconds) before any block of the cluster can leave.
+    if (*(volatile int *)a.abort_flag)
+        for (int i = 0; i < 100; ++i) __nanosleep(100000);
     // no block leaves while a cluster peer may still write into its shared memory
     cluster_sync();
 }
