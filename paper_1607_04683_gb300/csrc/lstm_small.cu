@@ -5,22 +5,24 @@
 // cluster owns cells [32 r, 32 r + 32): the 128 gate rows (cell c, gate g -> local row 4 c + g)
 // of Wx and Wh. The softmax layer's 8-bit product runs in further clusters, 128 rows of Wo per
 // block. A block has three kinds of warps:
-//   8 product warps   16 local rows each; Wh (or Wo) rows in registers, lane l holding bytes
-//                     [16 l, 16 l + 16) of each row (so K <= 512), Wx rows in shared memory.
+//   16 product warps  8 local rows each, dp4a (u8 x u8 -> s32) reduced across the warp; Wh (or
+//                     Wo) rows in registers, lane l holding bytes [16 l, 16 l + 16) of each row (so
+//                     K <= 512), Wx rows in shared memory.
 //   4 epilogue warps  one thread per (cell, gate): recovery, bias, gate nonlinearity, and in the
 //                     first lane of each quad the cell update (c stays in that register).
 //   1 loader warp     brings each frame's input row into a shared-memory ring: x_t for the first
 //                     layer, otherwise the previous layer's h_t, polled from global memory where
 //                     it is written tagged with the launch's epoch; it also finds the row's range.
 // Per frame t of a layer block:
-//   X  the product warps quantize the input row cooperatively (two values per thread, eq. 2 with
-//      the loader's range), multiply with Wx (dp4a, u8 x u8 -> s32, reduced across the warp) and
-//      hand the int32 sums to the epilogue warps (mbarrier).
-//   H  they wait until every block of the cluster has delivered its 32 values of h_{t-1} and their
-//      range (distributed shared memory stores + one remote mbarrier arrival per block), quantize
-//      h_{t-1} cooperatively, multiply with Wh and hand the sums over.
-//   E  the epilogue warps apply eq. 1's offsets, recover, add the bias, apply the gates and the
-//      cell update, then send the block's 32 new h values and their range to every block of the
+//   X  the product warps quantize the input row cooperatively (one value per thread, eq. 2 with
+//      the parameters the loader computed), multiply with Wx and hand the int32 partial sums to
+//      the epilogue warps (mbarrier).
+//   H  they wait until every epilogue warp of the cluster has delivered its 8 values of h_{t-1}
+//      and their range (st.async into distributed shared memory, completing on a transaction-count
+//      mbarrier), quantize h_{t-1} cooperatively, multiply with Wh and hand the sums over; then
+//      they start the input product of frame t + 1 while the epilogue works on frame t.
+//   E  the epilogue warps apply eq. 1's offsets, recover, add the bias, apply
+//      the gates and the cell update, send their new h values and range to every block of the
 //      cluster, and write them tagged to global memory for the next layer.
 // A layer's recurrence only waits on its own cluster; consecutive layers run one frame apart. Every
 // wait is bounded in time: one that gives up records QNN_ERR_TIMEOUT and raises an abort flag,
@@ -55,11 +57,12 @@ constexpr int kMaxCS = 16;
 constexpr int kMaxLayers = 8;
 constexpr unsigned long long kWaitNs = 2000000000ull;
 constexpr int kSpinCheck = 512;               // polls between checks of the clock and the abort flag
-constexpr int kHBytes = kCellsPerBlock * 4 + 8;  // one block's h values of one row and their range
-// Product warps start the next frame's input product only after the epilogue has finished its
-// gate arithmetic (instead of right after handing over the recurrent sums), so that the two do
-// not compete for issue slots on the recurrent critical path.
-constexpr bool kXAfterEpilogue = true;
+constexpr int kHParts = kMaxCS * kEW;          // range partials per row: one per epilogue warp of the cluster
+constexpr int kHBytes = 8 * 4 + 8;             // one epilogue warp's 8 h values of one row and their range
+// Whether product warps wait for the epilogue's gate arithmetic before the next frame's input
+// product (less contention on the critical path) or start it at once (overlap). Measured on
+// GB300 with the 5 x 500 stack: overlapping is faster (2.1 vs 2.8 us per frame).
+constexpr bool kXAfterEpilogue = false;
 
 struct SmallLayer {
     const uint8_t *wx;
@@ -103,17 +106,14 @@ struct RowMeta {  // quantized activation row: offset, scale, code sum
 
 struct Smem {
     float hbuf[2][kMaxB][kMaxK];        // h_{t} of the whole layer, by frame parity (cluster writes)
-    float2 hmm[2][kMaxB][kMaxCS];       // per source block: range of its 32 values
+    float2 hmm[2][kMaxB][kHParts];      // per source epilogue warp: range of its 8 values
     float ring[kRing][kMaxB][kMaxK];    // input rows (loader writes)
-    float2 ring_mm[kRing][kMaxB];       // their ranges
-    int ring_bad[kRing][kMaxB];         // non-finite flag
+    qnn_qparams ring_p[kRing][kMaxB];   // their quantization parameters (loader computes them)
     uint8_t codes_x[kMaxB][kMaxK];      // quantized input rows of the current frame
     uint8_t codes_h[kMaxB][kMaxK];      // quantized h_{t-1}
-    int acc_x[2][kMaxB][kRows];         // int32 sums, by frame parity
+    int acc_x[2][kMaxB][kRows];         // int32 sums [frame parity][seq][row]
     int acc_h[2][kMaxB][kRows];
     RowMeta meta_x[2][kMaxB], meta_h[2][kMaxB];
-    float hloc[2][kMaxB][kCellsPerBlock];  // this block's new h values
-    float2 emm[2][kMaxB][kEW];           // epilogue warps' ranges
     uint8_t wx[kRows][kMaxK];            // Wx rows of this block (local row order)
     unsigned long long bar_full[kRing], bar_empty[kRing], bar_h[2], bar_ax[2], bar_ah[2], bar_ep[2];
 };
@@ -245,6 +245,8 @@ __device__ __forceinline__ void code_row(const float *row, int len, const qnn_qp
 // lane l ends with the full sum of local row ((l >> 2) & 7). Also returns the row code sum.
 // `row(r)` yields this lane's 16 bytes of local row r (from registers or shared memory; a row is
 // fetched only when it is multiplied, so shared-memory rows never occupy registers all at once).
+// (dp4a rather than the warp-level integer MMA: on this GPU the two have the same peak rate, and
+// with one to four activation rows the MMA's eight columns would be mostly wasted.)
 template <typename RowBytes>
 __device__ __forceinline__ int dot8(RowBytes row, const uint8_t *codes, int &rs) {
     const int lane = threadIdx.x & 31;
@@ -326,8 +328,8 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         if (is_layer) {  // frames 0 and 1: every block of the cluster sends B x (32 values + range)
-            mbar_arrive_expect(hbar0, (uint32_t)(CS * B * kHBytes));
-            mbar_arrive_expect(hbar0 + 8, (uint32_t)(CS * B * kHBytes));
+            mbar_arrive_expect(hbar0, (uint32_t)(CS * kEW * B * kHBytes));
+            mbar_arrive_expect(hbar0 + 8, (uint32_t)(CS * kEW * B * kHBytes));
         }
     }
     if (is_layer) {
@@ -345,7 +347,7 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
             }
             mn = warp_min(mn);
             mx = warp_max(mx);
-            if (lane < kMaxCS) S.hmm[1][warp][lane] = make_float2(mn, mx);
+            for (int i = lane; i < kHParts; i += 32) S.hmm[1][warp][i] = make_float2(mn, mx);
         }
         // Wx rows of this block, local row 4c + g <- global row g H + j0 + c
         const SmallLayer &ly = a.layer[l];
@@ -417,10 +419,12 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 mn = warp_min(mn);
                 mx = warp_max(mx);
                 bad = __any_sync(0xffffffffu, bad);
-                if (lane == 0) {
-                    S.ring_mm[slot][b] = make_float2(mn, mx);
-                    S.ring_bad[slot][b] = bad ? 1 : 0;
+                if (bad) {
+                    if (lane == 0) record_status(a.status, QNN_ERR_NONFINITE);
+                    mn = 0.0f;
+                    mx = 0.0f;
                 }
+                if (lane == 0) S.ring_p[slot][b] = params_from_range(mn, mx);  // the row's unit (eq. 2)
             }
             mbar_arrive(full0 + 8 * slot);
         }
@@ -457,14 +461,7 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
             const int slot = t % kRing, par = t & 1;
             wait_cta(a, full0 + 8 * slot, (t / kRing) & 1);
             for (int b = 0; b < B; ++b) {
-                const float2 mm = S.ring_mm[slot][b];
-                float mn = mm.x, mx = mm.y;
-                if (S.ring_bad[slot][b]) {
-                    if (tid == 0) record_status(a.status, QNN_ERR_NONFINITE);
-                    mn = 0.0f;
-                    mx = 0.0f;
-                }
-                const qnn_qparams p = params_from_range(mn, mx);
+                const qnn_qparams p = S.ring_p[slot][b];
                 code_row(S.ring[slot][b], kin, p, S.codes_x[b], tid);
                 if (tid == 0) S.meta_x[par][b] = RowMeta{p.z, p.Q, 0, 0};
             }
@@ -475,12 +472,12 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 int s;
                 if (is_layer) {
                     s = dot8([&](int r) { return *reinterpret_cast<const uint4 *>(&S.wx[lr0 + r][lane * 16]); },
-                              S.codes_x[b], rs);
+                             S.codes_x[b], rs);
                     if (row_writer) S.acc_x[par][b][my_row] = s;
                     if (tid == 0) S.meta_x[par][b].rs = rs;
                 } else {
                     s = dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
-                              S.codes_x[b], rs);
+                             S.codes_x[b], rs);
                     if (row_writer && o_n >= 0) {
                         const RowMeta mt = S.meta_x[par][b];
                         const qnn_qparams po = a.wo_p[0];
@@ -506,18 +503,24 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 if (t > 0) {
                     wait_cluster(a, hbar0 + 8 * pb, ((t - 1) >> 1) & 1);
                     // re-arm this buffer's barrier for frame t + 1 (its senders need our frame t first)
-                    if (tid == 0 && t + 1 < T) mbar_arrive_expect(hbar0 + 8 * pb, (uint32_t)(CS * B * kHBytes));
+                    if (tid == 0 && t + 1 < T)
+                        mbar_arrive_expect(hbar0 + 8 * pb, (uint32_t)(CS * kEW * B * kHBytes));
                 }
                 // H phase: quantize h_{t-1} cooperatively, product with Wh
                 for (int b = 0; b < B; ++b) {
+                    // range of the row: lane i folds partials i and i + 32, then the warp reduces
                     float mn = FLT_MAX, mx = -FLT_MAX;
 #pragma unroll
-                    for (int s2 = 0; s2 < kMaxCS; ++s2)
-                        if (s2 < CS) {
-                            const float2 mm = S.hmm[pb][b][s2];
+                    for (int q = 0; q < kHParts / 32; ++q) {
+                        const int i = lane + 32 * q;
+                        if (i < CS * kEW) {
+                            const float2 mm = S.hmm[pb][b][i];
                             mn = fminf(mn, mm.x);
                             mx = fmaxf(mx, mm.y);
                         }
+                    }
+                    mn = warp_min(mn);
+                    mx = warp_max(mx);
                     const qnn_qparams p = params_from_range(mn, mx);
                     code_row(S.hbuf[pb][b], R, p, S.codes_h[b], tid);
                     if (tid == 0) S.meta_h[par][b] = RowMeta{p.z, p.Q, 0, 0};
@@ -527,7 +530,7 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                     int rs;
                     const int s =
                         dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
-                              S.codes_h[b], rs);
+                             S.codes_h[b], rs);
                     if (row_writer) S.acc_h[par][b][my_row] = s;
                     if (tid == 0) S.meta_h[par][b].rs = rs;
                 }
@@ -585,7 +588,6 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 lstm_cell(pi, pf, pg, po, c[b], m);
                 const float h = jv ? m : 0.0f;
                 hl[b] = h;
-                if (g == 0) S.hloc[par][b][cl] = h;
                 // range of the warp's 8 cells (the four lanes of a quad hold the same value)
                 float mn = jv ? h : FLT_MAX, mx = jv ? h : -FLT_MAX;
 #pragma unroll
@@ -593,7 +595,21 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                     mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
                     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
                 }
-                if (lane == 0) S.emm[par][b][ew] = make_float2(mn, mx);
+                // the warp's 8 values to every block of the cluster (lane d -> block d) with their
+                // range; the stores complete on the peer's barrier. The last frame's values are not
+                // sent: no block waits for them (nothing is in flight at exit).
+                float v8[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) v8[q] = __shfl_sync(0xffffffffu, h, 4 * q);
+                if (lane < CS && t + 1 < T) {
+                    const uint32_t rbar = map_rank(hbar0 + 8 * par, lane);
+                    const uint32_t dst =
+                        map_rank(hbuf_l + 4u * (uint32_t)((par * kMaxB + b) * kMaxK + j0 + 8 * ew), lane);
+                    st_async_v4(dst, make_float4(v8[0], v8[1], v8[2], v8[3]), rbar);
+                    st_async_v4(dst + 16u, make_float4(v8[4], v8[5], v8[6], v8[7]), rbar);
+                    st_async_v2(map_rank(hmm_l + 8u * (uint32_t)((par * kMaxB + b) * kHParts + rank * kEW + ew), lane),
+                                mn, mx, rbar);
+                }
                 if (g == 0 && jv) {
                     const int64_t o = (((int64_t)l * B + b) * T + t) * R + j;
                     if (tag_out) st_tag(a.hx + o, ((unsigned long long)a.epoch << 32) | __float_as_uint(h));
@@ -603,28 +619,6 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(saddr(&S.bar_ep[par]));  // gate arithmetic of frame t done
-            named_bar(2, kET);
-            // the first epilogue warp sends this block's 32 values and their range to every block
-            // of the cluster (lane d -> block d); the stores complete on the peer's barrier. The
-            // last frame's values are not sent: no block waits for them (nothing is in flight at exit).
-            if (ew == 0 && lane < CS && t + 1 < T) {
-                const uint32_t rbar = map_rank(hbar0 + 8 * par, lane);
-                for (int b = 0; b < B; ++b) {
-                    float mn = FLT_MAX, mx = -FLT_MAX;
-#pragma unroll
-                    for (int w = 0; w < kEW; ++w) {
-                        const float2 mm = S.emm[par][b][w];
-                        mn = fminf(mn, mm.x);
-                        mx = fmaxf(mx, mm.y);
-                    }
-                    const uint32_t dst = map_rank(hbuf_l + 4u * (uint32_t)((par * kMaxB + b) * kMaxK + j0), lane);
-#pragma unroll
-                    for (int q = 0; q < kCellsPerBlock / 4; ++q)
-                        st_async_v4(dst + 16u * q, *reinterpret_cast<const float4 *>(&S.hloc[par][b][4 * q]), rbar);
-                    st_async_v2(map_rank(hmm_l + 8u * (uint32_t)((par * kMaxB + b) * kMaxCS + rank), lane), mn, mx,
-                                rbar);
-                }
-            }
         }
         if (g == 0 && jv) {
 #pragma unroll
