@@ -242,20 +242,23 @@ __device__ __forceinline__ void code_row(const float *row, int len, const qnn_qp
 }
 
 // Eight row partial dot products of this lane (8 rows x 16 bytes), summed across the warp so that
-// lane l ends with the full sum of local row ((l >> 2) & 7). Also returns the row code sum.
+// lane l ends with the full sum of local row ((l >> 2) & 7). With want_rs it also returns the
+// row code sum in rs.
 // `row(r)` yields this lane's 16 bytes of local row r (from registers or shared memory; a row is
 // fetched only when it is multiplied, so shared-memory rows never occupy registers all at once).
 // (dp4a rather than the warp-level integer MMA: on this GPU the two have the same peak rate, and
 // with one to four activation rows the MMA's eight columns would be mostly wasted.)
 template <typename RowBytes>
-__device__ __forceinline__ int dot8(RowBytes row, const uint8_t *codes, int &rs) {
+__device__ __forceinline__ int dot8(RowBytes row, const uint8_t *codes, bool want_rs, int &rs) {
     const int lane = threadIdx.x & 31;
     const uint4 cv = *reinterpret_cast<const uint4 *>(codes + lane * 16);
     const uint32_t c[4] = {cv.x, cv.y, cv.z, cv.w};
-    unsigned bs = 0;
+    if (want_rs) {  // warp-uniform
+        unsigned bs = 0;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) bs = __dp4a(c[i], 0x01010101u, bs);
-    rs = warp_sum((int)bs);
+        for (int i = 0; i < 4; ++i) bs = __dp4a(c[i], 0x01010101u, bs);
+        rs = warp_sum((int)bs);
+    }
     int v[kRowsPW];
 #pragma unroll
     for (int r = 0; r < kRowsPW; ++r) {
@@ -468,16 +471,16 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
             named_bar(1, kPT);
             if (tid == 0) mbar_arrive(empty0 + 8 * slot);
             for (int b = 0; b < B; ++b) {
-                int rs;
+                int rs = 0;
                 int s;
                 if (is_layer) {
                     s = dot8([&](int r) { return *reinterpret_cast<const uint4 *>(&S.wx[lr0 + r][lane * 16]); },
-                             S.codes_x[b], rs);
+                             S.codes_x[b], warp == 0, rs);
                     if (row_writer) S.acc_x[par][b][my_row] = s;
                     if (tid == 0) S.meta_x[par][b].rs = rs;
                 } else {
                     s = dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
-                             S.codes_x[b], rs);
+                             S.codes_x[b], true, rs);
                     if (row_writer && o_n >= 0) {
                         const RowMeta mt = S.meta_x[par][b];
                         const qnn_qparams po = a.wo_p[0];
@@ -527,10 +530,10 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 }
                 named_bar(1, kPT);
                 for (int b = 0; b < B; ++b) {
-                    int rs;
+                    int rs = 0;
                     const int s =
                         dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
-                             S.codes_h[b], rs);
+                             S.codes_h[b], warp == 0, rs);
                     if (row_writer) S.acc_h[par][b][my_row] = s;
                     if (tid == 0) S.meta_h[par][b].rs = rs;
                 }
@@ -579,28 +582,30 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 const RowMeta mt = S.meta_h[par][b];
                 const long long Sv = offset_product(S.acc_h[par][b][et], mt.za, ph.z, mt.rs, csh, R);
                 const float pre = __fadd_rn(yx[b], recover_product(Sv, mt.Qa, ph.Q));
+                // each lane applies its own gate's nonlinearity, then the quad gathers the four
+                const float act = gate_activation(pre, g == 2);
                 const int q0 = lane & ~3;
-                const float pi = __shfl_sync(0xffffffffu, pre, q0 + 0);
-                const float pf = __shfl_sync(0xffffffffu, pre, q0 + 1);
-                const float pg = __shfl_sync(0xffffffffu, pre, q0 + 2);
-                const float po = __shfl_sync(0xffffffffu, pre, q0 + 3);
-                float m;
-                lstm_cell(pi, pf, pg, po, c[b], m);
+                const float ig = __shfl_sync(0xffffffffu, act, q0 + 0);
+                const float fg = __shfl_sync(0xffffffffu, act, q0 + 1);
+                const float gg = __shfl_sync(0xffffffffu, act, q0 + 2);
+                const float og = __shfl_sync(0xffffffffu, act, q0 + 3);
+                const float m = lstm_cell_update(ig, fg, gg, og, c[b]);
                 const float h = jv ? m : 0.0f;
                 hl[b] = h;
-                // range of the warp's 8 cells (the four lanes of a quad hold the same value)
-                float mn = jv ? h : FLT_MAX, mx = jv ? h : -FLT_MAX;
-#pragma unroll
-                for (int o = 4; o < 32; o <<= 1) {
-                    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-                    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-                }
-                // the warp's 8 values to every block of the cluster (lane d -> block d) with their
-                // range; the stores complete on the peer's barrier. The last frame's values are not
-                // sent: no block waits for them (nothing is in flight at exit).
+                // the warp's 8 values (quad q holds cell 8 ew + q) in every lane, and their range
                 float v8[8];
 #pragma unroll
                 for (int q = 0; q < 8; ++q) v8[q] = __shfl_sync(0xffffffffu, h, 4 * q);
+                float mn = FLT_MAX, mx = -FLT_MAX;
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    if (j0 + 8 * ew + q < H) {
+                        mn = fminf(mn, v8[q]);
+                        mx = fmaxf(mx, v8[q]);
+                    }
+                // ... sent to every block of the cluster (lane d -> block d); the stores complete on
+                // the peer's barrier. The last frame's values are not sent: no block waits for them
+                // (nothing is in flight at exit).
                 if (lane < CS && t + 1 < T) {
                     const uint32_t rbar = map_rank(hbar0 + 8 * par, lane);
                     const uint32_t dst =

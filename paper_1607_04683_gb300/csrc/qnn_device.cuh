@@ -98,11 +98,24 @@ __device__ __forceinline__ float ptanh(float x) {
     return __fsub_rn(1.0f, __fdiv_rn(2.0f, __fadd_rn(pexp(__fmul_rn(2.0f, x)), 1.0f)));
 }
 
-// LSTM cell (no peepholes, gates [i, f, g, o]): c' = f c + i g; m = o tanh(c').
+// psigmoid(x) or ptanh(x) without a branch (lanes of one warp may need different ones): the same
+// operations in the same order, 1/(E(-x) + 1) or 1 - 2/(E(2x) + 1).
+__device__ __forceinline__ float gate_activation(float x, bool is_tanh) {
+    const float e = pexp(is_tanh ? __fmul_rn(2.0f, x) : -x);
+    const float q = __fdiv_rn(is_tanh ? 2.0f : 1.0f, __fadd_rn(e, 1.0f));
+    return is_tanh ? __fsub_rn(1.0f, q) : q;
+}
+
+// LSTM cell update from the gate activations (no peepholes): c' = f c + i g; returns m = o tanh(c').
+__device__ __forceinline__ float lstm_cell_update(float ig, float fg, float gg, float og, float &c) {
+    c = __fadd_rn(__fmul_rn(fg, c), __fmul_rn(ig, gg));
+    return __fmul_rn(og, ptanh(c));
+}
+
+// LSTM cell from the gate pre-activations [i, f, g, o]: sigmoid, sigmoid, tanh, sigmoid, then the update.
 __device__ __forceinline__ void lstm_cell(float pi, float pf, float pg, float po, float &c, float &m) {
     float ig = psigmoid(pi), fg = psigmoid(pf), gg = ptanh(pg), og = psigmoid(po);
-    c = __fadd_rn(__fmul_rn(fg, c), __fmul_rn(ig, gg));
-    m = __fmul_rn(og, ptanh(c));
+    m = lstm_cell_update(ig, fg, gg, og, c);
 }
 
 // Warp-wide reductions.
