@@ -394,7 +394,10 @@ def run_sweep(args):
         print(json.dumps({
             "sweep": "qmatmul", "M": shape.M, "N": shape.N, "K": shape.K,
             "qmatmul_tops": ops / t_mm / 1e12, "qmatmul_ms": t_mm * 1e3,
+            "datapath": "tcgen05 fp16 (exact centered codes)" if shape.M >= 128 else "mma.sync u8",
+            "frac_of_datapath_peak": ops / t_mm / 1e12 / (peaks["bf16_tflops"] if shape.M >= 128 else imma),
             "frac_of_measured_mma_u8_peak": ops / t_mm / 1e12 / imma, "mma_u8_peak_tops": imma,
+            "f16_tensor_peak_tflops": peaks["bf16_tflops"],
             "qmatmul_gbs": mm_bytes / t_mm / 1e9,
             "fp32_in_tops": ops / t_all / 1e12, "quantize_ms": t_q * 1e3,
             "quantize_gbs_alg": 5.0 * shape.M * shape.K / t_q / 1e9, "hbm_peak_gbs": peaks["hbm_gbs"],

@@ -10,6 +10,7 @@
 // V'' = V' + round(Q Vmin)), then y = S / (Qa Qw) + bias (eq. 3 recovery and Fig. 1's bias), and
 // optionally the raw accumulator.
 #include <cstdlib>
+#include <cstring>
 
 #include "qnn_device.cuh"
 #include "qnn_host.h"
@@ -173,10 +174,10 @@ __global__ void __launch_bounds__(THREADS) qgemm_imma_kernel(
 
 }  // namespace
 
-qnn_status launch_qgemm(const uint8_t *A, int64_t lda, const qnn_qparams *pa, int ga, const int32_t *rsA, int64_t M,
-                        int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw, int64_t rows_per_block,
-                        const int32_t *csW, int64_t N, const float *bias, float *Y, int64_t ldy, int32_t *acc_out,
-                        cudaStream_t st) {
+qnn_status launch_qgemm_imma(const uint8_t *A, int64_t lda, const qnn_qparams *pa, int ga, const int32_t *rsA,
+                             int64_t M, int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw,
+                             int64_t rows_per_block, const int32_t *csW, int64_t N, const float *bias, float *Y,
+                             int64_t ldy, int32_t *acc_out, cudaStream_t st) {
     if (M == 0 || N == 0) return QNN_OK;
     static bool configured[2] = {false, false};
     const bool aligned = ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15) == 0 &&
@@ -192,6 +193,27 @@ qnn_status launch_qgemm(const uint8_t *A, int64_t lda, const qnn_qparams *pa, in
                                             N, bias, Y, ldy, acc_out);
     QNN_CUDA_TRY(cudaGetLastError());
     return QNN_OK;
+}
+
+// Datapath choice: the tcgen05 path runs whole 128 x 256 tiles at the fp16 tensor rate (after
+// centering both operands into fp16 scratch); below one tile of rows the integer MMA path, which
+// needs no conversion, is used. QNN_QGEMM=imma or =tc forces one (tests compare the two).
+qnn_status launch_qgemm(const uint8_t *A, int64_t lda, const qnn_qparams *pa, int ga, const int32_t *rsA, int64_t M,
+                        int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw, int64_t rows_per_block,
+                        const int32_t *csW, int64_t N, const float *bias, float *Y, int64_t ldy, int32_t *acc_out,
+                        cudaStream_t st) {
+    if (M == 0 || N == 0) return QNN_OK;
+    const char *force = std::getenv("QNN_QGEMM");
+    bool tc = M >= 128;
+    if (force && std::strcmp(force, "imma") == 0) tc = false;
+    if (force && std::strcmp(force, "tc") == 0) tc = true;
+    if (tc) {
+        void *ws = nullptr;
+        QNN_TRY(scratch(kScratchTc, tc_scratch_bytes(M, N, K), &ws));
+        return launch_qgemm_tc(A, lda, pa, ga, rsA, M, K, W, ldw, pw, rows_per_block, csW, N, bias, Y, ldy, acc_out, ws,
+                               st);
+    }
+    return launch_qgemm_imma(A, lda, pa, ga, rsA, M, K, W, ldw, pw, rows_per_block, csW, N, bias, Y, ldy, acc_out, st);
 }
 
 }  // namespace qnn

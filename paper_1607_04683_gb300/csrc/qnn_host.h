@@ -33,7 +33,7 @@ inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s
 bool is_device_ptr(const void *p);
 
 // Library-owned, grow-only device scratch of the current device (one slot per purpose).
-enum ScratchSlot { kScratchReduce = 0, kScratchCount = 1 };
+enum ScratchSlot { kScratchReduce = 0, kScratchTc = 1, kScratchCount = 2 };
 qnn_status scratch(ScratchSlot slot, size_t bytes, void **out);
 
 // The device status word of the current device (allocated and zeroed on first use).
@@ -66,6 +66,17 @@ qnn_status launch_qgemm(const uint8_t *A, int64_t lda, const qnn_qparams *pa, in
                         int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw, int64_t rows_per_block,
                         const int32_t *csW, int64_t N, const float *bias, float *Y, int64_t ldy, int32_t *acc_out,
                         cudaStream_t st);
+// The two product datapaths behind launch_qgemm: the warp-level integer MMA (any shape) and the
+// exact fp16 tcgen05 path (needs fp16 copies of both operands in `scratch`, tc_scratch_bytes).
+qnn_status launch_qgemm_imma(const uint8_t *A, int64_t lda, const qnn_qparams *pa, int ga, const int32_t *rsA,
+                             int64_t M, int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw,
+                             int64_t rows_per_block, const int32_t *csW, int64_t N, const float *bias, float *Y,
+                             int64_t ldy, int32_t *acc_out, cudaStream_t st);
+qnn_status launch_qgemm_tc(const uint8_t *A, int64_t lda, const qnn_qparams *pa, int ga, const int32_t *rsA, int64_t M,
+                           int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw, int64_t rows_per_block,
+                           const int32_t *csW, int64_t N, const float *bias, float *Y, int64_t ldy, int32_t *acc_out,
+                           void *scratch, cudaStream_t st);
+size_t tc_scratch_bytes(int64_t M, int64_t N, int64_t K);
 qnn_status launch_softmax_rows(const float *logits, int64_t rows, int64_t C, float *y, cudaStream_t st);
 
 }  // namespace qnn

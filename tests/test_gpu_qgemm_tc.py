@@ -1,0 +1,73 @@
+"""The exact fp16 tcgen05 product path against the oracle and against the integer-MMA path.
+
+Codes are centered (c - 128) into fp16, exact; products and sums of up to 1024 of them are exact in
+the fp32 tensor-memory accumulator; longer K is accumulated in chunks drained into int32. Every
+result must equal the oracle's bit for bit (int32 accumulator and recovered fp32)."""
+import numpy as np
+import pytest
+
+import oracle
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def qnn():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_1607_04683_gb300 import build, qnn as q
+    build.build()
+    q.lib()
+    torch.cuda.set_device(0)
+    return q
+
+
+def gpu(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _run(qnn, ca, pa, ga, ra, cw, pw, cs, nb=1, bias=None):
+    return qnn.qnn_qmatmul(gpu(ca), qnn.params_tensor(pa), ga, gpu(ra), gpu(cw), qnn.params_tensor(pw), gpu(cs),
+                           n_blocks=nb, bias=None if bias is None else gpu(bias), want_acc=True)
+
+
+TC_SHAPES = [(1, 8, 1), (3, 300, 40), (128, 256, 64), (130, 260, 100), (257, 2000, 500), (384, 512, 1024),
+             (200, 136, 1025), (129, 257, 2048), (256, 256, 8192)]
+
+
+@pytest.mark.parametrize("M,N,K", TC_SHAPES)
+def test_tc_path_bit_exact(qnn, M, N, K, monkeypatch):
+    g = np.random.Generator(np.random.PCG64(M * 31 + N * 7 + K))
+    A = g.normal(0.1, 1.0, (M, K)).astype(np.float32)
+    nb = 4 if N % 4 == 0 else 1
+    Ws = [g.uniform(-s, s, (N // nb, K)).astype(np.float32) for s in np.linspace(0.05, 0.4, nb)]
+    ca, pa, ra = oracle.quantize(A, oracle.PER_ROW)
+    parts = [oracle.quantize(w, oracle.PER_MATRIX) for w in Ws]
+    cw = np.concatenate([p[0] for p in parts])
+    pw = np.concatenate([p[1] for p in parts])
+    cs = np.concatenate([p[2] for p in parts])
+    bias = g.normal(0, 1, N).astype(np.float32)
+    ref = oracle.qmatmul(ca, pa, 1, cw, pw, n_blocks=nb, bias=bias)
+    for path in ("tc", "imma"):
+        monkeypatch.setenv("QNN_QGEMM", path)
+        Y, acc = _run(qnn, ca, pa, 1, ra, cw, pw, cs, nb, bias)
+        assert qnn.device_status() == qnn.QNN_OK
+        assert np.array_equal(acc.cpu().numpy(), ref["acc"]), path
+        assert np.array_equal(Y.cpu().numpy(), ref["y"]), path
+
+
+@pytest.mark.parametrize("K", [1024, 1025, 2048])
+@pytest.mark.parametrize("a_code,w_code", [(0, 0), (255, 255), (0, 255)])
+def test_tc_extreme_codes_at_the_exactness_limit(qnn, K, a_code, w_code, monkeypatch):
+    # centered values +-128 / 127 everywhere: |sum| reaches 2^24 at K = 1024, the fp32 limit
+    monkeypatch.setenv("QNN_QGEMM", "tc")
+    M, N = 128, 256
+    ca = np.full((M, K), a_code, np.uint8)
+    cw = np.full((N, K), w_code, np.uint8)
+    p = np.zeros(1, qnn.QPARAMS_DTYPE)
+    p[0] = (0.0, 1.0, 255.0, 0)
+    ra = ca.astype(np.int64).sum(1).astype(np.int32)
+    cs = cw.astype(np.int64).sum(1).astype(np.int32)
+    Y, acc = _run(qnn, ca, p, 0, ra, cw, p, cs)
+    assert np.all(acc.cpu().numpy() == a_code * w_code * K)
