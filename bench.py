@@ -77,10 +77,25 @@ def recurrent_bytes_per_launch(wl: inputs.LstmWorkload) -> int:
     return weights + wl.batch * wl.frames * per_frame
 
 
-def traffic_record(kernel: str, workload: str):
+def small_ops_per_launch(wl: inputs.LstmWorkload) -> int:
+    """Integer multiply-adds x 2 of one batch-of-few launch: every layer's input and recurrent
+    products and the output layer's, for B T frames."""
+    return ops_per_frame(wl) * wl.batch * wl.frames
+
+
+def small_bytes_per_launch(wl: inputs.LstmWorkload) -> int:
+    """Unique HBM bytes of one batch-of-few launch: every weight code once, the input frames,
+    and the logits (or top-layer outputs) written."""
+    H, R = wl.hidden, wl.R
+    w = sum(4 * H * (wl.layer_in(l) + R) for l in range(wl.num_layers)) + wl.num_classes * R
+    out = wl.num_classes if wl.num_classes > 0 else R
+    return w + wl.batch * wl.frames * (wl.input_dim + out) * 4
+
+
+def traffic_record(kernel: str, workload: str, source: str):
     """Per-launch DRAM bytes from the committed ncu summary, if taken on the current source."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
-    src = os.path.join(ROOT, "paper_1607_04683_gb300", "csrc", "lstm.cu")
+    src = os.path.join(ROOT, "paper_1607_04683_gb300", "csrc", source)
     try:
         sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
         for line in open(path):
@@ -312,17 +327,27 @@ def run_ours(args, wl, rank, world, local):
     kname = max(prof, key=lambda k: prof[k][1])
     launches, kms = prof[kname]
     avg_s = kms / launches / 1e3
+    roofline = None
+    share = kms / total_ms if world == 1 else None
     if kname == "lstm_recurrent":
         alg = recurrent_bytes_per_launch(wl)
-    else:
-        alg = None
-    roofline = None
-    if alg is not None:
         ach = alg / avg_s / 1e9
         roofline = {"bound": "hbm", "kernel": kname, "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                     "frac": ach / peaks["hbm_gbs"], "peak_kind": peak_kind,
-                    "traffic": traffic_record(kname, wl.name), "alg_bytes_per_launch": alg,
-                    "avg_launch_ms": avg_s * 1e3, "share_of_step": kms / total_ms if world == 1 else None}
+                    "traffic": traffic_record(kname, wl.name, "lstm.cu"), "alg_bytes_per_launch": alg,
+                    "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
+    elif kname == "lstm_small":
+        # the whole stack in one launch; its arithmetic is the integer products of every layer and
+        # of the output layer, which run as dp4a (u8 x u8 -> s32): roofline = the measured dp4a rate
+        ops = small_ops_per_launch(wl)
+        ach = ops / avg_s / 1e12
+        dp4a_peak = qnn.measure_peak(1)
+        roofline = {"bound": "alu", "kernel": kname, "achieved": ach, "peak": dp4a_peak, "unit": "TOP/s",
+                    "frac": ach / dp4a_peak, "peak_kind": "measured (qnn_measure_peak dp4a)",
+                    "traffic": traffic_record(kname, wl.name, "lstm_small.cu"), "alg_ops_per_launch": ops,
+                    "alg_bytes_per_launch": small_bytes_per_launch(wl), "hbm_frac":
+                        small_bytes_per_launch(wl) / avg_s / 1e9 / peaks["hbm_gbs"],
+                    "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
     line = {
         "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",

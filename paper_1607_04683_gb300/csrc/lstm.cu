@@ -28,6 +28,7 @@ constexpr int kRecThreads = 256;
 constexpr int kRecWarps = kRecThreads / 32;
 constexpr int kPad = 16;  // extra bytes per shared-memory code row (bank spread for ldmatrix)
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s per grid-wide wait
+constexpr int kDistQuantMinBatch = 8;  // batch from which rows are quantized once per step, grid-wide
 
 inline int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
@@ -72,6 +73,12 @@ struct RecArgs {
     unsigned *bar;            // grid barrier counter, zero at launch
     int *abort_flag;          // set when any wait gave up, zero at launch
     int *status;
+    // shared quantization (large batches): each row is quantized once per step by one warp of
+    // the grid into these buffers, then every block copies the rows it needs
+    uint8_t *qcodes;          // [B][ldq]
+    qnn_qparams *qprm;        // [B]
+    int *qsum;                // [B]
+    int ldq, distq;
     int B, T, H, R, P, ldh, ldp, nc, np, bc;
 };
 
@@ -159,6 +166,77 @@ __device__ __forceinline__ void quantize_rows_smem(const float *src, int64_t ld,
             sza[r] = p.z;
             sQa[r] = p.Q;
             srs[r] = s;
+        }
+    }
+}
+
+// Quantizes `rows` rows of `len` fp32 values (row r at src + r*ld) into the shared global buffers,
+// one warp per row, the rows spread over every warp of the grid.
+__device__ __forceinline__ void quantize_rows_global(const float *src, int64_t ld, int rows, int len, int kdim,
+                                                     const RecArgs &a) {
+    const int lane = threadIdx.x & 31;
+    const int gw = blockIdx.x * kRecWarps + (threadIdx.x >> 5), nw = gridDim.x * kRecWarps;
+    for (int r = gw; r < rows; r += nw) {
+        const float *xr = src + r * ld;
+        float mn = FLT_MAX, mx = -FLT_MAX;
+        bool bad = false;
+        for (int k = lane; k < len; k += 32) {
+            float v = __ldcg(xr + k);
+            bad |= !isfinite(v);
+            mn = fminf(mn, v);
+            mx = fmaxf(mx, v);
+        }
+        mn = warp_min(mn);
+        mx = warp_max(mx);
+        if (__any_sync(0xffffffffu, bad)) {
+            if (lane == 0) record_status(a.status, QNN_ERR_NONFINITE);
+            mn = 0.0f;
+            mx = 0.0f;
+        }
+        const qnn_qparams p = params_from_range(mn, mx);
+        uint8_t *dst = a.qcodes + (int64_t)r * a.ldq;
+        int s = 0;
+        for (int k4 = lane * 4; k4 < kdim; k4 += 128) {
+            uint32_t w = 0;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int k = k4 + e;
+                if (k < len) {
+                    uint32_t c = quant_code(__ldcg(xr + k), p.Q, p.z);
+                    s += (int)c;
+                    w |= c << (8 * e);
+                }
+            }
+            *reinterpret_cast<uint32_t *>(dst + k4) = w;
+        }
+        s = warp_sum(s);
+        if (lane == 0) {
+            a.qprm[r] = p;
+            a.qsum[r] = s;
+        }
+    }
+}
+
+// Copies rows b0 .. b0 + nb - 1 of the shared quantized rows (kdim bytes each) into shared memory
+// as quantize_rows_smem would have produced them; rows nb .. rows_total - 1 become zero rows.
+__device__ __forceinline__ void load_rows_smem(const RecArgs &a, int b0, int nb, int rows_total, int kdim,
+                                               uint8_t *sact, int srow, int *sza, float *sQa, int *srs) {
+    const int chunks = kdim / 16;
+    for (int i = threadIdx.x; i < rows_total * chunks; i += kRecThreads) {
+        const int r = i / chunks, ch = i % chunks;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (r < nb) v = __ldcg(reinterpret_cast<const uint4 *>(a.qcodes + (int64_t)(b0 + r) * a.ldq + ch * 16));
+        *reinterpret_cast<uint4 *>(sact + r * srow + ch * 16) = v;
+    }
+    for (int r = threadIdx.x; r < rows_total; r += kRecThreads) {
+        if (r < nb) {
+            sza[r] = __ldcg(&a.qprm[b0 + r].z);
+            sQa[r] = __ldcg(&a.qprm[b0 + r].Q);
+            srs[r] = __ldcg(a.qsum + b0 + r);
+        } else {
+            sza[r] = 0;
+            sQa[r] = 1.0f;
+            srs[r] = 0;
         }
     }
 }
@@ -267,11 +345,20 @@ __global__ void __launch_bounds__(kRecThreads, 1) lstm_recurrent_kernel(RecArgs 
 
     unsigned epoch = 0;
     for (int t = 0; t < T; ++t) {
+        if (a.distq) {  // every row of h_{t-1} quantized once, by one warp of the grid
+            const float *hsrc = (t == 0) ? a.h0 : a.out + (t - 1) * (int64_t)R;
+            quantize_rows_global(hsrc, (t == 0) ? R : (int64_t)T * R, a.B, R, a.ldh, a);
+            if (!grid_sync(a, epoch, &s_flag)) return;
+        }
         for (int b0 = 0; b0 < a.B; b0 += bc) {
             const int nb = min(bc, a.B - b0);
-            const float *hsrc = (t == 0) ? a.h0 + (int64_t)b0 * R : a.out + ((int64_t)b0 * T + (t - 1)) * R;
-            const int64_t hld = (t == 0) ? R : (int64_t)T * R;
-            quantize_rows_smem(hsrc, hld, nb, bc, R, a.ldh, sact, arow, sza, sQa, srs, a.status);
+            if (a.distq) {
+                load_rows_smem(a, b0, nb, bc, a.ldh, sact, arow, sza, sQa, srs);
+            } else {
+                const float *hsrc = (t == 0) ? a.h0 + (int64_t)b0 * R : a.out + ((int64_t)b0 * T + (t - 1)) * R;
+                const int64_t hld = (t == 0) ? R : (int64_t)T * R;
+                quantize_rows_smem(hsrc, hld, nb, bc, R, a.ldh, sact, arow, sza, sQa, srs, a.status);
+            }
             __syncthreads();
             product_block(sw_h, wrow_h, sact, arow, 4 * nc, bc, a.ldh, R, sza, sQa, srs, sy, h_row_info);
             __syncthreads();
@@ -296,11 +383,18 @@ __global__ void __launch_bounds__(kRecThreads, 1) lstm_recurrent_kernel(RecArgs 
         }
         if (a.P > 0) {
             if (!grid_sync(a, epoch, &s_flag)) return;
+            if (a.distq) {  // every row of m_t quantized once
+                quantize_rows_global(a.mbuf, H, a.B, H, a.ldp, a);
+                if (!grid_sync(a, epoch, &s_flag)) return;
+            }
             if (p0 < a.P) {
                 for (int b0 = 0; b0 < a.B; b0 += bc) {
                     const int nb = min(bc, a.B - b0);
-                    quantize_rows_smem(a.mbuf + (int64_t)b0 * H, H, nb, bc, H, a.ldp, sact, arow, sza, sQa, srs,
-                                       a.status);
+                    if (a.distq)
+                        load_rows_smem(a, b0, nb, bc, a.ldp, sact, arow, sza, sQa, srs);
+                    else
+                        quantize_rows_smem(a.mbuf + (int64_t)b0 * H, H, nb, bc, H, a.ldp, sact, arow, sza, sQa, srs,
+                                           a.status);
                     __syncthreads();
                     product_block(sw_p, wrow_p, sact, arow, np, bc, a.ldp, H, sza, sQa, srs, sy, p_row_info);
                     __syncthreads();
@@ -694,6 +788,10 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const size_t o_h0 = acct(B * R * 4 * L);
     const size_t o_c = acct(B * H * 4);
     const size_t o_m = acct(P > 0 ? B * H * 4 : 0);
+    const int64_t ldq = round_up(R > H ? R : H, 64);
+    const size_t o_qc = acct(B * ldq);
+    const size_t o_qp = acct(B * sizeof(qnn_qparams));
+    const size_t o_qs = acct(B * 4);
     const size_t o_lg = acct(C > 0 ? rows * C * 4 : 0);
     const size_t o_y = y_dev ? 0 : acct(rows * ycols * 4);
     if (need > m->ws_bytes) {
@@ -764,6 +862,11 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
         a.B = (int)B, a.T = (int)T, a.H = (int)H, a.R = (int)R, a.P = (int)P;
         a.ldh = (int)ly.wh.ld, a.ldp = P > 0 ? (int)ly.wp.ld : 0;
         a.nc = plan.nc, a.np = plan.np, a.bc = plan.bc;
+        a.qcodes = reinterpret_cast<uint8_t *>(ws + o_qc);
+        a.qprm = reinterpret_cast<qnn_qparams *>(ws + o_qp);
+        a.qsum = reinterpret_cast<int *>(ws + o_qs);
+        a.ldq = (int)ldq;
+        a.distq = B >= kDistQuantMinBatch;  // below this, each block quantizing its rows is cheaper
         void *args[] = {&a};
         ProfScope prof("lstm_recurrent", st);
         cudaError_t e = cudaLaunchCooperativeKernel((const void *)lstm_recurrent_kernel, dim3(plan.grid),

@@ -240,6 +240,7 @@ def _oracle(wl, params, x, **kw):
 SMALL_CASES = [dict(), dict(L=1, I=3, H=4, B=1, T=9), dict(L=3, H=16, C=11, B=3), dict(L=2, H=33, I=40, C=5, B=17, T=4),
                dict(L=2, I=6, H=10, P=4, C=7, B=2, T=5), dict(L=2, I=80, H=130, P=48, C=70, B=20, T=6),
                dict(L=2, H=12, C=5, mode=2), dict(L=1, I=40, H=500, B=70, T=3, C=2000, w=0.08),
+               dict(L=2, I=40, H=64, C=9, B=6, T=5), dict(L=2, I=40, H=50, P=16, C=9, B=6, T=4),
                dict(L=3, I=5, H=8, B=65, T=3, mu=0.5)]
 
 
