@@ -31,7 +31,7 @@ namespace qnn {
 namespace {
 
 constexpr int TBM = 128, TBN = 256, TBK = 64;     // fp16 elements per k-block (128 bytes)
-constexpr int TSTAGES = 4;
+constexpr int TSTAGES = 3;
 constexpr int A_BYTES = TBM * TBK * 2;            // 16 KB
 constexpr int B_BYTES = TBN * TBK * 2;            // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -150,15 +150,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // 1024-byte alignment for the swizzled tiles
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + TSTAGES * STAGE_BYTES);
+    int *stage_out = reinterpret_cast<int *>(smem + TSTAGES * STAGE_BYTES);        // [8 warps][32][33]
+    int *row_c = stage_out + 8 * 32 * 33;                                          // [8 warps][3][32]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(row_c + 8 * 3 * 32);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * TSTAGES + 4);
     const uint32_t full0 = su32(bars), empty0 = su32(bars + TSTAGES), chunk0 = su32(bars + 2 * TSTAGES),
                    drained0 = su32(bars + 2 * TSTAGES + 2);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t m0 = (int64_t)blockIdx.y * TBM, n0 = (int64_t)blockIdx.x * TBN;
     const int KB = args.KB;
-    const int kb_per_chunk = KCHUNK / TBK;  // 16
-    const int nchunks = (KB + kb_per_chunk - 1) / kb_per_chunk;
+    const int kpc = KCHUNK / TBK;  // k-blocks per chunk (16)
+    const int nchunks = (KB + kpc - 1) / kpc;
+    const int tiles_n = (int)((args.N + TBN - 1) / TBN);
+    const int64_t tiles = (int64_t)((args.M + TBM - 1) / TBM) * tiles_n;
     __shared__ int s_abort;
 
     if (threadIdx.x == 0) {
@@ -185,112 +188,162 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem_base = *tmem_slot;
 
+    // Persistent: block b takes tiles b, b + grid, ... (row-tile major, so neighbouring blocks share
+    // the same rows of A through L2). The k-block and chunk counters run across tiles, so the two
+    // accumulator buffers alternate and one tile's epilogue overlaps the next tile's MMAs.
     if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (lane == 0) {
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % TSTAGES;
-                if (kb >= TSTAGES && !mb_wait(empty0 + 8 * s, ((kb / TSTAGES) - 1) & 1, args.status)) {
-                    s_abort = 1;
-                    break;
+            int64_t g = 0;  // k-blocks issued by this block
+            for (int64_t tile = blockIdx.x; tile < tiles && !s_abort; tile += gridDim.x) {
+                const int m0 = (int)(tile / tiles_n) * TBM, n0 = (int)(tile % tiles_n) * TBN;
+                for (int kb = 0; kb < KB; ++kb, ++g) {
+                    const int s = (int)(g % TSTAGES);
+                    if (g >= TSTAGES && !mb_wait(empty0 + 8 * s, (unsigned)((g / TSTAGES) - 1) & 1, args.status)) {
+                        s_abort = 1;
+                        break;
+                    }
+                    const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
+                    mb_expect(full0 + 8 * s, STAGE_BYTES);
+                    tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
+                    tma_load_2d(sb, &mapW, full0 + 8 * s, kb * TBK, n0);
                 }
-                const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
-                mb_expect(full0 + 8 * s, STAGE_BYTES);
-                tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, (int)m0);
-                tma_load_2d(sb, &mapW, full0 + 8 * s, kb * TBK, (int)n0);
             }
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
-            for (int kb = 0; kb < KB; ++kb) {
-                const int s = kb % TSTAGES;
-                const int chunk = kb / kb_per_chunk, buf = chunk & 1;
-                const bool first_of_chunk = (kb % kb_per_chunk) == 0;
-                if (first_of_chunk && chunk >= 2 &&
-                    !mb_wait(drained0 + 8 * buf, ((chunk / 2) - 1) & 1, args.status)) {  // buffer free again
-                    s_abort = 1;
-                    break;
-                }
-                if (!mb_wait(full0 + 8 * s, (kb / TSTAGES) & 1, args.status)) {
-                    s_abort = 1;
-                    break;
-                }
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
-                const uint32_t tmem_d = tmem_base + (uint32_t)(buf * TBN);
+            int64_t g = 0, gc = 0;  // k-blocks and chunks consumed by this block
+            for (int64_t tile = blockIdx.x; tile < tiles && !s_abort; tile += gridDim.x) {
+                for (int kb = 0; kb < KB; ++kb, ++g) {
+                    const int s = (int)(g % TSTAGES);
+                    const int kc = kb % kpc;
+                    const int buf = (int)(gc & 1);
+                    if (kc == 0 && gc >= 2 &&
+                        !mb_wait(drained0 + 8 * buf, (unsigned)((gc / 2) - 1) & 1, args.status)) {  // buffer free
+                        s_abort = 1;
+                        break;
+                    }
+                    if (!mb_wait(full0 + 8 * s, (unsigned)(g / TSTAGES) & 1, args.status)) {
+                        s_abort = 1;
+                        break;
+                    }
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
+                    const uint32_t tmem_d = tmem_base + (uint32_t)(buf * TBN);
 #pragma unroll
-                for (int k = 0; k < TBK / 16; ++k) {
-                    // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
-                    mma_f16(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k),
-                            (first_of_chunk && k == 0) ? 0u : 1u);
+                    for (int k = 0; k < TBK / 16; ++k) {
+                        // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
+                        mma_f16(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k), (kc == 0 && k == 0) ? 0u : 1u);
+                    }
+                    mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
+                    if (kc == kpc - 1 || kb == KB - 1) {
+                        mma_commit(chunk0 + 8 * buf);
+                        ++gc;
+                    }
                 }
-                mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
-                if ((kb % kb_per_chunk) == kb_per_chunk - 1 || kb == KB - 1) mma_commit(chunk0 + 8 * buf);
+                if (s_abort) break;
             }
         }
     } else {
         // ---------------- epilogue (warps 2..9) ----------------
         const int q = warp & 3;                 // tensor-memory lane quarter this warp may read
         const int half = (warp - 2) >> 2;       // column half: 0 -> [0, 128), 1 -> [128, 256)
-        const int row_local = 32 * q + lane;    // accumulator lane = tile row
-        const int64_t m = m0 + row_local;
-        const bool row_ok = m < args.M;
-        const qnn_qparams qa = args.pa[args.a_per_row ? (row_ok ? m : 0) : 0];
-        const int ra = row_ok ? args.rsA[m] : 0;
+        const int ew = warp - 2;
+        int *stg = stage_out + ew * 32 * 33;
+        int *rz = row_c + ew * 96, *rr = rz + 32;
+        float *rq = reinterpret_cast<float *>(rz + 64);
         const int K = args.K;
-        // one output: exact centered product P of column `col` of this row -> eq. (1) offsets,
-        // eq. (3) recovery, bias
-        auto finish = [&](int col, int P) {
-            const int64_t n = n0 + col;
-            if (!row_ok || n >= args.N) return;
-            const qnn_qparams qw = args.pw[n / args.rows_per_block];
-            const int cs = args.csW[n];
-            const int acc = P + 128 * (ra + cs) - 16384 * K;  // raw code product (fits int32)
-            const long long S = offset_product(acc, qa.z, qw.z, ra, cs, K);
-            float y = recover_product(S, qa.Q, qw.Q);
-            if (args.bias) y = __fadd_rn(y, args.bias[n]);
-            if (args.Y) args.Y[m * args.ldy + n] = y;
-            if (args.acc_out) args.acc_out[m * args.N + n] = acc;
-        };
-        auto taddr_of = [&](int buf, int j) {
-            return tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * TBN + half * 128 + 32 * j);
-        };
-        if (nchunks == 1) {  // K <= 1024: read the accumulator and finish directly
-            if (__all_sync(0xffffffffu, mb_wait(chunk0, 0, args.status))) {
+        int64_t gc = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * TBN;
+            {  // this lane's row constants, shared with the warp for the transposed stores
+                const int64_t m = m0 + 32 * q + lane;
+                const bool mv = m < args.M;
+                const qnn_qparams qa = args.pa[args.a_per_row ? (mv ? m : 0) : 0];
+                rz[lane] = qa.z;
+                rq[lane] = qa.Q;
+                rr[lane] = mv ? args.rsA[m] : 0;
+            }
+            // 32 x 32 block: P values of rows (this warp's 32 lanes) x columns c0 .. c0 + 31, written
+            // row-wise to shared memory and read back column-wise, so that each store instruction
+            // writes 32 consecutive outputs of one row.
+            auto emit = [&](int c0, const int (&P)[32]) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) stg[lane * 33 + i] = P[i];
+                __syncwarp();
+                const int64_t n = n0 + c0 + lane;
+                const bool nv = n < args.N;
+                const qnn_qparams qw = args.pw[nv ? n / args.rows_per_block : 0];
+                const int cs = nv ? args.csW[n] : 0;
+                const float bn = (nv && args.bias) ? args.bias[n] : 0.0f;
+                for (int r = 0; r < 32; ++r) {
+                    const int64_t m = m0 + 32 * q + r;
+                    if (m >= args.M) break;
+                    if (nv) {
+                        const int ra = rr[r];
+                        const int acc = stg[r * 33 + lane] + 128 * (ra + cs) - 16384 * K;  // raw code product
+                        const long long S = offset_product(acc, rz[r], qw.z, ra, cs, K);
+                        float y = recover_product(S, rq[r], qw.Q);
+                        if (args.bias) y = __fadd_rn(y, bn);
+                        if (args.Y) args.Y[m * args.ldy + n] = y;
+                        if (args.acc_out) args.acc_out[m * args.N + n] = acc;
+                    }
+                }
+                __syncwarp();
+            };
+            auto taddr_of = [&](int buf, int j) {
+                return tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * TBN + half * 128 + 32 * j);
+            };
+            __syncwarp();
+            if (nchunks == 1) {  // K <= 1024: read the accumulator and finish directly
+                const int buf = (int)(gc & 1);
+                ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
+                if (!ok) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll 1
                 for (int j = 0; j < 4; ++j) {
                     uint32_t r[32];
-                    tmem_ld32<32>(taddr_of(0, j), r);
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) finish(half * 128 + 32 * j + i, __float2int_rn(__uint_as_float(r[i])));
-                }
-            }
-        } else {  // drain every chunk into int32 running sums
-            int run[128];
-#pragma unroll
-            for (int i = 0; i < 128; ++i) run[i] = 0;
-            bool ok = true;
-            for (int c = 0; c < nchunks; ++c) {
-                const int buf = c & 1;
-                ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (c / 2) & 1, args.status));
-                if (!ok) break;
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    uint32_t r[32];
                     tmem_ld32<32>(taddr_of(buf, j), r);
+                    int P[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) run[32 * j + i] += __float2int_rn(__uint_as_float(r[i]));
+                    for (int i = 0; i < 32; ++i) P[i] = __float2int_rn(__uint_as_float(r[i]));
+                    emit(half * 128 + 32 * j, P);
                 }
+                // the accumulator is free again: the tile after next may use it
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
                 if (lane == 0)
                     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+                ++gc;
+            } else {  // drain every chunk into int32 running sums
+                int run[4][32];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) run[j][i] = 0;
+                for (int c = 0; c < nchunks; ++c, ++gc) {
+                    const int buf = (int)(gc & 1);
+                    ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
+                    if (!ok) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        uint32_t rr32[32];
+                        tmem_ld32<32>(taddr_of(buf, j), rr32);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) run[j][i] += __float2int_rn(__uint_as_float(rr32[i]));
+                    }
+                    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0)
+                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+                }
+                if (!ok) break;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) emit(half * 128 + 32 * j, run[j]);
             }
-            if (ok)
-                for (int i = 0; i < 128; ++i) finish(half * 128 + i, run[i]);
         }
     }
     __syncwarp();
@@ -298,11 +351,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
     __syncthreads();
     if (s_abort && warp == 0 && lane == 0) {
         // let copies still in flight land before the block leaves (bounded)
-        for (int i = 0; i < TSTAGES; ++i) {
-            const unsigned long long t0 = gtime();
-            while (gtime() - t0 < 2000000ull) __nanosleep(1000);
-            (void)i;
-        }
+        const unsigned long long t0 = gtime();
+        while (gtime() - t0 < 4000000ull) __nanosleep(1000);
     }
     __syncthreads();
     if (warp == 1) {
@@ -393,7 +443,7 @@ qnn_status launch_qgemm_tc(const uint8_t *A, int64_t lda, const qnn_qparams *pa,
     int *status = nullptr;
     QNN_TRY(status_word(&status));
     TcArgs a{pa, ga == QNN_PER_ROW, rsA, pw, rows_per_block, csW, bias, Y, ldy, acc_out, M, N, (int)K, kp / TBK, status};
-    const size_t smem = (size_t)TSTAGES * STAGE_BYTES + 1024 + 256;
+    const size_t smem = (size_t)TSTAGES * STAGE_BYTES + 1024 + (8 * 32 * 33 + 8 * 96) * 4 + 256;
     static int configured = -1;
     int dev = 0;
     QNN_CUDA_TRY(cudaGetDevice(&dev));
@@ -401,7 +451,8 @@ qnn_status launch_qgemm_tc(const uint8_t *A, int64_t lda, const qnn_qparams *pa,
         QNN_CUDA_TRY(cudaFuncSetAttribute(qgemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
         configured = dev;
     }
-    dim3 grid((unsigned)((N + TBN - 1) / TBN), (unsigned)((M + TBM - 1) / TBM));
+    const int64_t tiles = ((M + TBM - 1) / TBM) * ((N + TBN - 1) / TBN);
+    dim3 grid((unsigned)std::min<int64_t>(tiles, sm_count()));  // persistent: at most one block per SM
     ProfScope prof("qgemm_tc", st);
     qgemm_tc_kernel<<<grid, TC_THREADS, smem, st>>>(mA, mW, a);
     QNN_CUDA_TRY(cudaGetLastError());
