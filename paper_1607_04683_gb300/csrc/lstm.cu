@@ -556,6 +556,7 @@ extern "C" void qnn_lstm_model_destroy(qnn_lstm_model *m) {
     cudaFree(m->weights);
     cudaFree(m->ws);
     cudaFree(m->sws);
+    cudaFree(m->tcw);
     cudaSetDevice(prev);
     delete m;
 }
@@ -762,12 +763,18 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const bool x_dev = is_device_ptr(x), y_dev = is_device_ptr(y);
     const bool hs_dev = h_state && is_device_ptr(h_state), cs_dev = c_state && is_device_ptr(c_state);
     const bool ha_dev = h_all && is_device_ptr(h_all);
-    if (path_choice() != PathChoice::kLayerwise) {
+    const PathChoice choice = path_choice();
+    if (choice == PathChoice::kAuto || choice == PathChoice::kSmall) {
         bool used = false;
         QNN_TRY(small_path_forward(m, x, B, T, y, h_state, c_state, h_all, st, &used));
         if (used) return QNN_OK;
-        if (path_choice() == PathChoice::kSmall) return QNN_ERR_INVALID_ARG;
+        if (choice == PathChoice::kSmall) return QNN_ERR_INVALID_ARG;
     }
+    // recurrence: tensor cores for large batches, else the persistent integer-MMA kernel
+    const bool use_tc = tc_recurrence_supported(m) && (!ha_dev || (reinterpret_cast<uintptr_t>(h_all) & 15) == 0) &&
+                        (choice == PathChoice::kTc || (choice == PathChoice::kAuto && B >= kTcMinBatch));
+    if (choice == PathChoice::kTc && !use_tc) return QNN_ERR_INVALID_ARG;
+    if (use_tc) QNN_TRY(tc_prepare(m));
     const FwdPlan plan = plan_recurrent(m, B);
 
     // workspace layout
@@ -794,6 +801,7 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const size_t o_qs = acct(B * 4);
     const size_t o_lg = acct(C > 0 ? rows * C * 4 : 0);
     const size_t o_y = y_dev ? 0 : acct(rows * ycols * 4);
+    const size_t o_tc = use_tc ? acct(tc_work_bytes(m, B)) : 0;
     if (need > m->ws_bytes) {
         if (m->ws) {
             QNN_CUDA_TRY(cudaStreamSynchronize(st));
@@ -852,30 +860,34 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
             QNN_CUDA_TRY(cudaMemcpyAsync(cbuf, c_state + l * B * H, B * H * 4, cudaMemcpyDefault, st));
         else
             QNN_CUDA_TRY(cudaMemsetAsync(cbuf, 0, B * H * 4, st));
-        QNN_CUDA_TRY(cudaMemsetAsync(bar, 0, 256, st));
-        RecArgs a{};
-        a.wh = ly.wh.codes, a.wh_sum = ly.wh.sums, a.wh_p = ly.wh.params;
-        a.px = px, a.h0 = h0 + l * B * R, a.cbuf = cbuf, a.out = outl;
-        a.wp = P > 0 ? ly.wp.codes : nullptr, a.wp_sum = P > 0 ? ly.wp.sums : nullptr;
-        a.wp_p = P > 0 ? ly.wp.params : nullptr, a.mbuf = mbuf;
-        a.bar = bar, a.abort_flag = abort_flag, a.status = status;
-        a.B = (int)B, a.T = (int)T, a.H = (int)H, a.R = (int)R, a.P = (int)P;
-        a.ldh = (int)ly.wh.ld, a.ldp = P > 0 ? (int)ly.wp.ld : 0;
-        a.nc = plan.nc, a.np = plan.np, a.bc = plan.bc;
-        a.qcodes = reinterpret_cast<uint8_t *>(ws + o_qc);
-        a.qprm = reinterpret_cast<qnn_qparams *>(ws + o_qp);
-        a.qsum = reinterpret_cast<int *>(ws + o_qs);
-        a.ldq = (int)ldq;
-        a.distq = B >= kDistQuantMinBatch;  // below this, each block quantizing its rows is cheaper
-        void *args[] = {&a};
-        ProfScope prof("lstm_recurrent", st);
-        cudaError_t e = cudaLaunchCooperativeKernel((const void *)lstm_recurrent_kernel, dim3(plan.grid),
-                                                    dim3(kRecThreads), args, plan.smem, st);
-        if (e == cudaErrorCooperativeLaunchTooLarge) {
-            cudaGetLastError();
-            return QNN_ERR_NO_COOP;
+        if (use_tc) {
+            QNN_TRY(tc_layer_recurrence(m, l, px, h0 + l * B * R, cbuf, outl, mbuf, B, T, ws + o_tc, st));
+        } else {
+            QNN_CUDA_TRY(cudaMemsetAsync(bar, 0, 256, st));
+            RecArgs a{};
+            a.wh = ly.wh.codes, a.wh_sum = ly.wh.sums, a.wh_p = ly.wh.params;
+            a.px = px, a.h0 = h0 + l * B * R, a.cbuf = cbuf, a.out = outl;
+            a.wp = P > 0 ? ly.wp.codes : nullptr, a.wp_sum = P > 0 ? ly.wp.sums : nullptr;
+            a.wp_p = P > 0 ? ly.wp.params : nullptr, a.mbuf = mbuf;
+            a.bar = bar, a.abort_flag = abort_flag, a.status = status;
+            a.B = (int)B, a.T = (int)T, a.H = (int)H, a.R = (int)R, a.P = (int)P;
+            a.ldh = (int)ly.wh.ld, a.ldp = P > 0 ? (int)ly.wp.ld : 0;
+            a.nc = plan.nc, a.np = plan.np, a.bc = plan.bc;
+            a.qcodes = reinterpret_cast<uint8_t *>(ws + o_qc);
+            a.qprm = reinterpret_cast<qnn_qparams *>(ws + o_qp);
+            a.qsum = reinterpret_cast<int *>(ws + o_qs);
+            a.ldq = (int)ldq;
+            a.distq = B >= kDistQuantMinBatch;  // below this, each block quantizing its rows is cheaper
+            void *args[] = {&a};
+            ProfScope prof("lstm_recurrent", st);
+            cudaError_t e = cudaLaunchCooperativeKernel((const void *)lstm_recurrent_kernel, dim3(plan.grid),
+                                                        dim3(kRecThreads), args, plan.smem, st);
+            if (e == cudaErrorCooperativeLaunchTooLarge) {
+                cudaGetLastError();
+                return QNN_ERR_NO_COOP;
+            }
+            QNN_CUDA_TRY(e);
         }
-        QNN_CUDA_TRY(e);
         if (h_state) {  // final h of this layer = its output at the last frame
             QNN_CUDA_TRY(cudaMemcpy2DAsync(h_state + l * B * R, R * 4, outl + (T - 1) * R, T * R * 4, R * 4, B,
                                            cudaMemcpyDefault, st));

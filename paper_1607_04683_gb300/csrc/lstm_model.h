@@ -6,6 +6,8 @@
 
 #include "qnn_host.h"
 
+struct __half;
+
 namespace qnn {
 
 struct QUnitDev {  // one quantized weight matrix (or the four gate matrices of one kind)
@@ -20,6 +22,12 @@ struct LayerDev {
     QUnitDev wx, wh, wp;    // wx/wh: 4 gate blocks of H rows (row g*H + j); wp: P x H
     float *bias = nullptr;  // [4H]
     int64_t kin = 0;
+};
+
+struct TcLayer {  // fp16 centered weight copies for the tensor-core recurrence (lstm_tc.cu)
+    __half *wh16 = nullptr;  // [4 * round_up(H, 8)][kh]: gate rows interleaved in 8-cell groups
+    __half *wp16 = nullptr;  // [P][kp] (P > 0)
+    int64_t kh = 0, kp = 0;
 };
 
 }  // namespace qnn
@@ -39,6 +47,9 @@ struct qnn_lstm_model {
     void *sws = nullptr;
     size_t sws_bytes = 0;
     uint32_t epoch = 0;
+    // fp16 weight copies of the tensor-core recurrence (made on first use)
+    void *tcw = nullptr;
+    std::vector<qnn::TcLayer> tc_layers;
     // host mirror of the unit parameters (filled at creation)
     std::vector<qnn_qparams> host_params;
 };
@@ -49,8 +60,22 @@ namespace qnn {
 // Arguments as for qnn_lstm_forward.
 qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
                               float *c_state, float *h_all, cudaStream_t st, bool *used);
-// Which forward path to take, from the QNN_LSTM_PATH environment variable: "layerwise", "small"
-// or unset/"auto" (small when it qualifies).
-enum class PathChoice { kAuto, kLayerwise, kSmall };
+// Which forward path to take, from the QNN_LSTM_PATH environment variable: "layerwise" (the
+// persistent integer-MMA recurrence), "tc" (the tensor-core recurrence), "small" or unset/"auto"
+// (small when it qualifies, else tc for batches of at least kTcMinBatch, else layerwise).
+enum class PathChoice { kAuto, kLayerwise, kTc, kSmall };
 PathChoice path_choice();
+constexpr int64_t kTcMinBatch = 64;
+
+// Tensor-core recurrence (lstm_tc.cu). Supported when H is a multiple of 4 and the recurrent input
+// (R values) fits one exact accumulation chunk (round_up(R, 64) <= 1024).
+bool tc_recurrence_supported(const qnn_lstm_model *m);
+// Makes the fp16 weight copies (once per model).
+qnn_status tc_prepare(qnn_lstm_model *m);
+// Device workspace bytes tc_layer_recurrence needs for a batch of B.
+size_t tc_work_bytes(const qnn_lstm_model *m, int64_t B);
+// The T recurrent steps of layer l: px [B*T][4H] (row b*T + t) recovered input products plus bias,
+// h0 [B][R], cbuf [B][H] cell state in/out, out [B][T][R] layer outputs, mbuf [B][H] (P > 0).
+qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
+                               float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st);
 }  // namespace qnn

@@ -652,6 +652,7 @@ PathChoice path_choice() {
     if (!v || !*v || std::strcmp(v, "auto") == 0) return PathChoice::kAuto;
     if (std::strcmp(v, "layerwise") == 0) return PathChoice::kLayerwise;
     if (std::strcmp(v, "small") == 0) return PathChoice::kSmall;
+    if (std::strcmp(v, "tc") == 0) return PathChoice::kTc;
     return PathChoice::kAuto;
 }
 

@@ -20,25 +20,56 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <cstdio>
 #include <cstdlib>
 #include <algorithm>
 #include <mutex>
 
 #include "qnn_device.cuh"
 #include "qnn_host.h"
+#include "tc_gemm.h"
 
 namespace qnn {
 namespace {
 
-constexpr int TBM = 128, TBN = 256, TBK = 64;     // fp16 elements per k-block (128 bytes)
-constexpr int TSTAGES = 3;
+constexpr int TBM = 128, TBK = 64;               // rows of A per tile; fp16 elements per k-block (128 bytes)
 constexpr int A_BYTES = TBM * TBK * 2;            // 16 KB
-constexpr int B_BYTES = TBN * TBK * 2;            // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TC_THREADS = 10 * 32;
 constexpr int KCHUNK = 1024;                      // exact fp32 accumulation bound (see above)
-constexpr int TMEM_COLS = 512;                    // two 128 x 256 fp32 accumulators
 constexpr unsigned long long TC_WAIT_NS = 2000000000ull;
+
+// kEpiLinear: recovered product, any K (chunked drains), outputs staged through shared memory.
+// kEpiRow: recovered product for K <= 1024, one output row per lane, two blocks per SM.
+// kEpiLstm: the LSTM cell update on gate-interleaved columns, K <= 1024, two blocks per SM.
+enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2 };
+
+struct ColConst {  // per-output-column constants of kEpiRow, staged in shared memory per tile
+    int cs, zw;
+    float Qw, bias;
+};
+
+// Per tile width BN (rows of W per tile) and epilogue: warps (TMA producer, MMA issuer, then the
+// epilogue warps), stage ring depth, tensor-memory columns (two fp32 accumulators of BN columns),
+// register cap, the epilogue's shared staging, and the MMA instruction descriptor (fp32
+// accumulator, fp16 A and B, both K-major, M = 128, N = BN). A block that allocates tensor memory
+// has its SM to itself, so the ALU-bound row and LSTM epilogues run sixteen warps (four per
+// tensor-memory lane quarter); eighteen warps fit the register file at 96 registers a thread.
+template <int BN, int EPI>
+struct Tile {
+    static_assert(EPI == kEpiLinear || BN <= 128, "row and LSTM epilogues take tiles of at most 128 columns");
+    static constexpr int EPI_WARPS = EPI == kEpiLinear ? 8 : 16;
+    static constexpr int THREADS = 32 * (2 + EPI_WARPS);
+    static constexpr int B_BYTES = BN * TBK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int STAGES = EPI == kEpiLinear ? (BN == 256 ? 3 : (BN == 128 ? 4 : 6)) : (BN == 128 ? 4 : 6);
+    static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
+    static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : 96;
+    static constexpr int EPI_BYTES = EPI == kEpiLinear ? (8 * 32 * 33 + 8 * 96) * 4
+                                     : EPI == kEpiRow  ? 2 * BN * (int)sizeof(ColConst)
+                                                       : 0;
+    static constexpr uint32_t IDESC =
+        (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TBM >> 4) << 24);
+    static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + EPI_BYTES + 256;
+};
 
 struct TcArgs {
     const qnn_qparams *pa;
@@ -55,6 +86,7 @@ struct TcArgs {
     int K;      // true K
     int KB;     // k-blocks of 64
     int *status;
+    TcLstmOut lstm;  // kEpiLstm only
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
@@ -115,9 +147,7 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
     return d;
 }
 
-// Instruction descriptor: fp32 accumulator, fp16 A and B, both K-major, M = 128, N = 256.
-constexpr uint32_t IDESC = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(TBN >> 3) << 17) | ((uint32_t)(TBM >> 4) << 24);
-
+template <uint32_t IDESC>
 __device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
     asm volatile(
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
@@ -129,10 +159,10 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
 
-template <int N>
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[N]);
-template <>
-__device__ __forceinline__ void tmem_ld32<32>(uint32_t taddr, uint32_t (&r)[32]) {
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// 32 consecutive fp32 columns of this warp's 32 tensor-memory lanes (one row per lane).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
         "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
@@ -141,45 +171,68 @@ __device__ __forceinline__ void tmem_ld32<32>(uint32_t taddr, uint32_t (&r)[32])
           "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
           "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
         : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    tmem_wait_ld();
+}
+// 16 consecutive fp32 columns.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    tmem_wait_ld();
+}
+// 4 consecutive fp32 columns, without the wait (the caller waits once for several loads).
+__device__ __forceinline__ void tmem_ld4_nowait(uint32_t taddr, uint32_t (&r)[4]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(taddr));
 }
 
-__global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_constant__ CUtensorMap mapA,
-                                                                 const __grid_constant__ CUtensorMap mapW,
-                                                                 const TcArgs args) {
+// Persistent tile loop. Warp 0: TMA producer; warp 1: tensor-memory owner and MMA issuer; warps
+// 2.. : epilogue. EPI = kEpiLinear / kEpiRow write the recovered product (plus bias) and
+// optionally the raw int32 accumulator; EPI = kEpiLstm treats the columns as gate-interleaved LSTM
+// pre-activations (8-cell groups of [i f g o] x 8 rows of W) and applies the cell update (K <= 1024).
+// With a programmatic dependent launch the block setup overlaps the previous kernel of the stream.
+template <int BN, int EPI>
+__global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN, EPI>::MAX_REGS))
+    qgemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapW,
+                    const TcArgs args) {
+    using TL = Tile<BN, EPI>;
+    constexpr int STAGES = TL::STAGES;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // 1024-byte alignment for the swizzled tiles
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    int *stage_out = reinterpret_cast<int *>(smem + TSTAGES * STAGE_BYTES);        // [8 warps][32][33]
-    int *row_c = stage_out + 8 * 32 * 33;                                          // [8 warps][3][32]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(row_c + 8 * 3 * 32);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * TSTAGES + 4);
-    const uint32_t full0 = su32(bars), empty0 = su32(bars + TSTAGES), chunk0 = su32(bars + 2 * TSTAGES),
-                   drained0 = su32(bars + 2 * TSTAGES + 2);
+    int *stage_out = reinterpret_cast<int *>(smem + STAGES * TL::STAGE_BYTES);     // [8 warps][32][33] (linear)
+    int *row_c = stage_out + 8 * 32 * 33;                                          // [8 warps][3][32] (linear)
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + STAGES * TL::STAGE_BYTES + TL::EPI_BYTES);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 4);
+    const uint32_t full0 = su32(bars), empty0 = su32(bars + STAGES), chunk0 = su32(bars + 2 * STAGES),
+                   drained0 = su32(bars + 2 * STAGES + 2);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int KB = args.KB;
     const int kpc = KCHUNK / TBK;  // k-blocks per chunk (16)
     const int nchunks = (KB + kpc - 1) / kpc;
-    const int tiles_n = (int)((args.N + TBN - 1) / TBN);
+    const int tiles_n = (int)((args.N + BN - 1) / BN);
     const int64_t tiles = (int64_t)((args.M + TBM - 1) / TBM) * tiles_n;
     __shared__ int s_abort;
 
     if (threadIdx.x == 0) {
         s_abort = 0;
-        for (int i = 0; i < TSTAGES; ++i) {
+        for (int i = 0; i < STAGES; ++i) {
             mb_init(full0 + 8 * i, 1);
             mb_init(empty0 + 8 * i, 1);
         }
         for (int i = 0; i < 2; ++i) {
             mb_init(chunk0 + 8 * i, 1);      // MMA -> epilogue: chunk accumulated in buffer i
-            mb_init(drained0 + 8 * i, 8);    // epilogue -> MMA: buffer i read out (8 epilogue warps)
+            mb_init(drained0 + 8 * i, TL::EPI_WARPS);  // epilogue -> MMA: buffer i read out by every epilogue warp
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     if (warp == 1) {  // allocate the two accumulators
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)),
-                     "r"(TMEM_COLS)
+                     "n"(TL::TMEM_COLS)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -187,6 +240,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem_base = *tmem_slot;
+    // With a programmatic dependent launch the setup above overlaps the previous kernel of the
+    // stream; its outputs (this kernel's operands) are complete and visible after this wait.
+    grid_dependency_wait();
+    grid_dependents_launch();
 
     // Persistent: block b takes tiles b, b + grid, ... (row-tile major, so neighbouring blocks share
     // the same rows of A through L2). The k-block and chunk counters run across tiles, so the two
@@ -196,15 +253,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
         if (lane == 0) {
             int64_t g = 0;  // k-blocks issued by this block
             for (int64_t tile = blockIdx.x; tile < tiles && !s_abort; tile += gridDim.x) {
-                const int m0 = (int)(tile / tiles_n) * TBM, n0 = (int)(tile % tiles_n) * TBN;
+                const int m0 = (int)(tile / tiles_n) * TBM, n0 = (int)(tile % tiles_n) * BN;
                 for (int kb = 0; kb < KB; ++kb, ++g) {
-                    const int s = (int)(g % TSTAGES);
-                    if (g >= TSTAGES && !mb_wait(empty0 + 8 * s, (unsigned)((g / TSTAGES) - 1) & 1, args.status)) {
+                    const int s = (int)(g % STAGES);
+                    if (g >= STAGES && !mb_wait(empty0 + 8 * s, (unsigned)((g / STAGES) - 1) & 1, args.status)) {
                         s_abort = 1;
                         break;
                     }
-                    const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
-                    mb_expect(full0 + 8 * s, STAGE_BYTES);
+                    const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
+                    mb_expect(full0 + 8 * s, TL::STAGE_BYTES);
                     tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
                     tma_load_2d(sb, &mapW, full0 + 8 * s, kb * TBK, n0);
                 }
@@ -216,7 +273,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
             int64_t g = 0, gc = 0;  // k-blocks and chunks consumed by this block
             for (int64_t tile = blockIdx.x; tile < tiles && !s_abort; tile += gridDim.x) {
                 for (int kb = 0; kb < KB; ++kb, ++g) {
-                    const int s = (int)(g % TSTAGES);
+                    const int s = (int)(g % STAGES);
                     const int kc = kb % kpc;
                     const int buf = (int)(gc & 1);
                     if (kc == 0 && gc >= 2 &&
@@ -224,17 +281,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
                         s_abort = 1;
                         break;
                     }
-                    if (!mb_wait(full0 + 8 * s, (unsigned)(g / TSTAGES) & 1, args.status)) {
+                    if (!mb_wait(full0 + 8 * s, (unsigned)(g / STAGES) & 1, args.status)) {
                         s_abort = 1;
                         break;
                     }
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                    const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
-                    const uint32_t tmem_d = tmem_base + (uint32_t)(buf * TBN);
+                    const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
+                    const uint32_t tmem_d = tmem_base + (uint32_t)(buf * BN);
 #pragma unroll
                     for (int k = 0; k < TBK / 16; ++k) {
                         // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
-                        mma_f16(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k), (kc == 0 && k == 0) ? 0u : 1u);
+                        mma_f16<TL::IDESC>(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k),
+                                           (kc == 0 && k == 0) ? 0u : 1u);
                     }
                     mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
                     if (kc == kpc - 1 || kb == KB - 1) {
@@ -245,10 +303,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
                 if (s_abort) break;
             }
         }
-    } else {
-        // ---------------- epilogue (warps 2..9) ----------------
+    } else if constexpr (EPI == kEpiLinear) {
+        // ---------------- epilogue (warps 2..9): recovered product ----------------
+        constexpr int NJ = BN / 64;             // 32-column blocks per warp
         const int q = warp & 3;                 // tensor-memory lane quarter this warp may read
-        const int half = (warp - 2) >> 2;       // column half: 0 -> [0, 128), 1 -> [128, 256)
+        const int half = (warp - 2) >> 2;       // column half: [0, BN/2) or [BN/2, BN)
         const int ew = warp - 2;
         int *stg = stage_out + ew * 32 * 33;
         int *rz = row_c + ew * 96, *rr = rz + 32;
@@ -257,7 +316,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
         int64_t gc = 0;
         bool ok = true;
         for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * TBN;
+            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * BN;
             {  // this lane's row constants, shared with the warp for the transposed stores
                 const int64_t m = m0 + 32 * q + lane;
                 const bool mv = m < args.M;
@@ -294,7 +353,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
                 __syncwarp();
             };
             auto taddr_of = [&](int buf, int j) {
-                return tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * TBN + half * 128 + 32 * j);
+                return tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + half * (BN / 2) + 32 * j);
             };
             __syncwarp();
             if (nchunks == 1) {  // K <= 1024: read the accumulator and finish directly
@@ -303,13 +362,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
                 if (!ok) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll 1
-                for (int j = 0; j < 4; ++j) {
+                for (int j = 0; j < NJ; ++j) {
                     uint32_t r[32];
-                    tmem_ld32<32>(taddr_of(buf, j), r);
+                    tmem_ld32(taddr_of(buf, j), r);
                     int P[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) P[i] = __float2int_rn(__uint_as_float(r[i]));
-                    emit(half * 128 + 32 * j, P);
+                    emit(half * (BN / 2) + 32 * j, P);
                 }
                 // the accumulator is free again: the tile after next may use it
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -318,9 +377,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
                     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
                 ++gc;
             } else {  // drain every chunk into int32 running sums
-                int run[4][32];
+                int run[NJ][32];
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
+                for (int j = 0; j < NJ; ++j)
 #pragma unroll
                     for (int i = 0; i < 32; ++i) run[j][i] = 0;
                 for (int c = 0; c < nchunks; ++c, ++gc) {
@@ -329,9 +388,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
                     if (!ok) break;
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
+                    for (int j = 0; j < NJ; ++j) {
                         uint32_t rr32[32];
-                        tmem_ld32<32>(taddr_of(buf, j), rr32);
+                        tmem_ld32(taddr_of(buf, j), rr32);
 #pragma unroll
                         for (int i = 0; i < 32; ++i) run[j][i] += __float2int_rn(__uint_as_float(rr32[i]));
                     }
@@ -342,8 +401,191 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
                 }
                 if (!ok) break;
 #pragma unroll
-                for (int j = 0; j < 4; ++j) emit(half * 128 + 32 * j, run[j]);
+                for (int j = 0; j < NJ; ++j) emit(half * (BN / 2) + 32 * j, run[j]);
             }
+        }
+    } else if constexpr (EPI == kEpiRow) {
+        // ---------------- epilogue (warps 2..17): recovered product, one row per lane ----------------
+        // Each lane owns one output row; the four warps of a lane quarter take its 16-column blocks
+        // in turn: eq. (1)'s offsets and eq. (3)'s recovery per element, stored as 16-byte vectors
+        // (ragged edges element by element). The column constants of the tile are staged in shared
+        // memory (double-buffered by tile parity; one named barrier of the epilogue warps per tile).
+        ColConst *scol = reinterpret_cast<ColConst *>(smem + STAGES * TL::STAGE_BYTES);
+        const int q = warp & 3;
+        const int part = (warp - 2) >> 2;
+        const int ew = warp - 2;
+        const int K = args.K;
+        const bool vec = args.Y && (args.ldy % 4 == 0) && ((reinterpret_cast<uintptr_t>(args.Y) & 15) == 0);
+        // Every epilogue warp runs every tile (the named barrier counts on it); after a wait gave
+        // up, the remaining tiles are skipped without waiting.
+        int64_t gc = 0;
+        bool failed = false;
+        for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * BN;
+            ColConst *cc = scol + (gc & 1) * BN;
+            for (int c = ew * 32 + lane; c < BN; c += 32 * TL::EPI_WARPS) {
+                const int64_t n = n0 + c;
+                ColConst v{0, 0, 1.0f, 0.0f};
+                if (n < args.N) {
+                    const qnn_qparams qw = args.pw[n / args.rows_per_block];
+                    v.cs = args.csW[n];
+                    v.zw = qw.z;
+                    v.Qw = qw.Q;
+                    v.bias = args.bias ? args.bias[n] : 0.0f;
+                }
+                cc[c] = v;
+            }
+            asm volatile("bar.sync 1, %0;" ::"n"(32 * TL::EPI_WARPS) : "memory");
+            const int64_t m = m0 + 32 * q + lane;
+            const bool mv = m < args.M;
+            int za = 0, ra = 0;
+            float Qa = 1.0f;
+            if (mv) {
+                const qnn_qparams qa = args.pa[args.a_per_row ? m : 0];
+                za = qa.z;
+                Qa = qa.Q;
+                ra = args.rsA[m];
+            }
+            const long long za128 = 128 + za;
+            const int buf = (int)(gc & 1);
+            if (!failed && *reinterpret_cast<volatile int *>(&s_abort)) failed = true;
+            if (!failed) {
+                failed = !__all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
+                if (failed) *reinterpret_cast<volatile int *>(&s_abort) = 1;
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll 1
+            for (int j = part; j < BN / 16 && !failed; j += TL::EPI_WARPS / 4) {
+                const int c0 = 16 * j;
+                uint32_t r[16];
+                tmem_ld16(tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + c0), r);
+                const int64_t nb = n0 + c0;
+                if (!mv || nb >= args.N) continue;
+                // one weight unit across the 16 columns (the usual case): row terms hoisted
+                const bool one_unit = (nb / args.rows_per_block) == ((nb + 15) / args.rows_per_block);
+                long long rt = 0;
+                float den = 0.0f;
+                if (one_unit) {
+                    const int zw = cc[c0].zw;
+                    rt = (long long)(128 + zw) * ra + (long long)K * ((long long)za * zw - 16384);
+                    den = __fmul_rn(Qa, cc[c0].Qw);
+                }
+                float *yr = args.Y ? args.Y + m * args.ldy + nb : nullptr;
+                const bool full = vec && nb + 16 <= args.N;
+#pragma unroll
+                for (int v4 = 0; v4 < 4; ++v4) {
+                    float y[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int i = 4 * v4 + e;
+                        const ColConst v = cc[c0 + i];
+                        const int P = __float2int_rn(__uint_as_float(r[i]));
+                        long long S;
+                        float dn;
+                        if (one_unit) {
+                            S = (long long)P + rt + za128 * v.cs;
+                            dn = den;
+                        } else {
+                            S = (long long)P + (long long)(128 + v.zw) * ra + za128 * v.cs +
+                                (long long)K * ((long long)za * v.zw - 16384);
+                            dn = __fmul_rn(Qa, v.Qw);
+                        }
+                        y[e] = __fdiv_rn(__ll2float_rn(S), dn);
+                        if (args.bias) y[e] = __fadd_rn(y[e], v.bias);
+                        if (args.acc_out && nb + i < args.N)
+                            args.acc_out[m * args.N + nb + i] = P + 128 * (ra + v.cs) - 16384 * K;  // raw code product
+                    }
+                    if (full) {
+                        *reinterpret_cast<float4 *>(yr + 4 * v4) = make_float4(y[0], y[1], y[2], y[3]);
+                    } else if (yr) {
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            if (nb + 4 * v4 + e < args.N) yr[4 * v4 + e] = y[e];
+                    }
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+            ++gc;
+        }
+    } else {
+        // ---------------- epilogue (warps 2..17): LSTM cell update ----------------
+        // Column n of the tile is gate g = (n % 32) / 8 of cell 8 * (n / 32) + n % 8. Each lane owns
+        // one batch row; the four warps of a lane quarter take 4-cell slices in turn, reading the
+        // four gates of their cells from tensor memory, so a thread has everything for eq. (1)/(3)
+        // and the cell update of 4 cells.
+        const int q = warp & 3;
+        const int eh = (warp - 2) >> 2;
+        const int K = args.K;
+        const TcLstmOut &E = args.lstm;
+        const int H = E.H;
+        int64_t gc = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * BN;
+            const int64_t b = m0 + 32 * q + lane;
+            const bool bv = b < args.M;
+            int za = 0, rs = 0;
+            float Qa = 1.0f;
+            if (bv) {
+                const qnn_qparams qa = args.pa[b];
+                za = qa.z;
+                Qa = qa.Q;
+                rs = args.rsA[b];
+            }
+            // eq. (1) expanded around the centered product P: S = P + rt[g] + (128 + za) csW
+            long long rt[4];
+            float den[4];
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+                const qnn_qparams qw = args.pw[g];
+                rt[g] = (long long)(128 + qw.z) * rs + (long long)K * ((long long)za * qw.z - 16384);
+                den[g] = __fmul_rn(Qa, qw.Q);
+            }
+            const long long za128 = 128 + za;
+            const int buf = (int)(gc & 1);
+            ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll 1
+            for (int s = eh; s < BN / 16; s += TL::EPI_WARPS / 4) {
+                const int gi = s >> 1, part = s & 1;
+                const int j0 = (int)(n0 / 4) + gi * 8 + part * 4;  // H is a multiple of 4: all 4 valid or none
+                uint32_t r[4][4];
+                const uint32_t ta = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + gi * 32 + part * 4);
+#pragma unroll
+                for (int g = 0; g < 4; ++g) tmem_ld4_nowait(ta + 8 * g, r[g]);
+                tmem_wait_ld();
+                if (bv && j0 < H) {
+                    const float *pxr = E.px + b * E.px_ld + j0;
+                    float *cr = E.c + b * (int64_t)H + j0;
+                    float pre[4][4];
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        const float4 v = *reinterpret_cast<const float4 *>(pxr + (int64_t)g * H);
+                        const int4 cs = *reinterpret_cast<const int4 *>(args.csW + g * H + j0);
+                        const int csv[4] = {cs.x, cs.y, cs.z, cs.w};
+                        const float pv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                        for (int jj = 0; jj < 4; ++jj) {
+                            const long long S =
+                                (long long)__float2int_rn(__uint_as_float(r[g][jj])) + rt[g] + za128 * csv[jj];
+                            pre[g][jj] = __fadd_rn(pv[jj], __fdiv_rn(__ll2float_rn(S), den[g]));
+                        }
+                    }
+                    float4 c4 = *reinterpret_cast<const float4 *>(cr);
+                    float cv[4] = {c4.x, c4.y, c4.z, c4.w}, mv[4];
+#pragma unroll
+                    for (int jj = 0; jj < 4; ++jj) lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
+                    *reinterpret_cast<float4 *>(cr) = make_float4(cv[0], cv[1], cv[2], cv[3]);
+                    *reinterpret_cast<float4 *>(E.h + b * E.h_ld + j0) = make_float4(mv[0], mv[1], mv[2], mv[3]);
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+            ++gc;
         }
     }
     __syncwarp();
@@ -357,7 +599,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) qgemm_tc_kernel(const __grid_co
     __syncthreads();
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "n"(TL::TMEM_COLS)
                      : "memory");
     }
 }
@@ -419,44 +661,162 @@ size_t tc_scratch_bytes(int64_t M, int64_t N, int64_t K) {
     return (size_t)(M + N) * kp * 2 + 512;
 }
 
+namespace {
+
+template <int BN, int EPI>
+qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cudaStream_t st) {
+    using TL = Tile<BN, EPI>;
+    static int configured = -1;
+    int dev = 0;
+    QNN_CUDA_TRY(cudaGetDevice(&dev));
+    if (configured != dev) {
+        QNN_CUDA_TRY(cudaFuncSetAttribute(qgemm_tc_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)TL::SMEM));
+        QNN_CUDA_TRY(cudaFuncSetAttribute(qgemm_tc_kernel<BN, EPI>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                          (int)cudaSharedmemCarveoutMaxShared));
+        int n = 0;
+        QNN_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, qgemm_tc_kernel<BN, EPI>, TL::THREADS, TL::SMEM));
+        if (n < 1) return QNN_ERR_CUDA;
+        configured = dev;
+        if (std::getenv("QNN_DEBUG")) {
+            cudaFuncAttributes fa{};
+            cudaFuncGetAttributes(&fa, qgemm_tc_kernel<BN, EPI>);
+            std::fprintf(stderr, "qnn: qgemm_tc_kernel<%d,%d>: %d threads, %d registers, %zu bytes dynamic shared, "
+                         "%d blocks per SM\n", BN, EPI, TL::THREADS, fa.numRegs, TL::SMEM, n);
+        }
+    }
+    const int64_t tiles = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN);
+    // persistent: one block per SM (a block holding tensor memory has its SM to itself)
+    const unsigned grid = (unsigned)std::min<int64_t>(tiles, (int64_t)sm_count());
+    ProfScope prof(name, st);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(TL::THREADS);
+    cfg.dynamicSmemBytes = TL::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = op.pdl ? 1 : 0;
+    QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, qgemm_tc_kernel<BN, EPI>, op.a, op.w, a));
+    return QNN_OK;
+}
+
+qnn_status dispatch_linear(const TcOperands &op, const TcArgs &a, cudaStream_t st) {
+    if (op.row_epilogue) {
+        switch (op.bn) {
+            case 64: return launch_tc<64, kEpiRow>(op, a, "qgemm_tc", st);
+            case 128: return launch_tc<128, kEpiRow>(op, a, "qgemm_tc", st);
+            default: return QNN_ERR_INVALID_ARG;
+        }
+    }
+    switch (op.bn) {
+        case 64: return launch_tc<64, kEpiLinear>(op, a, "qgemm_tc", st);
+        case 128: return launch_tc<128, kEpiLinear>(op, a, "qgemm_tc", st);
+        case 256: return launch_tc<256, kEpiLinear>(op, a, "qgemm_tc", st);
+        default: return QNN_ERR_INVALID_ARG;
+    }
+}
+
+qnn_status dispatch_lstm(const TcOperands &op, const TcArgs &a, cudaStream_t st) {
+    switch (op.bn) {
+        case 32: return launch_tc<32, kEpiLstm>(op, a, "lstm_gates_tc", st);
+        case 64: return launch_tc<64, kEpiLstm>(op, a, "lstm_gates_tc", st);
+        case 128: return launch_tc<128, kEpiLstm>(op, a, "lstm_gates_tc", st);
+        default: return QNN_ERR_INVALID_ARG;
+    }
+}
+
+}  // namespace
+
+int tc_choose_bn(int64_t M, int64_t N, const int *cands, int n) {
+    if (const char *e = std::getenv("QNN_TC_BN")) {
+        const int v = std::atoi(e);
+        for (int i = 0; i < n; ++i)
+            if (cands[i] == v) return v;
+    }
+    const int64_t mt = (M + TBM - 1) / TBM, sms = sm_count();
+    double eff[8] = {0};
+    double best = 0.0;
+    for (int i = 0; i < n; ++i) {
+        const int64_t tiles = mt * ((N + cands[i] - 1) / cands[i]);
+        const int64_t waves = (tiles + sms - 1) / sms;
+        eff[i] = (double)tiles / (double)(waves * sms);
+        best = std::max(best, eff[i]);
+    }
+    for (int i = 0; i < n; ++i)  // candidates widest first
+        if (eff[i] >= 0.9 * best) return cands[i];
+    return cands[n - 1];
+}
+
+int tc_pick_bn(int64_t M, int64_t N, int64_t kp) {
+    if (kp > KCHUNK) {  // chunked drains through the staged epilogue: widest tile
+        static const int c[] = {256, 128, 64};
+        return tc_choose_bn(M, N, c, 3);
+    }
+    static const int c[] = {128, 64};  // row epilogue
+    return tc_choose_bn(M, N, c, 2);
+}
+
+qnn_status tc_operands(TcOperands *op, const __half *A16, int64_t M, const __half *W16, int64_t N, int64_t kp, int bn) {
+    if (bn != 32 && bn != 64 && bn != 128 && bn != 256) return QNN_ERR_INVALID_ARG;
+    if (kp <= 0 || kp % TBK != 0 || M <= 0 || N <= 0) return QNN_ERR_INVALID_ARG;
+    QNN_TRY(make_map(&op->a, A16, M, kp, TBM));
+    QNN_TRY(make_map(&op->w, W16, N, kp, bn));
+    op->M = M, op->N = N, op->kp = kp, op->bn = bn, op->pdl = false;
+    op->row_epilogue = kp <= KCHUNK && (bn == 64 || bn == 128);
+    return QNN_OK;
+}
+
+qnn_status tc_linear(const TcOperands &op, const qnn_qparams *pa, int per_row, const int32_t *rsA, int64_t K,
+                     const qnn_qparams *pw, int64_t rows_per_block, const int32_t *csW, const float *bias, float *Y,
+                     int64_t ldy, int32_t *acc_out, cudaStream_t st) {
+    if (K <= 0 || K > QNN_K_MAX || K > op.kp) return QNN_ERR_INVALID_ARG;
+    int *status = nullptr;
+    QNN_TRY(status_word(&status));
+    TcArgs a{pa, per_row, rsA, pw, rows_per_block, csW, bias, Y, ldy, acc_out, op.M, op.N, (int)K,
+             (int)(op.kp / TBK), status, TcLstmOut{}};
+    return dispatch_linear(op, a, st);
+}
+
+qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int32_t *rsA, int64_t K,
+                         const qnn_qparams *pw4, const int32_t *cs, const TcLstmOut &out, cudaStream_t st) {
+    if (K <= 0 || op.kp > KCHUNK || K > op.kp || out.H <= 0 || out.H % 4 != 0) return QNN_ERR_INVALID_ARG;
+    if (op.N != 4 * ((out.H + 7) / 8 * 8)) return QNN_ERR_INVALID_ARG;
+    int *status = nullptr;
+    QNN_TRY(status_word(&status));
+    TcArgs a{pa, 1, rsA, pw4, 0, cs, nullptr, nullptr, 0, nullptr, op.M, op.N, (int)K, (int)(op.kp / TBK), status, out};
+    return dispatch_lstm(op, a, st);
+}
+
+qnn_status launch_center_fp16(const uint8_t *in, int64_t rows, int64_t K, int64_t ldi, __half *out, int64_t ldo,
+                              cudaStream_t st) {
+    if (rows == 0) return QNN_OK;
+    const int64_t tot = rows * (ldo / 8);
+    center_fp16_kernel<<<(unsigned)std::min<int64_t>((tot + 255) / 256, 65535 * 4), 256, 0, st>>>(in, rows, (int)K, ldi,
+                                                                                                  out, (int)ldo);
+    QNN_CUDA_TRY(cudaGetLastError());
+    return QNN_OK;
+}
+
 // Centers A and W into fp16 scratch and runs the tensor-core product (K <= QNN_K_MAX).
 qnn_status launch_qgemm_tc(const uint8_t *A, int64_t lda, const qnn_qparams *pa, int ga, const int32_t *rsA, int64_t M,
                            int64_t K, const uint8_t *W, int64_t ldw, const qnn_qparams *pw, int64_t rows_per_block,
                            const int32_t *csW, int64_t N, const float *bias, float *Y, int64_t ldy, int32_t *acc_out,
                            void *scratch_ptr, cudaStream_t st) {
     if (M == 0 || N == 0) return QNN_OK;
-    const int kp = (int)((K + 63) / 64 * 64);
+    const int64_t kp = (K + 63) / 64 * 64;
     __half *A16 = reinterpret_cast<__half *>(scratch_ptr);
     __half *W16 = A16 + M * kp;
     {
         ProfScope prof("center_fp16", st);
-        const int64_t totA = M * (kp / 8), totW = N * (kp / 8);
-        center_fp16_kernel<<<(unsigned)std::min<int64_t>((totA + 255) / 256, 65535 * 4), 256, 0, st>>>(A, M, (int)K, lda,
-                                                                                                      A16, kp);
-        center_fp16_kernel<<<(unsigned)std::min<int64_t>((totW + 255) / 256, 65535 * 4), 256, 0, st>>>(W, N, (int)K, ldw,
-                                                                                                      W16, kp);
-        QNN_CUDA_TRY(cudaGetLastError());
+        QNN_TRY(launch_center_fp16(A, M, K, lda, A16, kp, st));
+        QNN_TRY(launch_center_fp16(W, N, K, ldw, W16, kp, st));
     }
-    CUtensorMap mA, mW;
-    QNN_TRY(make_map(&mA, A16, M, kp, TBM));
-    QNN_TRY(make_map(&mW, W16, N, kp, TBN));
-    int *status = nullptr;
-    QNN_TRY(status_word(&status));
-    TcArgs a{pa, ga == QNN_PER_ROW, rsA, pw, rows_per_block, csW, bias, Y, ldy, acc_out, M, N, (int)K, kp / TBK, status};
-    const size_t smem = (size_t)TSTAGES * STAGE_BYTES + 1024 + (8 * 32 * 33 + 8 * 96) * 4 + 256;
-    static int configured = -1;
-    int dev = 0;
-    QNN_CUDA_TRY(cudaGetDevice(&dev));
-    if (configured != dev) {
-        QNN_CUDA_TRY(cudaFuncSetAttribute(qgemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        configured = dev;
-    }
-    const int64_t tiles = ((M + TBM - 1) / TBM) * ((N + TBN - 1) / TBN);
-    dim3 grid((unsigned)std::min<int64_t>(tiles, sm_count()));  // persistent: at most one block per SM
-    ProfScope prof("qgemm_tc", st);
-    qgemm_tc_kernel<<<grid, TC_THREADS, smem, st>>>(mA, mW, a);
-    QNN_CUDA_TRY(cudaGetLastError());
-    return QNN_OK;
+    TcOperands op;
+    QNN_TRY(tc_operands(&op, A16, M, W16, N, kp, tc_pick_bn(M, N, kp)));
+    return tc_linear(op, pa, ga == QNN_PER_ROW, rsA, K, pw, rows_per_block, csW, bias, Y, ldy, acc_out, st);
 }
 
 }  // namespace qnn

@@ -118,6 +118,13 @@ __device__ __forceinline__ void lstm_cell(float pi, float pf, float pg, float po
     m = lstm_cell_update(ig, fg, gg, og, c);
 }
 
+// Programmatic dependent launch: a kernel launched with the programmatic stream serialization
+// attribute may start while the previous kernel of its stream is still running. The wait returns
+// once that kernel has completed and its memory operations are visible (at once without such a
+// launch); the trigger lets the next kernel of the stream start early.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Warp-wide reductions.
 __device__ __forceinline__ float warp_min(float v) {
 #pragma unroll

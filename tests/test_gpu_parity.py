@@ -356,6 +356,56 @@ def test_small_and_layerwise_paths_agree(qnn, cfg, monkeypatch):
     assert np.array_equal(outs["small"]["y"], outs["layerwise"]["y"])
 
 
+# Tensor-core recurrence (large batches): forced on small cases, every tile width
+TC_CASES = [dict(L=1, I=40, H=128, B=5, T=6), dict(L=2, I=40, H=100, C=37, B=130, T=4),
+            dict(L=2, I=24, H=256, P=96, C=11, B=33, T=5), dict(L=1, I=40, H=500, B=256, T=3, w=0.08, mu=0.5),
+            dict(L=1, I=8, H=1024, B=64, T=2, w=0.05), dict(L=2, I=80, H=1100, P=64, C=20, B=40, T=3, w=0.05),
+            dict(L=3, I=5, H=8, B=3, T=4, mu=0.5)]
+
+
+@pytest.mark.parametrize("bn", ["32", "64", "128"])
+@pytest.mark.parametrize("cfg", TC_CASES)
+def test_tc_recurrence_bit_exact(qnn, cfg, bn, monkeypatch):
+    wl = _small(**cfg)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x, want_h_all=True)
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    monkeypatch.setenv("QNN_TC_BN", bn)
+    qnn.profile_read()
+    qnn.profile_enable(True)
+    got = _gpu_forward(qnn, wl, params, x)
+    qnn.profile_enable(False)
+    kernels = qnn.profile_read()
+    assert "lstm_gates_tc" in kernels and "lstm_recurrent" not in kernels, kernels
+    _compare(got, ref, wl)
+
+
+def test_tc_recurrence_state_round_trip(qnn, monkeypatch):
+    """Streaming: two calls on halves of the frames give the single call's outputs and state."""
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    wl = _small(L=2, I=12, H=68, P=20, C=0, B=70, T=8)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x, want_h_all=True)
+    first = _gpu_forward(qnn, wl, params, x[:, :3])
+    second = _gpu_forward(qnn, wl, params, x[:, 3:], h0=first["h"], c0=first["c"])
+    assert np.array_equal(np.concatenate([first["h_all"], second["h_all"]], axis=2), ref["h_all"])
+    assert np.array_equal(second["h"], ref["h"]) and np.array_equal(second["c"], ref["c"])
+
+
+def test_large_batches_take_the_tc_path(qnn, monkeypatch):
+    monkeypatch.delenv("QNN_LSTM_PATH", raising=False)
+    monkeypatch.delenv("QNN_TC_BN", raising=False)
+    for B, want in ((63, False), (64, True)):
+        wl = _small(L=1, I=8, H=32, B=B, T=2)
+        params, x = wl.make()
+        qnn.profile_read()
+        qnn.profile_enable(True)
+        got = _gpu_forward(qnn, wl, params, x)
+        qnn.profile_enable(False)
+        assert ("lstm_gates_tc" in qnn.profile_read()) == want
+        _compare(got, _oracle(wl, params, x, want_h_all=True), wl)
+
+
 def test_benchmarked_workload_takes_the_small_path(qnn, monkeypatch):
     monkeypatch.delenv("QNN_LSTM_PATH", raising=False)
     wl = inputs.LSTM_5x500_B1

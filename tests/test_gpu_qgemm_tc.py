@@ -49,12 +49,18 @@ def test_tc_path_bit_exact(qnn, M, N, K, monkeypatch):
     cs = np.concatenate([p[2] for p in parts])
     bias = g.normal(0, 1, N).astype(np.float32)
     ref = oracle.qmatmul(ca, pa, 1, cw, pw, n_blocks=nb, bias=bias)
-    for path in ("tc", "imma"):
+    # tile widths 64 and 128 take the row epilogue (two blocks per SM) when K <= 1024, 256 the
+    # staged one; K > 1024 always drains chunks through the staged epilogue
+    for path, bn in (("tc", None), ("tc", "64"), ("tc", "128"), ("tc", "256"), ("imma", None)):
         monkeypatch.setenv("QNN_QGEMM", path)
+        if bn:
+            monkeypatch.setenv("QNN_TC_BN", bn)
+        else:
+            monkeypatch.delenv("QNN_TC_BN", raising=False)
         Y, acc = _run(qnn, ca, pa, 1, ra, cw, pw, cs, nb, bias)
         assert qnn.device_status() == qnn.QNN_OK
-        assert np.array_equal(acc.cpu().numpy(), ref["acc"]), path
-        assert np.array_equal(Y.cpu().numpy(), ref["y"]), path
+        assert np.array_equal(acc.cpu().numpy(), ref["acc"]), (path, bn)
+        assert np.array_equal(Y.cpu().numpy(), ref["y"]), (path, bn)
 
 
 @pytest.mark.parametrize("K", [1024, 1025, 2048])
