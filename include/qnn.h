@@ -205,6 +205,12 @@ qnn_status qnn_profile_read(int capacity, const char **names, double *total_ms, 
  * Register-only loops on every SM; synchronous; the best of three timed runs. */
 qnn_status qnn_measure_peak(int kind, double *tops);
 
+/* Diagnostic (no counterpart in the paper): out[i] = in[i] rounded to the nearest fp32 value, ties
+ * to even, by the conversion the recovery of eq. (3) uses on the device for the exact int64 sums
+ * S of eq. (1). in [n] int64 and out [n] float are device buffers owned by the caller; errors:
+ * QNN_ERR_INVALID_ARG for n < 0 or null/host pointers with n > 0. Asynchronous on `stream`. */
+qnn_status qnn_selftest_s64_to_f32(const int64_t *in, float *out, int64_t n, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -6,6 +6,9 @@
 //
 // Every warp runs eight independent accumulator chains from registers (no memory traffic in the
 // loop); the result is written once so the work cannot be removed by the compiler.
+#include <algorithm>
+
+#include "qnn_device.cuh"
 #include "qnn_host.h"
 
 namespace qnn {
@@ -84,5 +87,24 @@ extern "C" qnn_status qnn_measure_peak(int kind, double *tops) {
     cudaEventDestroy(e1);
     cudaFree(sink);
     *tops = best;
+    return QNN_OK;
+}
+
+namespace qnn {
+namespace {
+__global__ void s64_to_f32_kernel(const int64_t *__restrict__ in, float *__restrict__ out, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        out[i] = s64_to_f32_rn(in[i]);
+}
+}  // namespace
+}  // namespace qnn
+
+extern "C" qnn_status qnn_selftest_s64_to_f32(const int64_t *in, float *out, int64_t n, void *stream) {
+    if (n < 0) return QNN_ERR_INVALID_ARG;
+    if (n == 0) return QNN_OK;
+    if (!in || !out || !qnn::is_device_ptr(in) || !qnn::is_device_ptr(out)) return QNN_ERR_INVALID_ARG;
+    const unsigned blocks = (unsigned)std::min<int64_t>((n + 255) / 256, 4096);
+    qnn::s64_to_f32_kernel<<<blocks, 256, 0, qnn::as_stream(stream)>>>(in, out, n);
+    QNN_CUDA_TRY(cudaGetLastError());
     return QNN_OK;
 }

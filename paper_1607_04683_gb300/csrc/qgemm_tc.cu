@@ -39,12 +39,17 @@ constexpr unsigned long long TC_WAIT_NS = 2000000000ull;
 
 // kEpiLinear: recovered product, any K (chunked drains), outputs staged through shared memory.
 // kEpiRow: recovered product for K <= 1024, one output row per lane, two blocks per SM.
-// kEpiLstm: the LSTM cell update on gate-interleaved columns, K <= 1024, two blocks per SM.
-enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2 };
+// kEpiLstm: the LSTM cell update on gate-interleaved columns, K <= 1024; kEpiLstmEarly the same
+// with the accumulator-independent loads issued before the accumulator wait (a block with a single
+// tile has no earlier epilogue to overlap them with).
+enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiLstmEarly = 3 };
 
 struct ColConst {  // per-output-column constants of kEpiRow, staged in shared memory per tile
     int cs, zw;
     float Qw, bias;
+};
+struct ColUnit {  // and the weight unit of each column (-1 past N)
+    int unit;
 };
 
 // Per tile width BN (rows of W per tile) and epilogue: warps (TMA producer, MMA issuer, then the
@@ -64,7 +69,7 @@ struct Tile {
     static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : 96;
     static constexpr int EPI_BYTES = EPI == kEpiLinear ? (8 * 32 * 33 + 8 * 96) * 4
-                                     : EPI == kEpiRow  ? 2 * BN * (int)sizeof(ColConst)
+                                     : EPI == kEpiRow  ? 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit))
                                                        : 0;
     static constexpr uint32_t IDESC =
         (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TBM >> 4) << 24);
@@ -411,6 +416,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         // (ragged edges element by element). The column constants of the tile are staged in shared
         // memory (double-buffered by tile parity; one named barrier of the epilogue warps per tile).
         ColConst *scol = reinterpret_cast<ColConst *>(smem + STAGES * TL::STAGE_BYTES);
+        ColUnit *sunit = reinterpret_cast<ColUnit *>(scol + 2 * BN);
         const int q = warp & 3;
         const int part = (warp - 2) >> 2;
         const int ew = warp - 2;
@@ -423,17 +429,21 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
             const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * BN;
             ColConst *cc = scol + (gc & 1) * BN;
+            ColUnit *cu = sunit + (gc & 1) * BN;
             for (int c = ew * 32 + lane; c < BN; c += 32 * TL::EPI_WARPS) {
                 const int64_t n = n0 + c;
                 ColConst v{0, 0, 1.0f, 0.0f};
+                int unit = -1;
                 if (n < args.N) {
-                    const qnn_qparams qw = args.pw[n / args.rows_per_block];
+                    unit = (int)(n / args.rows_per_block);
+                    const qnn_qparams qw = args.pw[unit];
                     v.cs = args.csW[n];
                     v.zw = qw.z;
                     v.Qw = qw.Q;
                     v.bias = args.bias ? args.bias[n] : 0.0f;
                 }
                 cc[c] = v;
+                cu[c].unit = unit;
             }
             asm volatile("bar.sync 1, %0;" ::"n"(32 * TL::EPI_WARPS) : "memory");
             const int64_t m = m0 + 32 * q + lane;
@@ -446,7 +456,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 Qa = qa.Q;
                 ra = args.rsA[m];
             }
-            const long long za128 = 128 + za;
+            const int za128 = 128 + za;
             const int buf = (int)(gc & 1);
             if (!failed && *reinterpret_cast<volatile int *>(&s_abort)) failed = true;
             if (!failed) {
@@ -462,7 +472,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 const int64_t nb = n0 + c0;
                 if (!mv || nb >= args.N) continue;
                 // one weight unit across the 16 columns (the usual case): row terms hoisted
-                const bool one_unit = (nb / args.rows_per_block) == ((nb + 15) / args.rows_per_block);
+                const bool one_unit = cu[c0].unit == cu[c0 + 15].unit;  // -1 past N: ragged blocks take the general way
                 long long rt = 0;
                 float den = 0.0f;
                 if (one_unit) {
@@ -479,18 +489,18 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     for (int e = 0; e < 4; ++e) {
                         const int i = 4 * v4 + e;
                         const ColConst v = cc[c0 + i];
-                        const int P = __float2int_rn(__uint_as_float(r[i]));
+                        const int P = f32_integer_to_s32(__uint_as_float(r[i]));
                         long long S;
                         float dn;
                         if (one_unit) {
-                            S = (long long)P + rt + za128 * v.cs;
+                            S = (long long)P + rt + (long long)za128 * v.cs;
                             dn = den;
                         } else {
-                            S = (long long)P + (long long)(128 + v.zw) * ra + za128 * v.cs +
+                            S = (long long)P + (long long)(128 + v.zw) * ra + (long long)za128 * v.cs +
                                 (long long)K * ((long long)za * v.zw - 16384);
                             dn = __fmul_rn(Qa, v.Qw);
                         }
-                        y[e] = __fdiv_rn(__ll2float_rn(S), dn);
+                        y[e] = __fdiv_rn(s64_to_f32_rn(S), dn);
                         if (args.bias) y[e] = __fadd_rn(y[e], v.bias);
                         if (args.acc_out && nb + i < args.N)
                             args.acc_out[m * args.N + nb + i] = P + 128 * (ra + v.cs) - 16384 * K;  // raw code product
@@ -543,8 +553,18 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 rt[g] = (long long)(128 + qw.z) * rs + (long long)K * ((long long)za * qw.z - 16384);
                 den[g] = __fmul_rn(Qa, qw.Q);
             }
-            const long long za128 = 128 + za;
+            const int za128 = 128 + za;
             const int buf = (int)(gc & 1);
+            // this warp's first slice: the input products and cell state do not depend on the
+            // accumulator, so they may be loaded before waiting for it
+            const int s0 = EPI == kEpiLstmEarly ? eh : -1;
+            float4 px0[4], c0v = make_float4(0.f, 0.f, 0.f, 0.f);
+            const int j00 = (int)(n0 / 4) + (eh >> 1) * 8 + (eh & 1) * 4;
+            if (EPI == kEpiLstmEarly && eh < BN / 16 && bv && j00 < H) {
+#pragma unroll
+                for (int g = 0; g < 4; ++g) px0[g] = *reinterpret_cast<const float4 *>(E.px + b * E.px_ld + j00 + (int64_t)g * H);
+                c0v = *reinterpret_cast<const float4 *>(E.c + b * (int64_t)H + j00);
+            }
             ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -563,18 +583,18 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     float pre[4][4];
 #pragma unroll
                     for (int g = 0; g < 4; ++g) {
-                        const float4 v = *reinterpret_cast<const float4 *>(pxr + (int64_t)g * H);
+                        const float4 v = s == s0 ? px0[g] : *reinterpret_cast<const float4 *>(pxr + (int64_t)g * H);
                         const int4 cs = *reinterpret_cast<const int4 *>(args.csW + g * H + j0);
                         const int csv[4] = {cs.x, cs.y, cs.z, cs.w};
                         const float pv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
                         for (int jj = 0; jj < 4; ++jj) {
-                            const long long S =
-                                (long long)__float2int_rn(__uint_as_float(r[g][jj])) + rt[g] + za128 * csv[jj];
-                            pre[g][jj] = __fadd_rn(pv[jj], __fdiv_rn(__ll2float_rn(S), den[g]));
+                            const long long S = (long long)f32_integer_to_s32(__uint_as_float(r[g][jj])) + rt[g] +
+                                                (long long)za128 * csv[jj];
+                            pre[g][jj] = __fadd_rn(pv[jj], __fdiv_rn(s64_to_f32_rn(S), den[g]));
                         }
                     }
-                    float4 c4 = *reinterpret_cast<const float4 *>(cr);
+                    const float4 c4 = s == s0 ? c0v : *reinterpret_cast<const float4 *>(cr);
                     float cv[4] = {c4.x, c4.y, c4.z, c4.w}, mv[4];
 #pragma unroll
                     for (int jj = 0; jj < 4; ++jj) lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
@@ -720,6 +740,15 @@ qnn_status dispatch_linear(const TcOperands &op, const TcArgs &a, cudaStream_t s
 }
 
 qnn_status dispatch_lstm(const TcOperands &op, const TcArgs &a, cudaStream_t st) {
+    const int64_t tiles = ((a.M + TBM - 1) / TBM) * ((a.N + op.bn - 1) / op.bn);
+    if (tiles <= sm_count()) {
+        switch (op.bn) {
+            case 32: return launch_tc<32, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
+            case 64: return launch_tc<64, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
+            case 128: return launch_tc<128, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
+            default: return QNN_ERR_INVALID_ARG;
+        }
+    }
     switch (op.bn) {
         case 32: return launch_tc<32, kEpiLstm>(op, a, "lstm_gates_tc", st);
         case 64: return launch_tc<64, kEpiLstm>(op, a, "lstm_gates_tc", st);

@@ -59,9 +59,40 @@ __device__ __forceinline__ uint32_t quant_code(float v, float Q, int z) {
     return (uint32_t)c;
 }
 
+// (float)S rounded to nearest, ties to even, without the 64-bit conversion instruction (which runs
+// on this part's narrow fp64 pipe). |S| < 2^31 converts from 32 bits; wider values are rounded to a
+// 24-bit significand by integer arithmetic: the bits below it decide the rounding (above half:
+// up; exactly half: to the even significand).
+// (float)S rounded to nearest, ties to even, without the 64-bit conversion instruction (which runs
+// on this part's narrow fp64 pipe). |S| < 2^31 converts from 32 bits; wider values (rare: large
+// offsets z) are rounded to a 24-bit significand by integer arithmetic out of line: the bits below
+// the significand decide (above half: up; exactly half: to the even significand).
+static __device__ __noinline__ float s64_to_f32_rn_wide(long long S) {
+    const unsigned long long u = S < 0 ? 0ULL - (unsigned long long)S : (unsigned long long)S;
+    const int top = 63 - __clzll((long long)u);  // position of the leading one, 31..63
+    const int sh = top - 23;                     // bits below the significand, >= 8
+    unsigned long long m = u >> sh;
+    const unsigned long long rem = u & ((1ULL << sh) - 1), half = 1ULL << (sh - 1);
+    m += (rem > half || (rem == half && (m & 1ULL))) ? 1ULL : 0ULL;
+    int e = top + 127;
+    if (m >> 24) {  // rounding carried into a new leading bit
+        m >>= 1;
+        ++e;
+    }
+    return __uint_as_float(((unsigned)e << 23) | ((unsigned)m & 0x7FFFFFu) | (S < 0 ? 0x80000000u : 0u));
+}
+__device__ __forceinline__ float s64_to_f32_rn(long long S) {
+    const int lo = (int)S;
+    if ((long long)lo == S) return __int2float_rn(lo);
+    return s64_to_f32_rn_wide(S);
+}
+
+// An integer-valued float (an exact tensor-core sum) as int.
+__device__ __forceinline__ int f32_integer_to_s32(float v) { return __float2int_rn(v); }
+
 // Eq. (1) recovery of the exact offset-applied product S: S / (Qa Qw), each op rounded once.
 __device__ __forceinline__ float recover_product(long long S, float Qa, float Qw) {
-    return __fdiv_rn(__ll2float_rn(S), __fmul_rn(Qa, Qw));
+    return __fdiv_rn(s64_to_f32_rn(S), __fmul_rn(Qa, Qw));
 }
 
 // S = acc + zw*rsA + za*csW + K*za*zw: eq. (1)'s sum of (a' + za)(w' + zw) expanded so that the
@@ -73,12 +104,14 @@ __device__ __forceinline__ long long offset_product(int acc, int za, int zw, int
 // Pinned fp32 exponential: Cody-Waite reduction x = n ln2 + r (n = round(x log2 e), ln 2 split
 // into a 16-significant-bit head and its remainder), e^r by its degree-7 Taylor polynomial in
 // Horner form with fused multiply-adds, times 2^n assembled from exponent bits. x is clamped to
-// [-87, 88] so every result is a finite normal number.
+// [-87, 88] so every result is a finite normal number. n is rounded half-to-even by adding
+// 1.5 * 2^23 (|x log2 e| <= 127), which leaves n in the low significand bits.
 __device__ __forceinline__ float pexp(float x) {
     x = x < -87.0f ? -87.0f : x;
     x = x > 88.0f ? 88.0f : x;
-    float nf = rintf(__fmul_rn(x, 1.44269504088896341f));
-    int n = (int)nf;
+    const float t = __fadd_rn(__fmul_rn(x, 1.44269504088896341f), 12582912.0f);
+    const int n = __float_as_int(t) - 0x4B400000;
+    const float nf = __fsub_rn(t, 12582912.0f);
     float r = __fmaf_rn(-nf, 0.693145751953125f, x);
     r = __fmaf_rn(-nf, 1.428606820309417232e-06f, r);
     float p = 1.984126984126984127e-04f;

@@ -32,7 +32,8 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 # Every symbol the header declares (checked by the CPU test that loads the library).
 EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmul", "qnn_lstm_param_count",
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
-           "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static")
+           "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static",
+           "qnn_selftest_s64_to_f32")
 
 
 class QnnError(RuntimeError):
@@ -82,6 +83,8 @@ def lib():
         L.qnn_profile_read.restype = i32
         L.qnn_measure_peak.argtypes = [i32, C.POINTER(C.c_double)]
         L.qnn_measure_peak.restype = i32
+        L.qnn_selftest_s64_to_f32.argtypes = [P, P, i64, P]
+        L.qnn_selftest_s64_to_f32.restype = i32
         L.qnn_quantize_matrix_static.argtypes = [P, i64, i64, i64, P, i64, P, P, P, P]
         L.qnn_quantize_matrix_static.restype = i32
         _lib = L
@@ -97,6 +100,16 @@ def measure_peak(kind: int) -> float:
     v = C.c_double(0.0)
     _check(lib().qnn_measure_peak(kind, C.byref(v)), "qnn_measure_peak")
     return v.value
+
+
+def selftest_s64_to_f32(values):
+    """The device's int64 -> fp32 round-to-nearest conversion of the recovery, on a torch int64
+    CUDA tensor; returns a float32 tensor (diagnostic)."""
+    import torch
+    out = torch.empty(values.shape, dtype=torch.float32, device=values.device)
+    _check(lib().qnn_selftest_s64_to_f32(values.data_ptr(), out.data_ptr(), values.numel(),
+                                         torch.cuda.current_stream().cuda_stream), "qnn_selftest_s64_to_f32")
+    return out
 
 
 def profile_read() -> dict:

@@ -360,7 +360,7 @@ def test_small_and_layerwise_paths_agree(qnn, cfg, monkeypatch):
 TC_CASES = [dict(L=1, I=40, H=128, B=5, T=6), dict(L=2, I=40, H=100, C=37, B=130, T=4),
             dict(L=2, I=24, H=256, P=96, C=11, B=33, T=5), dict(L=1, I=40, H=500, B=256, T=3, w=0.08, mu=0.5),
             dict(L=1, I=8, H=1024, B=64, T=2, w=0.05), dict(L=2, I=80, H=1100, P=64, C=20, B=40, T=3, w=0.05),
-            dict(L=3, I=5, H=8, B=3, T=4, mu=0.5)]
+            dict(L=3, I=5, H=8, B=3, T=4, mu=0.5), dict(L=1, I=40, H=800, B=300, T=2, w=0.05)]
 
 
 @pytest.mark.parametrize("bn", ["32", "64", "128"])

@@ -77,3 +77,48 @@ def test_tc_extreme_codes_at_the_exactness_limit(qnn, K, a_code, w_code, monkeyp
     cs = cw.astype(np.int64).sum(1).astype(np.int32)
     Y, acc = _run(qnn, ca, p, 0, ra, cw, p, cs)
     assert np.all(acc.cpu().numpy() == a_code * w_code * K)
+
+
+@pytest.mark.parametrize("K", [64, 1000, 3000])
+def test_tc_large_offsets_bit_exact(qnn, K, monkeypatch):
+    """Rows with a narrow range far from zero have large offsets z (eq. 2), so the offset-applied
+    sums S of eq. (1) reach far beyond 2^22 and the recovery converts them the wide way."""
+    monkeypatch.delenv("QNN_TC_BN", raising=False)
+    g = np.random.Generator(np.random.PCG64(K))
+    M, N = 300, 200
+    A = (1000.0 + g.uniform(0.0, 0.5, (M, K))).astype(np.float32)
+    A[::7] = g.normal(0, 1, (A[::7].shape)).astype(np.float32)  # and some ordinary rows
+    W = g.uniform(-0.1, 0.1, (N, K)).astype(np.float32)
+    ca, pa, ra = oracle.quantize(A, oracle.PER_ROW)
+    cw, pw, cs = oracle.quantize(W, oracle.PER_MATRIX)
+    assert np.abs(pa["z"]).max() > 1 << 18
+    ref = oracle.qmatmul(ca, pa, 1, cw, pw)
+    for path in ("tc", "imma"):
+        monkeypatch.setenv("QNN_QGEMM", path)
+        Y, acc = _run(qnn, ca, pa, 1, ra, cw, pw, cs)
+        assert qnn.device_status() == qnn.QNN_OK
+        assert np.array_equal(acc.cpu().numpy(), ref["acc"]), path
+        assert np.array_equal(Y.cpu().numpy(), ref["y"]), path
+
+
+def test_s64_to_f32_rounds_to_nearest_even(qnn):
+    """The recovery's int64 -> fp32 conversion against the host's IEEE conversion: every magnitude,
+    exact halfway cases (ties to even) and their neighbours, and the carry into a new leading bit."""
+    g = np.random.Generator(np.random.PCG64(11))
+    parts = [g.integers(-(1 << 62), 1 << 62, 200000, dtype=np.int64)]
+    for top in range(20, 63):  # random values with a given leading-bit position
+        parts.append(g.integers(1 << top, 1 << (top + 1), 2000, dtype=np.int64))
+    ties = []
+    for sh in range(1, 40):
+        m = g.integers(1 << 23, 1 << 24, 200, dtype=np.int64)
+        base = (m << sh) + (1 << (sh - 1))  # exactly halfway between two fp32 values
+        ties += [base, base - 1, base + 1]
+    parts += ties
+    parts.append(np.array([(1 << 24) - 1, 1 << 24, (1 << 24) + 1, (1 << 31) - 1, 1 << 31, -(1 << 31), -(1 << 31) - 1,
+                           (1 << 63) - 1, -(1 << 63), ((1 << 24) - 1) << 39, (((1 << 24) - 1) << 39) + (1 << 38)],
+                          dtype=np.int64))
+    v = np.concatenate(parts)
+    v = np.concatenate([v, -v[v != -(1 << 63)]])
+    got = qnn.selftest_s64_to_f32(torch.from_numpy(v).cuda()).cpu().numpy()
+    want = v.astype(np.float32)
+    assert np.array_equal(got.view(np.int32), want.view(np.int32))
