@@ -92,12 +92,27 @@ def small_bytes_per_launch(wl: inputs.LstmWorkload) -> int:
     return w + wl.batch * wl.frames * (wl.input_dim + out) * 4
 
 
-def traffic_record(kernel: str, workload: str, source: str):
-    """Per-launch DRAM bytes from the committed ncu summary, if taken on the current source."""
+def source_sha(sources) -> str:
+    """Hash of the kernel's source files (the .cu and the headers its arithmetic comes from)."""
+    h = hashlib.sha256()
+    for name in sources:
+        h.update(open(os.path.join(ROOT, "paper_1607_04683_gb300", "csrc", name), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def gates_bytes_per_launch(wl) -> float:
+    """Algorithmic DRAM bytes of one tensor-core recurrent step: the step's input products px
+    (B x 4H fp32), the cell state read and written (B x H fp32 each way), the cell outputs written
+    (B x H fp32), the recurrent input codes (B x R bytes) and the gate weight codes (4H x R bytes)."""
+    B, H, R = wl.batch, wl.hidden, wl.R
+    return float(B * 4 * H * 4 + 2 * B * H * 4 + B * H * 4 + B * R + 4 * H * R)
+
+
+def traffic_record(kernel: str, workload: str, sources):
+    """Per-launch DRAM bytes from the committed ncu summary, if taken on the current sources."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
-    src = os.path.join(ROOT, "paper_1607_04683_gb300", "csrc", source)
     try:
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        sha = source_sha(sources)
         for line in open(path):
             f = line.split()
             if len(f) >= 4 and not line.startswith("#") and f[0] == kernel and f[1] == workload and f[3] == sha:
@@ -340,7 +355,7 @@ def run_ours(args, wl, rank, world, local):
         ach = alg / avg_s / 1e9
         roofline = {"bound": "hbm", "kernel": kname, "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                     "frac": ach / peaks["hbm_gbs"], "peak_kind": peak_kind,
-                    "traffic": traffic_record(kname, wl.name, "lstm.cu"), "alg_bytes_per_launch": alg,
+                    "traffic": traffic_record(kname, wl.name, ["lstm.cu", "qnn_device.cuh"]), "alg_bytes_per_launch": alg,
                     "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
     elif kname == "lstm_small":
         # the whole stack in one launch; its arithmetic is the integer products of every layer and
@@ -350,9 +365,21 @@ def run_ours(args, wl, rank, world, local):
         dp4a_peak = qnn.measure_peak(1)
         roofline = {"bound": "alu", "kernel": kname, "achieved": ach, "peak": dp4a_peak, "unit": "TOP/s",
                     "frac": ach / dp4a_peak, "peak_kind": "measured (qnn_measure_peak dp4a)",
-                    "traffic": traffic_record(kname, wl.name, "lstm_small.cu"), "alg_ops_per_launch": ops,
+                    "traffic": traffic_record(kname, wl.name, ["lstm_small.cu", "qnn_device.cuh"]), "alg_ops_per_launch": ops,
                     "alg_bytes_per_launch": small_bytes_per_launch(wl), "hbm_frac":
                         small_bytes_per_launch(wl) / avg_s / 1e9 / peaks["hbm_gbs"],
+                    "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
+    elif kname == "lstm_gates_tc":
+        # one recurrent step of one layer: the tcgen05 gate product with the LSTM cell in its
+        # epilogue; reported against HBM with the step's algorithmic bytes, plus its tensor rate
+        alg = gates_bytes_per_launch(wl)
+        ach = alg / avg_s / 1e9
+        flops = 2.0 * wl.batch * 4 * wl.hidden * wl.R
+        roofline = {"bound": "hbm", "kernel": kname, "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                    "frac": ach / peaks["hbm_gbs"], "peak_kind": peak_kind,
+                    "traffic": traffic_record(kname, wl.name, ["qgemm_tc.cu", "qnn_device.cuh"]),
+                    "alg_bytes_per_launch": alg, "tensor_tflops": flops / avg_s / 1e12,
+                    "tensor_frac": flops / avg_s / 1e12 / peaks["bf16_tflops"],
                     "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
     line = {
         "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": world, "steps": args.steps,

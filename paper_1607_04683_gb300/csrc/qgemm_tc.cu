@@ -65,12 +65,12 @@ struct Tile {
     static constexpr int THREADS = 32 * (2 + EPI_WARPS);
     static constexpr int B_BYTES = BN * TBK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = EPI == kEpiLinear ? (BN == 256 ? 3 : (BN == 128 ? 4 : 6)) : (BN == 128 ? 4 : 6);
+    static constexpr int STAGES = EPI == kEpiLinear ? (BN == 256 ? 4 : 6) : (BN == 128 ? 4 : 6);
     static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : 96;
-    static constexpr int EPI_BYTES = EPI == kEpiLinear ? (8 * 32 * 33 + 8 * 96) * 4
-                                     : EPI == kEpiRow  ? 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit))
-                                                       : 0;
+    static constexpr int EPI_BYTES = EPI == kEpiLstm || EPI == kEpiLstmEarly
+                                         ? 0
+                                         : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
     static constexpr uint32_t IDESC =
         (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TBM >> 4) << 24);
     static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + EPI_BYTES + 256;
@@ -194,6 +194,19 @@ __device__ __forceinline__ void tmem_ld4_nowait(uint32_t taddr, uint32_t (&r)[4]
                  : "r"(taddr));
 }
 
+// Tile order: groups of kGroupM row tiles, columns outer within a group, so that the tiles one
+// wave of blocks works on span a compact block of A and W (both stay in L2 across the wave).
+constexpr int kGroupM = 16;
+__device__ __forceinline__ void tile_origin(int64_t tile, int64_t tiles_m, int tiles_n, int bn, int64_t &m0,
+                                            int64_t &n0) {
+    const int64_t per_group = (int64_t)kGroupM * tiles_n;
+    const int64_t first = (tile / per_group) * kGroupM;
+    const int64_t rows = tiles_m - first < kGroupM ? tiles_m - first : kGroupM;
+    const int64_t local = tile % per_group;
+    m0 = (first + local % rows) * TBM;
+    n0 = (local / rows) * bn;
+}
+
 // Persistent tile loop. Warp 0: TMA producer; warp 1: tensor-memory owner and MMA issuer; warps
 // 2.. : epilogue. EPI = kEpiLinear / kEpiRow write the recovered product (plus bias) and
 // optionally the raw int32 accumulator; EPI = kEpiLstm treats the columns as gate-interleaved LSTM
@@ -208,8 +221,6 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // 1024-byte alignment for the swizzled tiles
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    int *stage_out = reinterpret_cast<int *>(smem + STAGES * TL::STAGE_BYTES);     // [8 warps][32][33] (linear)
-    int *row_c = stage_out + 8 * 32 * 33;                                          // [8 warps][3][32] (linear)
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + STAGES * TL::STAGE_BYTES + TL::EPI_BYTES);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 4);
     const uint32_t full0 = su32(bars), empty0 = su32(bars + STAGES), chunk0 = su32(bars + 2 * STAGES),
@@ -219,7 +230,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     const int kpc = KCHUNK / TBK;  // k-blocks per chunk (16)
     const int nchunks = (KB + kpc - 1) / kpc;
     const int tiles_n = (int)((args.N + BN - 1) / BN);
-    const int64_t tiles = (int64_t)((args.M + TBM - 1) / TBM) * tiles_n;
+    const int64_t tiles_m = (args.M + TBM - 1) / TBM;
+    const int64_t tiles = tiles_m * tiles_n;
     __shared__ int s_abort;
 
     if (threadIdx.x == 0) {
@@ -250,15 +262,16 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     grid_dependency_wait();
     grid_dependents_launch();
 
-    // Persistent: block b takes tiles b, b + grid, ... (row-tile major, so neighbouring blocks share
-    // the same rows of A through L2). The k-block and chunk counters run across tiles, so the two
-    // accumulator buffers alternate and one tile's epilogue overlaps the next tile's MMAs.
+    // Persistent: block b takes tiles b, b + grid, ... in grouped order (tile_origin). The k-block
+    // and chunk counters run across tiles, so the two accumulator buffers alternate and one tile's
+    // epilogue overlaps the next tile's MMAs.
     if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (lane == 0) {
             int64_t g = 0;  // k-blocks issued by this block
             for (int64_t tile = blockIdx.x; tile < tiles && !s_abort; tile += gridDim.x) {
-                const int m0 = (int)(tile / tiles_n) * TBM, n0 = (int)(tile % tiles_n) * BN;
+                int64_t m0, n0;
+                tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
                 for (int kb = 0; kb < KB; ++kb, ++g) {
                     const int s = (int)(g % STAGES);
                     if (g >= STAGES && !mb_wait(empty0 + 8 * s, (unsigned)((g / STAGES) - 1) & 1, args.status)) {
@@ -309,104 +322,103 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             }
         }
     } else if constexpr (EPI == kEpiLinear) {
-        // ---------------- epilogue (warps 2..9): recovered product ----------------
+        // ---------------- epilogue (warps 2..9): recovered product, any K ----------------
+        // Each lane owns one output row and one column half of the tile. Every K chunk is drained
+        // from tensor memory into int32 running sums in registers; after the last chunk the sums
+        // are recovered (eq. 1 offsets, eq. 3) and stored as 16-byte vectors straight from
+        // registers (ragged or unaligned outputs element by element). Column constants are staged
+        // in shared memory per tile (double-buffered; one named barrier of the epilogue warps).
         constexpr int NJ = BN / 64;             // 32-column blocks per warp
+        ColConst *scol = reinterpret_cast<ColConst *>(smem + STAGES * TL::STAGE_BYTES);
+        ColUnit *sunit = reinterpret_cast<ColUnit *>(scol + 2 * BN);
         const int q = warp & 3;                 // tensor-memory lane quarter this warp may read
         const int half = (warp - 2) >> 2;       // column half: [0, BN/2) or [BN/2, BN)
         const int ew = warp - 2;
-        int *stg = stage_out + ew * 32 * 33;
-        int *rz = row_c + ew * 96, *rr = rz + 32;
-        float *rq = reinterpret_cast<float *>(rz + 64);
         const int K = args.K;
-        int64_t gc = 0;
-        bool ok = true;
-        for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * BN;
-            {  // this lane's row constants, shared with the warp for the transposed stores
-                const int64_t m = m0 + 32 * q + lane;
-                const bool mv = m < args.M;
-                const qnn_qparams qa = args.pa[args.a_per_row ? (mv ? m : 0) : 0];
-                rz[lane] = qa.z;
-                rq[lane] = qa.Q;
-                rr[lane] = mv ? args.rsA[m] : 0;
+        const bool vec = args.Y && (args.ldy % 4 == 0) && ((reinterpret_cast<uintptr_t>(args.Y) & 15) == 0);
+        int64_t gc = 0, it = 0;
+        bool failed = false;
+        for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
+            int64_t m0, n0;
+            tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
+            ColConst *cc = scol + (it & 1) * BN;
+            ColUnit *cu = sunit + (it & 1) * BN;
+            for (int c = ew * 32 + lane; c < BN; c += 32 * TL::EPI_WARPS) {
+                const int64_t n = n0 + c;
+                ColConst v{0, 0, 1.0f, 0.0f};
+                int unit = -1;
+                if (n < args.N) {
+                    unit = (int)(n / args.rows_per_block);
+                    const qnn_qparams qw = args.pw[unit];
+                    v.cs = args.csW[n];
+                    v.zw = qw.z;
+                    v.Qw = qw.Q;
+                    v.bias = args.bias ? args.bias[n] : 0.0f;
+                }
+                cc[c] = v;
+                cu[c].unit = unit;
             }
-            // 32 x 32 block: P values of rows (this warp's 32 lanes) x columns c0 .. c0 + 31, written
-            // row-wise to shared memory and read back column-wise, so that each store instruction
-            // writes 32 consecutive outputs of one row.
-            auto emit = [&](int c0, const int (&P)[32]) {
+            asm volatile("bar.sync 1, %0;" ::"n"(32 * TL::EPI_WARPS) : "memory");
+            int run[NJ][32];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) stg[lane * 33 + i] = P[i];
-                __syncwarp();
-                const int64_t n = n0 + c0 + lane;
-                const bool nv = n < args.N;
-                const qnn_qparams qw = args.pw[nv ? n / args.rows_per_block : 0];
-                const int cs = nv ? args.csW[n] : 0;
-                const float bn = (nv && args.bias) ? args.bias[n] : 0.0f;
-                for (int r = 0; r < 32; ++r) {
-                    const int64_t m = m0 + 32 * q + r;
-                    if (m >= args.M) break;
-                    if (nv) {
-                        const int ra = rr[r];
-                        const int acc = stg[r * 33 + lane] + 128 * (ra + cs) - 16384 * K;  // raw code product
-                        const long long S = offset_product(acc, rz[r], qw.z, ra, cs, K);
-                        float y = recover_product(S, rq[r], qw.Q);
-                        if (args.bias) y = __fadd_rn(y, bn);
-                        if (args.Y) args.Y[m * args.ldy + n] = y;
-                        if (args.acc_out) args.acc_out[m * args.N + n] = acc;
-                    }
-                }
-                __syncwarp();
-            };
-            auto taddr_of = [&](int buf, int j) {
-                return tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + half * (BN / 2) + 32 * j);
-            };
-            __syncwarp();
-            if (nchunks == 1) {  // K <= 1024: read the accumulator and finish directly
+            for (int j = 0; j < NJ; ++j)
+#pragma unroll
+                for (int i = 0; i < 32; ++i) run[j][i] = 0;
+            for (int c = 0; c < nchunks; ++c, ++gc) {
                 const int buf = (int)(gc & 1);
-                ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
-                if (!ok) break;
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-#pragma unroll 1
-                for (int j = 0; j < NJ; ++j) {
-                    uint32_t r[32];
-                    tmem_ld32(taddr_of(buf, j), r);
-                    int P[32];
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) P[i] = __float2int_rn(__uint_as_float(r[i]));
-                    emit(half * (BN / 2) + 32 * j, P);
+                if (!failed && *reinterpret_cast<volatile int *>(&s_abort)) failed = true;
+                if (!failed) {
+                    failed = !__all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
+                    if (failed) *reinterpret_cast<volatile int *>(&s_abort) = 1;
                 }
-                // the accumulator is free again: the tile after next may use it
-                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-                __syncwarp();
-                if (lane == 0)
-                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
-                ++gc;
-            } else {  // drain every chunk into int32 running sums
-                int run[NJ][32];
-#pragma unroll
-                for (int j = 0; j < NJ; ++j)
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) run[j][i] = 0;
-                for (int c = 0; c < nchunks; ++c, ++gc) {
-                    const int buf = (int)(gc & 1);
-                    ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
-                    if (!ok) break;
-                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                if (!failed) {
 #pragma unroll
                     for (int j = 0; j < NJ; ++j) {
-                        uint32_t rr32[32];
-                        tmem_ld32(taddr_of(buf, j), rr32);
+                        uint32_t r32[32];
+                        tmem_ld32(tmem_base + ((uint32_t)(32 * q) << 16) +
+                                      (uint32_t)(buf * BN + half * (BN / 2) + 32 * j),
+                                  r32);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) run[j][i] += __float2int_rn(__uint_as_float(rr32[i]));
+                        for (int i = 0; i < 32; ++i) run[j][i] += f32_integer_to_s32(__uint_as_float(r32[i]));
                     }
-                    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-                    __syncwarp();
-                    if (lane == 0)
-                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
                 }
-                if (!ok) break;
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+            }
+            const int64_t m = m0 + 32 * q + lane;
+            if (failed || m >= args.M) continue;
+            const qnn_qparams qa = args.pa[args.a_per_row ? m : 0];
+            const int za = qa.z, ra = args.rsA[m];
+            const float Qa = qa.Q;
 #pragma unroll
-                for (int j = 0; j < NJ; ++j) emit(half * (BN / 2) + 32 * j, run[j]);
+            for (int j = 0; j < NJ; ++j) {
+                const int c0 = half * (BN / 2) + 32 * j;
+                const int64_t nb = n0 + c0;
+                if (nb >= args.N) continue;
+                const bool full = vec && nb + 32 <= args.N;
+                float *yr = args.Y ? args.Y + m * args.ldy + nb : nullptr;
+#pragma unroll
+                for (int v4 = 0; v4 < 8; ++v4) {
+                    float y[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int i = 4 * v4 + e;
+                        const ColConst v = cc[c0 + i];
+                        const int acc = run[j][i] + 128 * (ra + v.cs) - 16384 * K;  // raw code product
+                        y[e] = recover_product(offset_product(acc, za, v.zw, ra, v.cs, K), Qa, v.Qw);
+                        if (args.bias) y[e] = __fadd_rn(y[e], v.bias);
+                        if (args.acc_out && nb + i < args.N) args.acc_out[m * args.N + nb + i] = acc;
+                    }
+                    if (full) {
+                        *reinterpret_cast<float4 *>(yr + 4 * v4) = make_float4(y[0], y[1], y[2], y[3]);
+                    } else if (yr) {
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            if (nb + 4 * v4 + e < args.N) yr[4 * v4 + e] = y[e];
+                    }
+                }
             }
         }
     } else if constexpr (EPI == kEpiRow) {
@@ -427,7 +439,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         int64_t gc = 0;
         bool failed = false;
         for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
-            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * BN;
+            int64_t m0, n0;
+            tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
             ColConst *cc = scol + (gc & 1) * BN;
             ColUnit *cu = sunit + (gc & 1) * BN;
             for (int c = ew * 32 + lane; c < BN; c += 32 * TL::EPI_WARPS) {
@@ -533,7 +546,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         int64_t gc = 0;
         bool ok = true;
         for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-            const int64_t m0 = (tile / tiles_n) * TBM, n0 = (tile % tiles_n) * BN;
+            int64_t m0, n0;
+            tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
             const int64_t b = m0 + 32 * q + lane;
             const bool bv = b < args.M;
             int za = 0, rs = 0;
@@ -780,9 +794,15 @@ int tc_choose_bn(int64_t M, int64_t N, const int *cands, int n) {
 }
 
 int tc_pick_bn(int64_t M, int64_t N, int64_t kp) {
-    if (kp > KCHUNK) {  // chunked drains through the staged epilogue: widest tile
-        static const int c[] = {256, 128, 64};
-        return tc_choose_bn(M, N, c, 3);
+    if (kp > KCHUNK) {  // chunked drains: the widest tile whose tiles fill three quarters of the SMs
+        if (const char *e = std::getenv("QNN_TC_BN")) {
+            const int v = std::atoi(e);
+            if (v == 64 || v == 128 || v == 256) return v;
+        }
+        const int64_t mt = (M + TBM - 1) / TBM;
+        for (int bn : {256, 128})
+            if (4 * mt * ((N + bn - 1) / bn) >= 3 * (int64_t)sm_count()) return bn;
+        return 64;
     }
     static const int c[] = {128, 64};  // row epilogue
     return tc_choose_bn(M, N, c, 2);
