@@ -44,6 +44,10 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="standalone quantized matmul sweep instead")
     ap.add_argument("--shape", default="", help="with --sweep: one shape M,N,K only")
+    ap.add_argument("--frames", type=int, default=0,
+                    help="profiling aid: run only the first N frames of the workload (same per-launch shapes)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling aid: run only the first L layers of the workload (same per-launch shapes)")
     return ap.parse_args()
 
 
@@ -471,6 +475,15 @@ def main():
         return run_sweep(args)
     rank, world, local = dist_info()
     wl = inputs.LSTM_WORKLOADS[args.workload]
+    if args.frames or args.layers:  # a cut of the named workload (its name says so)
+        import dataclasses
+        cut = {}
+        if args.frames:
+            cut["frames"] = min(args.frames, wl.frames)
+        if args.layers:
+            cut["num_layers"] = min(args.layers, wl.num_layers)
+        wl = dataclasses.replace(wl, name=f"{wl.name}_cut_L{cut.get('num_layers', wl.num_layers)}"
+                                          f"_T{cut.get('frames', wl.frames)}", **cut)
     if world > 1 and args.impl == "ours":
         import torch
         import torch.distributed as dist
