@@ -88,6 +88,8 @@ def lib():
             L.orc_lstm_forward.argtypes = [C.POINTER(LstmDesc), P, P, i64, i64, P, P, P, P, P]
             L.orc_lstm_forward.restype = C.c_int
             L.orc_lstm_quantize_weights.argtypes = [C.POINTER(LstmDesc), P, P, P, C.POINTER(i64)]
+            L.orc_stack_frames.argtypes = [P, i64, i64, i64, C.c_int, C.c_int, P]
+            L.orc_stack_frames.restype = C.c_int
             L.orc_lstm_quantize_weights.restype = C.c_int
             _lib = L
     return _lib
@@ -226,3 +228,13 @@ def lstm_quantize_weights(d: LstmDesc, params: np.ndarray):
     nu = C.c_int64(0)
     _check(lib().orc_lstm_quantize_weights(C.byref(d), _ptr(params), _ptr(codes), _ptr(qp), C.byref(nu)))
     return codes, qp[: nu.value]
+
+
+def stack_frames(x: np.ndarray, n: int, stride: int) -> np.ndarray:
+    """Sec. 4 frontend (reading R9): x [B, T, I] -> [B, ceil(T/stride), n*I]; input t' concatenates
+    frames stride*t' .. stride*t' + n - 1, the last frame standing in past the end."""
+    x = np.ascontiguousarray(x, np.float32)
+    B, T, I = x.shape
+    out = np.empty((B, (T + stride - 1) // stride, n * I), np.float32)
+    _check(lib().orc_stack_frames(_ptr(x), B, T, I, n, stride, _ptr(out)))
+    return out

@@ -31,6 +31,9 @@
  *      one unit per row (one frame of one sequence) inside the LSTM.
  *   R7 output layer: logits = R(Q(r) Wo) + bo then softmax ("quant-all", Sec. 5); the float
  *      variant ("quant") computes the logits in fp64 and rounds them once to fp32.
+ *   R9 frame stacking (Sec. 4 frontend): network input t' is the n frames starting at frame
+ *      stride*t' (the frame and n-1 frames of right context), concatenated; T' = ceil(T/stride)
+ *      inputs; frames past the end of the sequence repeat its last frame.
  */
 #include <math.h>
 #include <stdint.h>
@@ -514,4 +517,22 @@ int orc_lstm_quantize_weights(const orc_lstm_desc *d, const float *params, uint8
     }
     if (n_units) *n_units = u;
     return st;
+}
+
+/* Sec. 4 frontend: features of n consecutive frames are stacked (the frame and n-1 frames of
+ * right context) and only every stride-th stacked frame is presented to the network.
+ * x [B][T][I] -> out [B][T'][n*I], T' = ceil(T / stride); out[b][t'][k*I + i] is frame
+ * stride*t' + k of sequence b (the last frame where that is past the end, R9). */
+int orc_stack_frames(const float *x, int64_t B, int64_t T, int64_t I, int n, int stride, float *out)
+{
+    if (B < 0 || T < 1 || I < 1 || n < 1 || stride < 1) return ORC_ERR_INVALID_ARG;
+    const int64_t Tp = (T + stride - 1) / stride;
+    for (int64_t b = 0; b < B; ++b)
+        for (int64_t tp = 0; tp < Tp; ++tp)
+            for (int k = 0; k < n; ++k) {
+                int64_t t = tp * stride + k;
+                if (t > T - 1) t = T - 1;
+                for (int64_t i = 0; i < I; ++i) out[((b * Tp + tp) * n + k) * I + i] = x[(b * T + t) * I + i];
+            }
+    return ORC_OK;
 }

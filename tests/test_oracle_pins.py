@@ -510,3 +510,46 @@ def test_golden_fixtures_unchanged():
     res = oracle.lstm_forward(oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, 0, wl.num_classes), params, x)
     assert [float(v).hex() for v in res["y"].ravel()] == g["y_hex"]
     assert [float(v).hex() for v in res["h"].ravel()] == g["h_hex"]
+
+
+# ------------------------------------------------------------------------------------------
+# Frame stacking (Sec. 4 frontend; reading R9 for the sequence end)
+# ------------------------------------------------------------------------------------------
+
+def _stack_reference(x, n, stride):
+    """The same definition by array slicing: pad the end by repeating the last frame, take n
+    shifted views, concatenate along features, keep every stride-th."""
+    B, T, I = x.shape
+    padded = np.concatenate([x, np.repeat(x[:, -1:], n - 1, axis=1)], axis=1)
+    windows = np.concatenate([padded[:, k:k + T] for k in range(n)], axis=2)
+    return windows[:, ::stride]
+
+
+def test_stack_frames_identity_and_subsampling():
+    g = np.random.Generator(np.random.PCG64(21))
+    x = g.normal(0, 1, (3, 11, 5)).astype(np.float32)
+    assert np.array_equal(oracle.stack_frames(x, 1, 1), x)
+    assert np.array_equal(oracle.stack_frames(x, 1, 3), x[:, ::3])
+
+
+@pytest.mark.parametrize("n,stride,T", [(8, 3, 300), (8, 3, 7), (8, 3, 1), (3, 2, 10), (5, 1, 4), (2, 7, 20)])
+def test_stack_frames_matches_sliced_windows(n, stride, T):
+    g = np.random.Generator(np.random.PCG64(n * 100 + stride * 10 + T))
+    x = g.normal(0, 1, (2, T, 6)).astype(np.float32)
+    got = oracle.stack_frames(x, n, stride)
+    assert got.shape == (2, -(-T // stride), n * 6)
+    assert np.array_equal(got, _stack_reference(x, n, stride))
+
+
+def test_stack_frames_paper_frontend():
+    """40-dim frames, 8 stacked (7 of right context), every third presented: 320 features per input,
+    one input per 30 ms of 10 ms frames (T = 300 frames -> 100 inputs)."""
+    x = np.arange(1 * 300 * 40, dtype=np.float32).reshape(1, 300, 40)
+    s = oracle.stack_frames(x, 8, 3)
+    assert s.shape == (1, 100, 320)
+    for t in (0, 1, 50, 97):
+        for k in range(8):
+            assert np.array_equal(s[0, t, 40 * k:40 * (k + 1)], x[0, 3 * t + k])
+    # the last input reaches past frame 299: frames 297..304 -> 297, 298, 299, 299, ...
+    last = s[0, 99].reshape(8, 40)[:, 0] / 40
+    assert list(last) == [297, 298, 299, 299, 299, 299, 299, 299]
