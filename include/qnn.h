@@ -119,12 +119,18 @@ typedef struct {
     int32_t proj;        /* P, recurrent projection units after each layer; 0 = none */
     int32_t num_classes; /* C, softmax outputs; 0 = no output layer */
     int32_t output_mode; /* qnn_output_mode; must be QNN_OUT_NONE iff num_classes == 0 */
+    int32_t stack;        /* Sec. 4 frontend: frames stacked into one network input (the frame and
+                             stack - 1 frames of right context; the paper uses 8); 0 or 1 = none.
+                             The first layer then takes I * stack features. */
+    int32_t stack_stride; /* only every stack_stride-th stacked frame is presented (the paper: 3);
+                             0 or 1 = every frame */
 } qnn_lstm_desc;
 
 typedef struct qnn_lstm_model qnn_lstm_model;
 
 /* Number of fp32 values in the packed parameter buffer. Layout, layer by layer, with
- * Ik = I for the first layer and R = (P > 0 ? P : H) otherwise, gates in the order [i, f, g, o]:
+ * Ik = I * max(stack, 1) for the first layer and R = (P > 0 ? P : H) otherwise, gates in the order
+ * [i, f, g, o]:
  *   Wx[4][H][Ik], Wh[4][H][R], b[4][H], then Wp[P][H] if P > 0;
  * after the last layer, if C > 0: Wo[C][R], bo[C]. Returns -1 on an invalid descriptor. */
 int64_t qnn_lstm_param_count(const qnn_lstm_desc *d);
@@ -145,7 +151,10 @@ qnn_status qnn_lstm_model_weights(const qnn_lstm_model *m, uint8_t *codes_host, 
 
 /*
  * qnn_lstm_forward — inference over B independent sequences of T frames.
- *   x        [B][T][I] fp32 frames.
+ *   x        [B][T][I] fp32 frames. With frame stacking (desc.stack, desc.stack_stride) the
+ *            network runs on T' = ceil(T / stride) stacked inputs, formed as qnn_stack_frames does
+ *            within this call (frames past the end of x repeat its last frame); every output
+ *            below then has T' frames instead of T.
  *   y        [B][T][C] softmax outputs if the model has an output layer, else [B][T][R] top-layer
  *            outputs.
  *   h_state  [L][B][R], c_state [L][B][H], nullable: initial state in, final state out (a
@@ -160,6 +169,19 @@ qnn_status qnn_lstm_model_weights(const qnn_lstm_model *m, uint8_t *codes_host, 
  */
 qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
                             float *c_state, float *h_all, void *stream);
+
+/*
+ * qnn_stack_frames — the frontend of Sec. 4: features of n consecutive frames are stacked (the frame
+ * and n - 1 frames of right context) and only every stride-th stacked frame is kept.
+ *   x   [B][T][I] fp32, device memory, caller-owned.
+ *   out [B][T'][n I] fp32, T' = ceil(T / stride), device memory, caller-owned: out[b][t'] is frames
+ *       stride t' .. stride t' + n - 1 of sequence b, concatenated; a frame past the end of the
+ *       sequence is replaced by its last frame (the paper does not say).
+ * QNN_ERR_INVALID_ARG for B < 0, T < 1, I < 1, n < 1, stride < 1 or non-device pointers (B > 0).
+ * Asynchronous on `stream`.
+ */
+qnn_status qnn_stack_frames(const float *x, int64_t B, int64_t T, int64_t I, int32_t n, int32_t stride, float *out,
+                            void *stream);
 
 /*
  * qnn_quantize_matrix_static — qnn_quantize with QNN_PER_MATRIX, allocating nothing.

@@ -503,8 +503,12 @@ using namespace qnn;
 
 namespace {
 
+// Features per network input: the frame features times the frames stacked (Sec. 4 frontend).
+int64_t network_input_dim(const qnn_lstm_desc *d) { return (int64_t)d->input_dim * (d->stack > 1 ? d->stack : 1); }
+
 bool valid_desc(const qnn_lstm_desc *d) {
     if (!d || d->num_layers < 1 || d->input_dim < 1 || d->hidden < 1 || d->proj < 0 || d->num_classes < 0) return false;
+    if (d->stack < 0 || d->stack_stride < 0) return false;
     if ((d->num_classes == 0) != (d->output_mode == QNN_OUT_NONE)) return false;
     if (d->output_mode < QNN_OUT_NONE || d->output_mode > QNN_OUT_FLOAT) return false;
     return true;
@@ -540,7 +544,7 @@ extern "C" int64_t qnn_lstm_param_count(const qnn_lstm_desc *d) {
     const int64_t H = d->hidden, P = d->proj, R = P > 0 ? P : H;
     int64_t n = 0;
     for (int l = 0; l < d->num_layers; ++l) {
-        const int64_t Ik = l == 0 ? d->input_dim : R;
+        const int64_t Ik = l == 0 ? network_input_dim(d) : R;
         n += 4 * H * Ik + 4 * H * R + 4 * H + (P > 0 ? P * H : 0);
     }
     if (d->num_classes > 0) n += (int64_t)d->num_classes * R + d->num_classes;
@@ -557,6 +561,7 @@ extern "C" void qnn_lstm_model_destroy(qnn_lstm_model *m) {
     cudaFree(m->ws);
     cudaFree(m->sws);
     cudaFree(m->tcw);
+    cudaFree(m->fws);
     cudaSetDevice(prev);
     delete m;
 }
@@ -564,7 +569,7 @@ extern "C" void qnn_lstm_model_destroy(qnn_lstm_model *m) {
 extern "C" qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float *params, qnn_lstm_model **out) {
     if (!out || !params || !valid_desc(d)) return QNN_ERR_INVALID_ARG;
     *out = nullptr;
-    const int64_t L = d->num_layers, I = d->input_dim, H = d->hidden, P = d->proj, C = d->num_classes;
+    const int64_t L = d->num_layers, I = network_input_dim(d), H = d->hidden, P = d->proj, C = d->num_classes;
     const int64_t R = P > 0 ? P : H;
     if (I > QNN_K_MAX || H > QNN_K_MAX || R > QNN_K_MAX) return QNN_ERR_K_TOO_LARGE;
     const int64_t n_params = qnn_lstm_param_count(d);
@@ -572,6 +577,9 @@ extern "C" qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float 
     auto *m = new qnn_lstm_model();
     m->d = *d;
     m->L = L, m->I = I, m->H = H, m->P = P, m->C = C, m->R = R;
+    m->frame_dim = d->input_dim;
+    m->stack = d->stack > 1 ? d->stack : 1;
+    m->stack_stride = d->stack_stride > 1 ? d->stack_stride : 1;
     cudaGetDevice(&m->device);
     m->layers.resize(L);
 
@@ -750,12 +758,48 @@ FwdPlan plan_recurrent(const qnn_lstm_model *m, int64_t B) {
 
 }  // namespace
 
+namespace {
+
+// Frame stacking (Sec. 4 frontend) ahead of the first layer: x [B][T][frame_dim] (host or device)
+// -> the model's frontend workspace [B][T'][I]; *xs and *Tn receive the network input and T'.
+qnn_status stack_input(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, cudaStream_t st, const float **xs,
+                       int64_t *Tn) {
+    const int64_t Tp = (T + m->stack_stride - 1) / m->stack_stride;
+    const bool x_dev = is_device_ptr(x);
+    const size_t raw = x_dev ? 0 : (size_t)round_up(B * T * m->frame_dim * 4, 256);
+    const size_t need = raw + (size_t)(B * Tp * m->I * 4);
+    if (need > m->fws_bytes) {
+        if (m->fws) {
+            QNN_CUDA_TRY(cudaStreamSynchronize(st));
+            QNN_CUDA_TRY(cudaFree(m->fws));
+            m->fws = nullptr;
+            m->fws_bytes = 0;
+        }
+        QNN_CUDA_TRY(cudaMalloc(&m->fws, need));
+        m->fws_bytes = need;
+    }
+    char *w = reinterpret_cast<char *>(m->fws);
+    const float *src = x;
+    if (!x_dev) {
+        QNN_CUDA_TRY(cudaMemcpyAsync(w, x, B * T * m->frame_dim * 4, cudaMemcpyHostToDevice, st));
+        src = reinterpret_cast<const float *>(w);
+    }
+    float *out = reinterpret_cast<float *>(w + raw);
+    QNN_TRY(launch_stack_frames(src, B, T, m->frame_dim, (int)m->stack, (int)m->stack_stride, out, st));
+    *xs = out;
+    *Tn = Tp;
+    return QNN_OK;
+}
+
+}  // namespace
+
 extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y,
                                        float *h_state, float *c_state, float *h_all, void *stream) {
     if (!m || B < 0 || T < 0) return QNN_ERR_INVALID_ARG;
     if (B == 0 || T == 0) return QNN_OK;
     if (!x || !y) return QNN_ERR_INVALID_ARG;
     cudaStream_t st = as_stream(stream);
+    if (m->stack > 1 || m->stack_stride > 1) QNN_TRY(stack_input(m, x, B, T, st, &x, &T));
     const int64_t L = m->L, I = m->I, H = m->H, P = m->P, C = m->C, R = m->R;
     const int64_t rows = B * T;
     const int64_t ld_in = round_up(I > R ? I : R, 64);

@@ -34,7 +34,11 @@ struct TcLayer {  // fp16 centered weight copies for the tensor-core recurrence 
 
 struct qnn_lstm_model {
     qnn_lstm_desc d{};
-    int64_t L = 0, I = 0, H = 0, P = 0, C = 0, R = 0;
+    int64_t L = 0, I = 0, H = 0, P = 0, C = 0, R = 0;  // I: features per network input
+    // frame stacking (Sec. 4 frontend): I = frame_dim * stack; one input every stack_stride frames
+    int64_t frame_dim = 0, stack = 1, stack_stride = 1;
+    void *fws = nullptr;  // frontend workspace: staged host frames and the stacked inputs
+    size_t fws_bytes = 0;
     int device = 0;
     void *weights = nullptr;
     std::vector<qnn::LayerDev> layers;

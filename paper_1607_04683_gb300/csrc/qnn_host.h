@@ -78,5 +78,8 @@ qnn_status launch_qgemm_tc(const uint8_t *A, int64_t lda, const qnn_qparams *pa,
                            void *scratch, cudaStream_t st);
 size_t tc_scratch_bytes(int64_t M, int64_t N, int64_t K);
 qnn_status launch_softmax_rows(const float *logits, int64_t rows, int64_t C, float *y, cudaStream_t st);
+// Sec. 4 frame stacking (frontend.cu): x [B][T][I] -> out [B][ceil(T/stride)][n I], device memory.
+qnn_status launch_stack_frames(const float *x, int64_t B, int64_t T, int64_t I, int n, int stride, float *out,
+                               cudaStream_t st);
 
 }  // namespace qnn

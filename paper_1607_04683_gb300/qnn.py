@@ -33,7 +33,7 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmul", "qnn_lstm_param_count",
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
            "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static",
-           "qnn_selftest_s64_to_f32")
+           "qnn_selftest_s64_to_f32", "qnn_stack_frames")
 
 
 class QnnError(RuntimeError):
@@ -45,7 +45,8 @@ class QnnError(RuntimeError):
 
 class LstmDesc(C.Structure):
     _fields_ = [("num_layers", C.c_int32), ("input_dim", C.c_int32), ("hidden", C.c_int32),
-                ("proj", C.c_int32), ("num_classes", C.c_int32), ("output_mode", C.c_int32)]
+                ("proj", C.c_int32), ("num_classes", C.c_int32), ("output_mode", C.c_int32),
+                ("stack", C.c_int32), ("stack_stride", C.c_int32)]
 
 
 _lib = None
@@ -84,6 +85,8 @@ def lib():
         L.qnn_measure_peak.argtypes = [i32, C.POINTER(C.c_double)]
         L.qnn_measure_peak.restype = i32
         L.qnn_selftest_s64_to_f32.argtypes = [P, P, i64, P]
+        L.qnn_stack_frames.argtypes = [P, i64, i64, i64, i32, i32, P, P]
+        L.qnn_stack_frames.restype = i32
         L.qnn_selftest_s64_to_f32.restype = i32
         L.qnn_quantize_matrix_static.argtypes = [P, i64, i64, i64, P, i64, P, P, P, P]
         L.qnn_quantize_matrix_static.restype = i32
@@ -187,10 +190,22 @@ def qnn_qmatmul(A, pa, ga, rsA, W, pw, csW, n_blocks=1, bias=None, want_acc=Fals
     return Y, acc
 
 
-def lstm_desc(num_layers, input_dim, hidden, proj=0, num_classes=0, output_mode=None) -> LstmDesc:
+def lstm_desc(num_layers, input_dim, hidden, proj=0, num_classes=0, output_mode=None, stack=0,
+              stack_stride=0) -> LstmDesc:
     if output_mode is None:
         output_mode = OUT_QUANT if num_classes > 0 else OUT_NONE
-    return LstmDesc(num_layers, input_dim, hidden, proj, num_classes, output_mode)
+    return LstmDesc(num_layers, input_dim, hidden, proj, num_classes, output_mode, stack, stack_stride)
+
+
+def stack_frames(x, n: int, stride: int, out=None, stream=None):
+    """Sec. 4 frontend on a CUDA tensor x [B, T, I]: [B, ceil(T/stride), n*I], input t' = frames
+    stride*t' .. stride*t' + n - 1 concatenated (the last frame standing in past the end)."""
+    import torch
+    B, T, I = x.shape
+    if out is None:
+        out = torch.empty((B, (T + stride - 1) // stride, n * I), dtype=torch.float32, device=x.device)
+    _check(lib().qnn_stack_frames(_p(x), B, T, I, n, stride, _p(out), _stream(stream)), "qnn_stack_frames")
+    return out
 
 
 def qnn_lstm_param_count(d: LstmDesc) -> int:
@@ -235,11 +250,13 @@ class LstmModel:
         B, T, I = x.shape
         d = self.desc
         ycols = d.num_classes if d.num_classes > 0 else self.R
+        if d.stack_stride > 1:  # frame stacking: one network input every stack_stride frames
+            T = (T + d.stack_stride - 1) // d.stack_stride
         if y is None:
             if isinstance(x, np.ndarray):
                 y = np.empty((B, T, ycols), np.float32)
             else:
                 y = torch.empty((B, T, ycols), dtype=torch.float32, device=x.device)
-        _check(lib().qnn_lstm_forward(self._h, _p(x), B, T, _p(y), _p(h_state), _p(c_state), _p(h_all),
+        _check(lib().qnn_lstm_forward(self._h, _p(x), B, x.shape[1], _p(y), _p(h_state), _p(c_state), _p(h_all),
                                       _stream(stream)), "qnn_lstm_forward")
         return y

@@ -43,6 +43,10 @@ def test_param_count_matches_oracle_layout(qlib):
         d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes)
         od = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes)
         assert qnn.qnn_lstm_param_count(d) == oracle.lstm_param_count(od) == wl.param_count()
+    # frame stacking: the first layer takes input_dim * stack features
+    d = qnn.lstm_desc(2, 40, 64, 16, 10, stack=8, stack_stride=3)
+    assert qnn.qnn_lstm_param_count(d) == oracle.lstm_param_count(oracle.desc(2, 320, 64, 16, 10))
+    assert qnn.qnn_lstm_param_count(qnn.lstm_desc(1, 40, 8, stack=-1)) == -1
     bad = qnn.lstm_desc(0, 4, 4)
     assert qnn.qnn_lstm_param_count(bad) == -1
     bad = qnn.LstmDesc(1, 4, 4, 0, 5, qnn.OUT_NONE)  # classes without an output layer mode
@@ -61,3 +65,5 @@ def test_argument_errors_need_no_gpu(qlib):
                             None) == qnn.QNN_ERR_INVALID_ARG
     h = C.c_void_p()
     assert qlib.qnn_lstm_model_create(C.byref(qnn.lstm_desc(0, 1, 1)), None, C.byref(h)) == qnn.QNN_ERR_INVALID_ARG
+    for args in ((-1, 3, 4, 8, 3), (1, 0, 4, 8, 3), (1, 3, 0, 8, 3), (1, 3, 4, 0, 3), (1, 3, 4, 8, 0)):
+        assert qlib.qnn_stack_frames(None, *args, None, None) == qnn.QNN_ERR_INVALID_ARG

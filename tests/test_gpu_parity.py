@@ -415,3 +415,42 @@ def test_benchmarked_workload_takes_the_small_path(qnn, monkeypatch):
     _gpu_forward(qnn, wl, params, x, h_all=False)
     qnn.profile_enable(False)
     assert "lstm_small" in qnn.profile_read()
+
+
+# ------------------------------------------------------------------------------------------
+# Frame stacking (Sec. 4 frontend)
+# ------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("B,T,I,n,stride", [(1, 300, 40, 8, 3), (3, 17, 40, 8, 3), (2, 5, 7, 3, 2), (4, 1, 12, 8, 3),
+                                            (2, 50, 80, 1, 1), (5, 31, 3, 4, 5)])
+def test_stack_frames_bit_exact(qnn, B, T, I, n, stride):
+    x = rng(B * 1000 + T + I).normal(0, 1, (B, T, I)).astype(np.float32)
+    got = qnn.stack_frames(gpu(x), n, stride)
+    assert qnn.device_status() == qnn.QNN_OK
+    assert np.array_equal(got.cpu().numpy(), oracle.stack_frames(x, n, stride))
+
+
+@pytest.mark.parametrize("path,B", [("small", 2), ("layerwise", 5), ("tc", 70)])
+def test_lstm_with_stacked_frames(qnn, path, B, monkeypatch):
+    """A model with the paper's frontend (8 frames of 40 features, every third presented) against the
+    oracle run on the stacked frames; raw frames passed as device memory and as host memory."""
+    monkeypatch.setenv("QNN_LSTM_PATH", path)
+    L, I, H, C, T, n, stride = 2, 40, 64, 11, 20, 8, 3
+    wl = _small(L=L, I=I * n, H=H, C=C, B=B, T=T, w=0.1)
+    params, _ = wl.make()
+    x = rng(B + 7).normal(0, 1, (B, T, I)).astype(np.float32)
+    xs = oracle.stack_frames(x, n, stride)
+    ref = _oracle(wl, params, xs, want_h_all=True)
+    d = qnn.lstm_desc(L, I, H, 0, C, stack=n, stack_stride=stride)
+    model = qnn.LstmModel(d, gpu(params))
+    Tp = xs.shape[1]
+    ha = torch.empty((L, B, Tp, H), dtype=torch.float32, device="cuda")
+    hs = torch.zeros((L, B, H), dtype=torch.float32, device="cuda")
+    cs = torch.zeros((L, B, H), dtype=torch.float32, device="cuda")
+    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha)
+    assert qnn.device_status() == qnn.QNN_OK
+    assert y.shape == (B, Tp, C)
+    got = {"y": y.cpu().numpy(), "h": hs.cpu().numpy(), "c": cs.cpu().numpy(), "h_all": ha.cpu().numpy()}
+    _compare(got, ref, wl)
+    y_host = model.forward(x)  # host frames: staged inside the call
+    assert np.array_equal(y_host, got["y"])
