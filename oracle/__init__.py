@@ -51,7 +51,8 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 
 class LstmDesc(C.Structure):
     _fields_ = [("num_layers", C.c_int32), ("input_dim", C.c_int32), ("hidden", C.c_int32),
-                ("proj", C.c_int32), ("num_classes", C.c_int32), ("output_mode", C.c_int32)]
+                ("proj", C.c_int32), ("num_classes", C.c_int32), ("output_mode", C.c_int32),
+                ("weight_blocks", C.c_int32)]
 
 
 def build(force: bool = False) -> str:
@@ -183,10 +184,11 @@ def tanh(x: float) -> float:
     return float(lib().orc_tanh(C.c_float(x)))
 
 
-def desc(num_layers, input_dim, hidden, proj=0, num_classes=0, output_mode=None) -> LstmDesc:
+def desc(num_layers, input_dim, hidden, proj=0, num_classes=0, output_mode=None, weight_blocks=0) -> LstmDesc:
+    """weight_blocks: quantization units per weight matrix, as equal blocks of rows (Sec. 3.1)."""
     if output_mode is None:
         output_mode = OUT_QUANT if num_classes > 0 else OUT_NONE
-    return LstmDesc(num_layers, input_dim, hidden, proj, num_classes, output_mode)
+    return LstmDesc(num_layers, input_dim, hidden, proj, num_classes, output_mode, weight_blocks)
 
 
 def lstm_param_count(d: LstmDesc) -> int:
@@ -224,7 +226,8 @@ def lstm_quantize_weights(d: LstmDesc, params: np.ndarray):
     params = np.ascontiguousarray(params, np.float32)
     n = lstm_param_count(d)
     codes = np.zeros(n, np.uint8)
-    qp = np.zeros(9 * d.num_layers + 1, QPARAMS_DTYPE)
+    nb = max(1, d.weight_blocks)
+    qp = np.zeros(nb * (9 * d.num_layers + 1), QPARAMS_DTYPE)
     nu = C.c_int64(0)
     _check(lib().orc_lstm_quantize_weights(C.byref(d), _ptr(params), _ptr(codes), _ptr(qp), C.byref(nu)))
     return codes, qp[: nu.value]

@@ -27,8 +27,9 @@
  *      with a projection r = R(Q(m) Wp), no bias, no nonlinearity.
  *   R5 E: a pinned fp32 exponential (Cody-Waite reduction, degree-7 Taylor polynomial by fmaf
  *      Horner, exact power-of-two scale) used for sigmoid, tanh and softmax on both sides.
- *   R6 granularity: weights one unit per gate matrix (Sec. 3.1 last paragraph); activations
- *      one unit per row (one frame of one sequence) inside the LSTM.
+ *   R6 granularity: weights one unit per gate matrix (Sec. 3.1 last paragraph), or per block of
+ *      its rows when the descriptor asks for sub-matrices; activations one unit per row (one frame
+ *      of one sequence) inside the LSTM.
  *   R7 output layer: logits = R(Q(r) Wo) + bo then softmax ("quant-all", Sec. 5); the float
  *      variant ("quant") computes the logits in fp64 and rounds them once to fp32.
  *   R9 frame stacking (Sec. 4 frontend): network input t' is the n frames starting at frame
@@ -270,6 +271,8 @@ typedef struct {
     int32_t proj;        /* P, recurrent projection size; 0 = none */
     int32_t num_classes; /* C, output classes; 0 = no output layer */
     int32_t output_mode; /* ORC_OUT_NONE / ORC_OUT_QUANT / ORC_OUT_FLOAT */
+    int32_t weight_blocks; /* Sec. 3.1 granularity: units per weight matrix, as equal blocks of rows
+                              (sub-matrices); 0 or 1 = one unit per matrix */
 } orc_lstm_desc;
 
 /* Packed fp32 parameter layout, layer by layer (Ik = I for the first layer, else Rr = P or H):
@@ -286,26 +289,54 @@ int64_t orc_lstm_param_count(const orc_lstm_desc *d)
     return n;
 }
 
-typedef struct { /* one quantized weight unit: rows x cols codes with one set of parameters */
+/* One quantized weight matrix: rows x cols codes, its rows split into nb equal blocks
+ * (sub-matrices), each block one quantization unit with its own parameters (Sec. 3.1). */
+typedef struct {
     uint8_t *codes;
-    orc_qparams p;
-    int64_t rows, cols;
+    orc_qparams *p; /* [nb] */
+    int64_t rows, cols, nb;
 } qunit;
 
-static int make_unit(const float *w, int64_t rows, int64_t cols, qunit *u)
+static int make_unit(const float *w, int64_t rows, int64_t cols, int64_t nb, qunit *u)
 {
     u->rows = rows;
     u->cols = cols;
+    u->nb = nb;
     u->codes = (uint8_t *)malloc((size_t)(rows * cols));
-    if (!u->codes) return ORC_ERR_INVALID_ARG;
-    return orc_quantize(w, rows, cols, cols, ORC_PER_MATRIX, u->codes, cols, &u->p, NULL);
+    u->p = (orc_qparams *)calloc((size_t)nb, sizeof(orc_qparams));
+    if (!u->codes || !u->p || rows % nb) return ORC_ERR_INVALID_ARG;
+    const int64_t per = rows / nb;
+    for (int64_t b = 0; b < nb; ++b) {
+        int st = orc_quantize(w + b * per * cols, per, cols, cols, ORC_PER_MATRIX, u->codes + b * per * cols, cols,
+                              &u->p[b], NULL);
+        if (st) return st;
+    }
+    return ORC_OK;
 }
 
-/* Recovered product of one quantized activation row with row n of a weight unit. */
+static void free_unit(qunit *u)
+{
+    free(u->codes);
+    free(u->p);
+}
+
+/* Recovered product of one quantized activation row with row n of a weight matrix, with the
+ * parameters of the block (unit) that row belongs to. */
 static float unit_dot(const uint8_t *a, const orc_qparams *pa, const qunit *u, int64_t n)
 {
-    int64_t S = offset_product(a, pa->z, u->codes + n * u->cols, u->p.z, u->cols);
-    return recover_product(S, pa->Q, u->p.Q);
+    const orc_qparams *pw = &u->p[n / (u->rows / u->nb)];
+    int64_t S = offset_product(a, pa->z, u->codes + n * u->cols, pw->z, u->cols);
+    return recover_product(S, pa->Q, pw->Q);
+}
+
+/* Units per weight matrix (Sec. 3.1 granularity), or 0 when a matrix's rows do not split evenly. */
+static int64_t blocks_of(const orc_lstm_desc *d)
+{
+    const int64_t nb = d->weight_blocks > 1 ? d->weight_blocks : 1;
+    if (d->hidden % nb) return 0;
+    if (d->proj > 0 && d->proj % nb) return 0;
+    if (d->num_classes > 0 && d->output_mode == ORC_OUT_QUANT && d->num_classes % nb) return 0;
+    return nb;
 }
 
 /* Quantize one activation row (one unit, reading R6). */
@@ -347,8 +378,10 @@ int orc_lstm_forward(const orc_lstm_desc *d, const float *params, const float *x
     if (L <= 0 || I <= 0 || H <= 0 || P < 0 || C < 0 || B < 0 || T < 0) return ORC_ERR_INVALID_ARG;
     if (C > 0 && d->output_mode != ORC_OUT_QUANT && d->output_mode != ORC_OUT_FLOAT) return ORC_ERR_INVALID_ARG;
     if (I > ORC_K_MAX || H > ORC_K_MAX || R > ORC_K_MAX) return ORC_ERR_K_TOO_LARGE;
+    const int64_t nb = blocks_of(d);
+    if (!nb) return ORC_ERR_INVALID_ARG;
 
-    /* a1: offline weight quantization, one unit per gate matrix */
+    /* a1: offline weight quantization, one unit per gate matrix (or per block of its rows) */
     qunit *wx = (qunit *)calloc((size_t)(4 * L), sizeof(qunit));
     qunit *wh = (qunit *)calloc((size_t)(4 * L), sizeof(qunit));
     qunit *wp = (qunit *)calloc((size_t)L, sizeof(qunit));
@@ -360,20 +393,20 @@ int orc_lstm_forward(const orc_lstm_desc *d, const float *params, const float *x
     const float *q = params;
     for (int64_t l = 0; l < L && !st; ++l) {
         int64_t Ik = (l == 0) ? I : R;
-        for (int g = 0; g < 4 && !st; ++g) st = make_unit(q + g * H * Ik, H, Ik, &wx[4 * l + g]);
+        for (int g = 0; g < 4 && !st; ++g) st = make_unit(q + g * H * Ik, H, Ik, nb, &wx[4 * l + g]);
         q += 4 * H * Ik;
-        for (int g = 0; g < 4 && !st; ++g) st = make_unit(q + g * H * R, H, R, &wh[4 * l + g]);
+        for (int g = 0; g < 4 && !st; ++g) st = make_unit(q + g * H * R, H, R, nb, &wh[4 * l + g]);
         q += 4 * H * R;
         bias[l] = q;
         q += 4 * H;
         if (P > 0) {
-            if (!st) st = make_unit(q, P, H, &wp[l]);
+            if (!st) st = make_unit(q, P, H, nb, &wp[l]);
             q += P * H;
         }
     }
     if (C > 0 && !st) {
         wo_f = q;
-        if (d->output_mode == ORC_OUT_QUANT) st = make_unit(q, C, R, &wo);
+        if (d->output_mode == ORC_OUT_QUANT) st = make_unit(q, C, R, nb, &wo);
         q += C * R;
         bo = q;
     }
@@ -459,11 +492,11 @@ int orc_lstm_forward(const orc_lstm_desc *d, const float *params, const float *x
     }
 
     for (int64_t i = 0; i < 4 * L; ++i) {
-        free(wx[i].codes);
-        free(wh[i].codes);
+        free_unit(&wx[i]);
+        free_unit(&wh[i]);
     }
-    for (int64_t i = 0; i < L; ++i) free(wp[i].codes);
-    free(wo.codes);
+    for (int64_t i = 0; i < L; ++i) free_unit(&wp[i]);
+    free_unit(&wo);
     free(wx);
     free(wh);
     free(wp);
@@ -488,33 +521,39 @@ int orc_lstm_quantize_weights(const orc_lstm_desc *d, const float *params, uint8
 {
     const int64_t L = d->num_layers, I = d->input_dim, H = d->hidden, P = d->proj, C = d->num_classes;
     const int64_t R = P > 0 ? P : H;
+    const int64_t nb = blocks_of(d);
+    if (!nb) return ORC_ERR_INVALID_ARG;
     const float *q = params;
     int64_t u = 0, off = 0;
     int st = ORC_OK;
+    /* one matrix of `rows` rows as nb units of rows/nb rows each, codes at the packed offset */
+#define ORC_UNITS(W, ROWS, COLS)                                                                      \
+    for (int64_t b_ = 0; b_ < nb && !st; ++b_, ++u)                                                   \
+        st = orc_quantize((W) + b_ * ((ROWS) / nb) * (COLS), (ROWS) / nb, (COLS), (COLS), ORC_PER_MATRIX, \
+                          codes + off + b_ * ((ROWS) / nb) * (COLS), (COLS), &qp[u], NULL);
     for (int64_t l = 0; l < L && !st; ++l) {
         int64_t Ik = (l == 0) ? I : R;
-        for (int g = 0; g < 4 && !st; ++g, ++u) {
-            st = orc_quantize(q + g * H * Ik, H, Ik, Ik, ORC_PER_MATRIX, codes + off, Ik, &qp[u], NULL);
+        for (int g = 0; g < 4 && !st; ++g) {
+            ORC_UNITS(q + g * H * Ik, H, Ik)
             off += H * Ik;
         }
         q += 4 * H * Ik;
-        for (int g = 0; g < 4 && !st; ++g, ++u) {
-            st = orc_quantize(q + g * H * R, H, R, R, ORC_PER_MATRIX, codes + off, R, &qp[u], NULL);
+        for (int g = 0; g < 4 && !st; ++g) {
+            ORC_UNITS(q + g * H * R, H, R)
             off += H * R;
         }
         q += 4 * H * R + 4 * H;
         off += 4 * H; /* bias slot: no codes */
         if (P > 0 && !st) {
-            st = orc_quantize(q, P, H, H, ORC_PER_MATRIX, codes + off, H, &qp[u], NULL);
-            ++u;
+            ORC_UNITS(q, P, H)
             off += P * H;
             q += P * H;
         }
     }
     if (C > 0 && d->output_mode == ORC_OUT_QUANT && !st) {
-        st = orc_quantize(q, C, R, R, ORC_PER_MATRIX, codes + off, R, &qp[u], NULL);
-        ++u;
+        ORC_UNITS(q, C, R)
     }
+#undef ORC_UNITS
     if (n_units) *n_units = u;
     return st;
 }

@@ -311,16 +311,20 @@ def _recovered_row(v):
     return (c[0].astype(np.float64) + int(p[0]["z"])) / float(p[0]["Q"])
 
 
-def _recovered_mat(w):
-    c, p, _ = oracle.quantize(np.asarray(w, F32), oracle.PER_MATRIX)
-    return (c.astype(np.float64) + int(p[0]["z"])) / float(p[0]["Q"])
+def _recovered_mat(w, nb=1):
+    """eq. (3) recovery of a weight matrix quantized as nb row blocks, each its own unit."""
+    out = []
+    for blk in np.split(np.asarray(w, F32), nb):
+        c, p, _ = oracle.quantize(blk, oracle.PER_MATRIX)
+        out.append((c.astype(np.float64) + int(p[0]["z"])) / float(p[0]["Q"]))
+    return np.concatenate(out)
 
 
 def _sig(x):
     return 1.0 / (1.0 + np.exp(-x))
 
 
-def _textbook_check(wl, params, x, res, tol_h):
+def _textbook_check(wl, params, x, res, tol_h, nb=1):
     """Teacher-forced: every step of the oracle's LSTM equals a float64 textbook LSTM step (no
     peepholes, gates [i, f, g, o]) applied to eq. (3)-recovered inputs and weights, fed with the
     oracle's own previous outputs."""
@@ -329,9 +333,9 @@ def _textbook_check(wl, params, x, res, tol_h):
     H = wl.hidden
     worst = 0.0
     for l, (wx, wh, b, wp) in enumerate(layers):
-        rwx = np.stack([_recovered_mat(wx[g]) for g in range(4)])
-        rwh = np.stack([_recovered_mat(wh[g]) for g in range(4)])
-        rwp = _recovered_mat(wp) if wp is not None else None
+        rwx = np.stack([_recovered_mat(wx[g], nb) for g in range(4)])
+        rwh = np.stack([_recovered_mat(wh[g], nb) for g in range(4)])
+        rwp = _recovered_mat(wp, nb) if wp is not None else None
         for bb in range(B):
             c = np.zeros(H)
             hprev = np.zeros(wl.R, F32)
@@ -350,7 +354,7 @@ def _textbook_check(wl, params, x, res, tol_h):
     assert worst <= tol_h, worst
     if out is not None and wl.output_mode == oracle.OUT_QUANT:
         wo, bo = out
-        rwo = _recovered_mat(wo)
+        rwo = _recovered_mat(wo, nb)
         for bb in range(B):
             for t in range(T):
                 r = _recovered_row(res["h_all"][-1, bb, t])
@@ -366,8 +370,8 @@ def _small(name="t", L=2, I=7, H=9, P=0, C=0, B=2, T=6, seed=5, mode=None, fb=1.
                                output_mode=(mode if mode is not None else (1 if C > 0 else 0)))
 
 
-def _run(wl, params, x, **kw):
-    d = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+def _run(wl, params, x, nb=0, **kw):
+    d = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode, nb)
     return oracle.lstm_forward(d, params, x, want_h_all=True, want_logits=wl.num_classes > 0, **kw)
 
 
@@ -553,3 +557,74 @@ def test_stack_frames_paper_frontend():
     # the last input reaches past frame 299: frames 297..304 -> 297, 298, 299, 299, ...
     last = s[0, 99].reshape(8, 40)[:, 0] / 40
     assert list(last) == [297, 298, 299, 299, 299, 299, 299, 299]
+
+
+
+# ------------------------------------------------------------------------------------------
+# Sub-matrix granularity (Sec. 3.1): a weight matrix quantized as row blocks, each its own unit
+# ------------------------------------------------------------------------------------------
+
+def _heterogeneous_blocks(wl, params, nb, seed=3):
+    """Rescale the row blocks of every weight matrix by very different factors (the case finer
+    granularity is for)."""
+    layers, out = _unpack(wl, params)
+    p = params.copy()
+    f = np.random.Generator(np.random.PCG64(seed)).choice([0.05, 0.3, 1.0, 4.0], size=nb)
+    scale = lambda w: (w.reshape(nb, -1) * f[:, None]).reshape(w.shape)
+    chunks = []
+    for wx, wh, b, wp in layers:
+        chunks += [np.stack([scale(wx[g]) for g in range(4)]).ravel(),
+                   np.stack([scale(wh[g]) for g in range(4)]).ravel(), b.ravel()]
+        if wp is not None:
+            chunks.append(scale(wp).ravel())
+    if out is not None:
+        chunks += [scale(out[0]).ravel(), out[1].ravel()]
+    return np.concatenate(chunks).astype(F32)
+
+
+@pytest.mark.parametrize("cfg,nb", [(dict(L=2, I=7, H=12, C=6), 3), (dict(L=2, I=6, H=16, P=8, C=8, T=5), 4),
+                                    (dict(L=1, I=5, H=6, B=1, T=8), 6)])
+def test_sub_matrix_units_reduce_to_textbook(cfg, nb):
+    """With nb units per matrix the oracle's LSTM is the textbook LSTM on operands recovered block
+    by block; using another block's parameters would break this by the ratio of their scales."""
+    wl = _small(**cfg)
+    params, x = wl.make()
+    params = _heterogeneous_blocks(wl, params, nb)
+    res = _run(wl, params, x, nb=nb)
+    _textbook_check(wl, params, x, res, tol_h=2e-3 if wl.proj else 2e-6, nb=nb)
+
+
+def test_sub_matrix_units_are_more_precise():
+    """Sec. 3.1: subdividing a matrix into individually quantized sub-matrices gives better
+    precision: the recovered weights of blocks with very different scales are closer to the
+    float weights, block by block, and so is the quantized LSTM to the float LSTM."""
+    wl = _small(L=1, I=16, H=32, B=1, T=30)
+    params, x = wl.make()
+    params = _heterogeneous_blocks(wl, params, 4)
+    wx = _unpack(wl, params)[0][0][0]
+    for g in range(4):
+        e1 = np.abs(_recovered_mat(wx[g], 1) - wx[g]).max(axis=1)
+        e4 = np.abs(_recovered_mat(wx[g], 4) - wx[g]).max(axis=1)
+        assert np.all(e4 <= e1 * (1 + 1e-6))
+    one, four = _run(wl, params, x, nb=1), _run(wl, params, x, nb=4)
+    float_h = _run(wl, params, x, nb=32)  # one unit per row: closest to float
+    d1 = np.abs(one["h_all"] - float_h["h_all"]).mean()
+    d4 = np.abs(four["h_all"] - float_h["h_all"]).mean()
+    assert d4 < d1
+
+
+def test_sub_matrix_weight_codes_by_block():
+    wl = _small(L=2, I=5, H=8, P=4, C=4)
+    params, _ = wl.make()
+    d = oracle.desc(2, 5, 8, 4, 4, oracle.OUT_QUANT, 2)
+    codes, prm = oracle.lstm_quantize_weights(d, params)
+    assert len(prm) == 2 * (9 * 2 + 1)
+    wx0 = _unpack(wl, params)[0][0][0][0]  # first gate matrix of layer 0: two units of 4 rows
+    for blk in range(2):
+        c, p, _ = oracle.quantize(wx0[4 * blk:4 * blk + 4], oracle.PER_MATRIX)
+        assert np.array_equal(codes[4 * blk * 5:(4 * blk + 4) * 5].reshape(4, 5), c)
+        assert prm[blk]["Q"] == p[0]["Q"] and prm[blk]["z"] == p[0]["z"]
+    assert oracle.lstm_param_count(d) == params.size
+    bad = oracle.desc(1, 5, 9, 0, 0, oracle.OUT_NONE, 2)  # 9 rows do not split in 2
+    with pytest.raises(oracle.OracleError):
+        oracle.lstm_forward(bad, np.zeros(oracle.lstm_param_count(bad), F32), np.zeros((1, 1, 5), F32))
