@@ -124,6 +124,10 @@ typedef struct {
                              The first layer then takes I * stack features. */
     int32_t stack_stride; /* only every stack_stride-th stacked frame is presented (the paper: 3);
                              0 or 1 = every frame */
+    int32_t weight_blocks; /* Sec. 3.1 granularity: every weight matrix (each gate's Wx and Wh, Wp,
+                              Wo) is quantized as this many equal blocks of rows (sub-matrices), each
+                              its own unit; 0 or 1 = one unit per matrix, the paper's setting. H, P
+                              and (quantized output layer) C must be multiples of it. */
 } qnn_lstm_desc;
 
 typedef struct qnn_lstm_model qnn_lstm_model;
@@ -136,7 +140,7 @@ typedef struct qnn_lstm_model qnn_lstm_model;
 int64_t qnn_lstm_param_count(const qnn_lstm_desc *d);
 
 /* Quantizes the weights offline (Sec. 3.1: one unit per gate matrix, per projection and per
- * output matrix) and keeps device copies in the model. `params` (host or device) is read during
+ * output matrix, or weight_blocks units per matrix) and keeps device copies in the model. `params` (host or device) is read during
  * the call only. The call is synchronous. *out receives the model (destroy with
  * qnn_lstm_model_destroy). */
 qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float *params, qnn_lstm_model **out);
@@ -145,7 +149,8 @@ void qnn_lstm_model_destroy(qnn_lstm_model *m);
 
 /* Copies the model's weight codes (host buffer, qnn_lstm_param_count bytes; the packed layout
  * with every bias slot zero) and the parameters of each unit in order (4 Wx, 4 Wh, Wp per layer,
- * then Wo; host buffer of at least 9 L + 1 entries) and their count. Synchronous. */
+ * then Wo, each matrix's blocks in row order; host buffer of at least S (9 L + 1) entries,
+ * S = max(weight_blocks, 1)) and their count. Synchronous. */
 qnn_status qnn_lstm_model_weights(const qnn_lstm_model *m, uint8_t *codes_host, qnn_qparams *params_host,
                                   int64_t *n_units);
 

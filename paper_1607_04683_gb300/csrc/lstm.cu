@@ -80,6 +80,7 @@ struct RecArgs {
     int *qsum;                // [B]
     int ldq, distq;
     int B, T, H, R, P, ldh, ldp, nc, np, bc;
+    int ups, cpu, ppu;        // weight units per gate matrix; cells (Wh rows) and Wp rows per unit
 };
 
 // Grid-wide barrier with a bounded wait: returns false if this or another block gave up, in
@@ -329,7 +330,7 @@ __global__ void __launch_bounds__(kRecThreads, 1) lstm_recurrent_kernel(RecArgs 
     auto h_row_info = [&](int lr, int &zw, float &Qw, int &csw, bool &valid) {
         const int gate = lr / nc, j = j0 + lr % nc;
         valid = j < H;
-        const qnn_qparams q = a.wh_p[gate];
+        const qnn_qparams q = a.wh_p[gate * a.ups + (valid ? j : 0) / a.cpu];  // the row's unit
         zw = q.z;
         Qw = q.Q;
         csw = valid ? a.wh_sum[gate * H + j] : 0;
@@ -337,7 +338,7 @@ __global__ void __launch_bounds__(kRecThreads, 1) lstm_recurrent_kernel(RecArgs 
     auto p_row_info = [&](int lr, int &zw, float &Qw, int &csw, bool &valid) {
         const int p = p0 + lr;
         valid = p < a.P;
-        const qnn_qparams q = a.wp_p[0];
+        const qnn_qparams q = a.wp_p[(valid ? p : 0) / a.ppu];
         zw = q.z;
         Qw = q.Q;
         csw = valid ? a.wp_sum[p] : 0;
@@ -508,7 +509,10 @@ int64_t network_input_dim(const qnn_lstm_desc *d) { return (int64_t)d->input_dim
 
 bool valid_desc(const qnn_lstm_desc *d) {
     if (!d || d->num_layers < 1 || d->input_dim < 1 || d->hidden < 1 || d->proj < 0 || d->num_classes < 0) return false;
-    if (d->stack < 0 || d->stack_stride < 0) return false;
+    if (d->stack < 0 || d->stack_stride < 0 || d->weight_blocks < 0) return false;
+    const int S = d->weight_blocks > 1 ? d->weight_blocks : 1;  // units per weight matrix
+    if (d->hidden % S || (d->proj > 0 && d->proj % S)) return false;
+    if (d->num_classes > 0 && d->output_mode == QNN_OUT_QUANT && d->num_classes % S) return false;
     if ((d->num_classes == 0) != (d->output_mode == QNN_OUT_NONE)) return false;
     if (d->output_mode < QNN_OUT_NONE || d->output_mode > QNN_OUT_FLOAT) return false;
     return true;
@@ -578,23 +582,25 @@ extern "C" qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float 
     m->d = *d;
     m->L = L, m->I = I, m->H = H, m->P = P, m->C = C, m->R = R;
     m->frame_dim = d->input_dim;
+    m->S = d->weight_blocks > 1 ? d->weight_blocks : 1;
     m->stack = d->stack > 1 ? d->stack : 1;
     m->stack_stride = d->stack_stride > 1 ? d->stack_stride : 1;
     cudaGetDevice(&m->device);
     m->layers.resize(L);
 
     // sizes
+    const int64_t S = m->S;
     size_t bytes = 0;
     auto acct = [&](size_t n) { bytes = (size_t)round_up((int64_t)bytes, 256) + n; };
     for (int64_t l = 0; l < L; ++l) {
         const int64_t kin = l == 0 ? I : R;
-        acct(4 * H * round_up(kin, 64)), acct(4 * H * 4), acct(4 * sizeof(qnn_qparams));
-        acct(4 * H * round_up(R, 64)), acct(4 * H * 4), acct(4 * sizeof(qnn_qparams));
+        acct(4 * H * round_up(kin, 64)), acct(4 * H * 4), acct(4 * S * sizeof(qnn_qparams));
+        acct(4 * H * round_up(R, 64)), acct(4 * H * 4), acct(4 * S * sizeof(qnn_qparams));
         acct(4 * H * 4);
-        if (P > 0) acct(P * round_up(H, 64)), acct(P * 4), acct(sizeof(qnn_qparams));
+        if (P > 0) acct(P * round_up(H, 64)), acct(P * 4), acct(S * sizeof(qnn_qparams));
     }
     if (C > 0) {
-        acct(C * round_up(R, 64)), acct(C * 4), acct(sizeof(qnn_qparams)), acct(C * 4);
+        acct(C * round_up(R, 64)), acct(C * 4), acct(S * sizeof(qnn_qparams)), acct(C * 4);
         if (d->output_mode == QNN_OUT_FLOAT) acct(C * R * 4);
     }
     acct((size_t)n_params * 4);  // device copy of the fp32 parameters (freed region reused later)
@@ -621,16 +627,16 @@ extern "C" qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float 
             u.sums = bp.take<int32_t>(rows);
             u.params = bp.take<qnn_qparams>(units);
         };
-        mk(ly.wx, 4 * H, ly.kin, 4);
-        mk(ly.wh, 4 * H, R, 4);
+        mk(ly.wx, 4 * H, ly.kin, 4 * (int)m->S);
+        mk(ly.wh, 4 * H, R, 4 * (int)m->S);
         ly.bias = bp.take<float>(4 * H);
-        if (P > 0) mk(ly.wp, P, H, 1);
+        if (P > 0) mk(ly.wp, P, H, (int)m->S);
     }
     if (C > 0) {
-        m->wo.rows = C, m->wo.cols = R, m->wo.ld = round_up(R, 64), m->wo.n_units = 1;
+        m->wo.rows = C, m->wo.cols = R, m->wo.ld = round_up(R, 64), m->wo.n_units = (int)m->S;
         m->wo.codes = bp.take<uint8_t>(C * m->wo.ld);
         m->wo.sums = bp.take<int32_t>(C);
-        m->wo.params = bp.take<qnn_qparams>(1);
+        m->wo.params = bp.take<qnn_qparams>(m->S);
         m->bo = bp.take<float>(C);
         if (d->output_mode == QNN_OUT_FLOAT) m->wo_f = bp.take<float>(C * R);
     }
@@ -644,21 +650,21 @@ extern "C" qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float 
     const float *q = pdev;
     for (int64_t l = 0; l < L && st == QNN_OK; ++l) {
         LayerDev &ly = m->layers[l];
-        st = quantize_units(q, 4 * H, ly.kin, 4, ly.wx, partials, counter, max_blocks, s);
+        st = quantize_units(q, 4 * H, ly.kin, ly.wx.n_units, ly.wx, partials, counter, max_blocks, s);
         q += 4 * H * ly.kin;
-        if (st == QNN_OK) st = quantize_units(q, 4 * H, R, 4, ly.wh, partials, counter, max_blocks, s);
+        if (st == QNN_OK) st = quantize_units(q, 4 * H, R, ly.wh.n_units, ly.wh, partials, counter, max_blocks, s);
         q += 4 * H * R;
         if (st == QNN_OK && cudaMemcpy(ly.bias, q, 4 * H * 4, cudaMemcpyDeviceToDevice) != cudaSuccess)
             st = QNN_ERR_CUDA;
         q += 4 * H;
         if (P > 0) {
-            if (st == QNN_OK) st = quantize_units(q, P, H, 1, ly.wp, partials, counter, max_blocks, s);
+            if (st == QNN_OK) st = quantize_units(q, P, H, ly.wp.n_units, ly.wp, partials, counter, max_blocks, s);
             q += P * H;
         }
     }
     if (C > 0 && st == QNN_OK) {
         if (d->output_mode == QNN_OUT_QUANT)
-            st = quantize_units(q, C, R, 1, m->wo, partials, counter, max_blocks, s);
+            st = quantize_units(q, C, R, m->wo.n_units, m->wo, partials, counter, max_blocks, s);
         else if (cudaMemcpy(m->wo_f, q, C * R * 4, cudaMemcpyDeviceToDevice) != cudaSuccess)
             st = QNN_ERR_CUDA;
         q += C * R;
@@ -671,24 +677,20 @@ extern "C" qnn_status qnn_lstm_model_create(const qnn_lstm_desc *d, const float 
     }
     // host mirror of the unit parameters, in the documented order
     if (st == QNN_OK) {
+        auto mirror = [&](const QUnitDev &u) {
+            std::vector<qnn_qparams> tmp(u.n_units);
+            if (cudaMemcpy(tmp.data(), u.params, u.n_units * sizeof(qnn_qparams), cudaMemcpyDeviceToHost) !=
+                cudaSuccess)
+                st = QNN_ERR_CUDA;
+            m->host_params.insert(m->host_params.end(), tmp.begin(), tmp.end());
+        };
         for (int64_t l = 0; l < L && st == QNN_OK; ++l) {
-            qnn_qparams tmp[4];
-            LayerDev &ly = m->layers[l];
-            if (cudaMemcpy(tmp, ly.wx.params, sizeof(tmp), cudaMemcpyDeviceToHost) != cudaSuccess) st = QNN_ERR_CUDA;
-            m->host_params.insert(m->host_params.end(), tmp, tmp + 4);
-            if (cudaMemcpy(tmp, ly.wh.params, sizeof(tmp), cudaMemcpyDeviceToHost) != cudaSuccess) st = QNN_ERR_CUDA;
-            m->host_params.insert(m->host_params.end(), tmp, tmp + 4);
-            if (P > 0) {
-                if (cudaMemcpy(tmp, ly.wp.params, sizeof(qnn_qparams), cudaMemcpyDeviceToHost) != cudaSuccess)
-                    st = QNN_ERR_CUDA;
-                m->host_params.push_back(tmp[0]);
-            }
+            const LayerDev &ly = m->layers[l];
+            mirror(ly.wx);
+            mirror(ly.wh);
+            if (P > 0) mirror(ly.wp);
         }
-        if (C > 0 && d->output_mode == QNN_OUT_QUANT && st == QNN_OK) {
-            qnn_qparams tmp;
-            if (cudaMemcpy(&tmp, m->wo.params, sizeof(tmp), cudaMemcpyDeviceToHost) != cudaSuccess) st = QNN_ERR_CUDA;
-            m->host_params.push_back(tmp);
-        }
+        if (C > 0 && d->output_mode == QNN_OUT_QUANT && st == QNN_OK) mirror(m->wo);
     }
     if (st != QNN_OK) {
         qnn_lstm_model_destroy(m);
@@ -896,8 +898,8 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
         // 1. quantize every frame of the layer input (one unit per row)
         QNN_TRY(launch_quantize_rows(in, rows, kin, kin, codes, ld_in, prm, rs, st));
         // 2. batched input product, recovered, plus bias
-        QNN_TRY(launch_qgemm(codes, ld_in, prm, QNN_PER_ROW, rs, rows, kin, ly.wx.codes, ly.wx.ld, ly.wx.params, H,
-                             ly.wx.sums, 4 * H, ly.bias, px, 4 * H, nullptr, st));
+        QNN_TRY(launch_qgemm(codes, ld_in, prm, QNN_PER_ROW, rs, rows, kin, ly.wx.codes, ly.wx.ld, ly.wx.params,
+                             H / m->S, ly.wx.sums, 4 * H, ly.bias, px, 4 * H, nullptr, st));
         // 3. recurrence
         float *outl = (ha_dev ? h_all + l * rows * R : seq[l & 1]);
         if (c_state)
@@ -922,6 +924,7 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
             a.qsum = reinterpret_cast<int *>(ws + o_qs);
             a.ldq = (int)ldq;
             a.distq = B >= kDistQuantMinBatch;  // below this, each block quantizing its rows is cheaper
+            a.ups = (int)m->S, a.cpu = (int)(H / m->S), a.ppu = P > 0 ? (int)(P / m->S) : 1;
             void *args[] = {&a};
             ProfScope prof("lstm_recurrent", st);
             cudaError_t e = cudaLaunchCooperativeKernel((const void *)lstm_recurrent_kernel, dim3(plan.grid),
@@ -945,8 +948,8 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     if (C > 0) {
         if (m->d.output_mode == QNN_OUT_QUANT) {
             QNN_TRY(launch_quantize_rows(in, rows, R, R, codes, ld_in, prm, rs, st));
-            QNN_TRY(launch_qgemm(codes, ld_in, prm, QNN_PER_ROW, rs, rows, R, m->wo.codes, m->wo.ld, m->wo.params, C,
-                                 m->wo.sums, C, m->bo, lg, C, nullptr, st));
+            QNN_TRY(launch_qgemm(codes, ld_in, prm, QNN_PER_ROW, rs, rows, R, m->wo.codes, m->wo.ld, m->wo.params,
+                                 C / m->S, m->wo.sums, C, m->bo, lg, C, nullptr, st));
         } else {
             dim3 grid((unsigned)((C + 31) / 32), (unsigned)((rows + 31) / 32));
             ProfScope prof("float_linear", st);

@@ -37,6 +37,7 @@ struct qnn_lstm_model {
     int64_t L = 0, I = 0, H = 0, P = 0, C = 0, R = 0;  // I: features per network input
     // frame stacking (Sec. 4 frontend): I = frame_dim * stack; one input every stack_stride frames
     int64_t frame_dim = 0, stack = 1, stack_stride = 1;
+    int64_t S = 1;  // quantization units per weight matrix (equal row blocks, Sec. 3.1 granularity)
     void *fws = nullptr;  // frontend workspace: staged host frames and the stacked inputs
     size_t fws_bytes = 0;
     int device = 0;

@@ -93,6 +93,7 @@ struct SmallArgs {
     int *abort_flag;
     unsigned epoch;
     int L, I, H, R, C, B, T, CS;
+    int ups, cpu, opu;  // weight units per matrix; cells per gate unit; output rows per Wo unit
 };
 
 // ---- shared memory layout ---------------------------------------------------------------------
@@ -483,7 +484,7 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                              S.codes_x[b], true, rs);
                     if (row_writer && o_n >= 0) {
                         const RowMeta mt = S.meta_x[par][b];
-                        const qnn_qparams po = a.wo_p[0];
+                        const qnn_qparams po = a.wo_p[o_n / a.opu];
                         const long long Sv = offset_product(s, mt.za, po.z, rs, o_cs, R);
                         a.logits[((int64_t)b * T + t) * a.C + o_n] = __fadd_rn(recover_product(Sv, mt.Qa, po.Q), o_b);
                     }
@@ -554,7 +555,8 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
         const int64_t n = (int64_t)g * H + (jv ? j : 0);
         const int csx = jv ? ly.wx_sum[n] : 0, csh = jv ? ly.wh_sum[n] : 0;
         const float bias = jv ? ly.bias[n] : 0.0f;
-        const qnn_qparams px = ly.wx_p[g], ph = ly.wh_p[g];
+        const int unit = g * a.ups + (jv ? j : 0) / a.cpu;  // this (cell, gate) row's weight unit
+        const qnn_qparams px = ly.wx_p[unit], ph = ly.wh_p[unit];
         const int ew = warp - kPW;
         const bool tag_out = (l < a.L - 1) || (a.C > 0);
         float c[kMaxB], hl[kMaxB];
@@ -770,6 +772,7 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
     a.abort_flag = reinterpret_cast<int *>(ws + o_flag);
     a.epoch = m->epoch;
     a.L = (int)L, a.I = (int)I, a.H = (int)H, a.R = (int)R, a.C = (int)C, a.B = (int)B, a.T = (int)T, a.CS = CS;
+    a.ups = (int)m->S, a.cpu = (int)(H / m->S), a.opu = C > 0 ? (int)(C / m->S) : 1;
     {
         ProfScope prof("lstm_small", st);
         QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, lstm_small_kernel, a));

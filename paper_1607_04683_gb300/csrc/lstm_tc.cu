@@ -227,7 +227,7 @@ bool pdl_enabled() {
 }  // namespace
 
 bool tc_recurrence_supported(const qnn_lstm_model *m) {
-    return m->H % 4 == 0 && round_up(m->R, 64) <= 1024;
+    return m->H % 4 == 0 && (m->H / m->S) % 4 == 0 && round_up(m->R, 64) <= 1024;
 }
 
 qnn_status tc_prepare(qnn_lstm_model *m) {
@@ -313,12 +313,13 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
         const float *src = t == 0 ? h0 : out + (t - 1) * R;
         const int64_t ld = t == 0 ? R : T * R;
         QNN_TRY(launch_quantize_rows_f16(src, ld, B, R, kh, a16, prm, rs, status, t > 0 && gates.pdl, st));
-        TcLstmOut o{px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R, (int)H};
+        TcLstmOut o{px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R, (int)H,
+                    (int)m->S, (int)(H / m->S)};
         QNN_TRY(tc_lstm_gates(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, st));
         if (P > 0) {
             QNN_TRY(launch_quantize_rows_f16(mbuf, H, B, H, kpj, m16, prm_m, rs_m, status, gates.pdl, st));
-            QNN_TRY(tc_linear(proj, prm_m, 1, rs_m, H, ly.wp.params, P, ly.wp.sums, nullptr, out + t * R, T * R,
-                              nullptr, st));
+            QNN_TRY(tc_linear(proj, prm_m, 1, rs_m, H, ly.wp.params, P / m->S, ly.wp.sums, nullptr, out + t * R,
+                              T * R, nullptr, st));
         }
     }
     return QNN_OK;

@@ -558,15 +558,6 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 Qa = qa.Q;
                 rs = args.rsA[b];
             }
-            // eq. (1) expanded around the centered product P: S = P + rt[g] + (128 + za) csW
-            long long rt[4];
-            float den[4];
-#pragma unroll
-            for (int g = 0; g < 4; ++g) {
-                const qnn_qparams qw = args.pw[g];
-                rt[g] = (long long)(128 + qw.z) * rs + (long long)K * ((long long)za * qw.z - 16384);
-                den[g] = __fmul_rn(Qa, qw.Q);
-            }
             const int za128 = 128 + za;
             const int buf = (int)(gc & 1);
             // this warp's first slice: the input products and cell state do not depend on the
@@ -592,6 +583,17 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 for (int g = 0; g < 4; ++g) tmem_ld4_nowait(ta + 8 * g, r[g]);
                 tmem_wait_ld();
                 if (bv && j0 < H) {
+                    // eq. (1) expanded around the centered product P: S = P + rt[g] + (128 + za) csW,
+                    // with the weight unit of the slice's cells (one per gate matrix, or per block)
+                    long long rt[4];
+                    float den[4];
+                    const int unit = j0 / E.cpu;
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        const qnn_qparams qw = args.pw[g * E.ups + unit];
+                        rt[g] = (long long)(128 + qw.z) * rs + (long long)K * ((long long)za * qw.z - 16384);
+                        den[g] = __fmul_rn(Qa, qw.Q);
+                    }
                     const float *pxr = E.px + b * E.px_ld + j0;
                     float *cr = E.c + b * (int64_t)H + j0;
                     float pre[4][4];
@@ -832,6 +834,7 @@ qnn_status tc_linear(const TcOperands &op, const qnn_qparams *pa, int per_row, c
 qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int32_t *rsA, int64_t K,
                          const qnn_qparams *pw4, const int32_t *cs, const TcLstmOut &out, cudaStream_t st) {
     if (K <= 0 || op.kp > KCHUNK || K > op.kp || out.H <= 0 || out.H % 4 != 0) return QNN_ERR_INVALID_ARG;
+    if (out.ups < 1 || out.cpu < 4 || out.cpu % 4 != 0 || out.cpu * out.ups != out.H) return QNN_ERR_INVALID_ARG;
     if (op.N != 4 * ((out.H + 7) / 8 * 8)) return QNN_ERR_INVALID_ARG;
     int *status = nullptr;
     QNN_TRY(status_word(&status));

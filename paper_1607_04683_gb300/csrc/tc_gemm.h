@@ -48,12 +48,14 @@ struct TcLstmOut {
     float *h;
     int64_t h_ld;
     int H;
+    int ups = 1;  // weight units per gate matrix (Sec. 3.1 sub-matrices); pw4 then has 4 ups entries
+    int cpu = 0;  // cells per unit (H / ups, a multiple of 4)
 };
 
 // One recurrent step's gate product and cell update: A = centered codes of h_{t-1} (one unit per
 // row: pa, rsA), W = the four Wh gate matrices interleaved in 8-cell groups [i f g o] x 8 rows
-// (op.N = 4 * round_up(H, 8)), pw4 the four gate units, cs their row code sums in gate-major order
-// [4][H]. K (true) <= 1024.
+// (op.N = 4 * round_up(H, 8)), pw4 the gate units (4 ups, gate-major), cs their row code sums in
+// gate-major order [4][H]. K (true) <= 1024.
 qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int32_t *rsA, int64_t K,
                          const qnn_qparams *pw4, const int32_t *cs, const TcLstmOut &out, cudaStream_t st);
 

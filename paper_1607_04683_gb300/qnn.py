@@ -46,7 +46,7 @@ class QnnError(RuntimeError):
 class LstmDesc(C.Structure):
     _fields_ = [("num_layers", C.c_int32), ("input_dim", C.c_int32), ("hidden", C.c_int32),
                 ("proj", C.c_int32), ("num_classes", C.c_int32), ("output_mode", C.c_int32),
-                ("stack", C.c_int32), ("stack_stride", C.c_int32)]
+                ("stack", C.c_int32), ("stack_stride", C.c_int32), ("weight_blocks", C.c_int32)]
 
 
 _lib = None
@@ -191,10 +191,11 @@ def qnn_qmatmul(A, pa, ga, rsA, W, pw, csW, n_blocks=1, bias=None, want_acc=Fals
 
 
 def lstm_desc(num_layers, input_dim, hidden, proj=0, num_classes=0, output_mode=None, stack=0,
-              stack_stride=0) -> LstmDesc:
+              stack_stride=0, weight_blocks=0) -> LstmDesc:
     if output_mode is None:
         output_mode = OUT_QUANT if num_classes > 0 else OUT_NONE
-    return LstmDesc(num_layers, input_dim, hidden, proj, num_classes, output_mode, stack, stack_stride)
+    return LstmDesc(num_layers, input_dim, hidden, proj, num_classes, output_mode, stack, stack_stride,
+                    weight_blocks)
 
 
 def stack_frames(x, n: int, stride: int, out=None, stream=None):

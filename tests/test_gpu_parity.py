@@ -5,6 +5,8 @@ bit-exact (the whole recurrence is the same sequence of fp32 operations on both 
 difference would be a bug); softmax outputs within 1e-4 absolute (their sums run in a different
 order on the GPU).
 """
+import ctypes
+
 import numpy as np
 import pytest
 
@@ -454,3 +456,78 @@ def test_lstm_with_stacked_frames(qnn, path, B, monkeypatch):
     _compare(got, ref, wl)
     y_host = model.forward(x)  # host frames: staged inside the call
     assert np.array_equal(y_host, got["y"])
+
+
+# ------------------------------------------------------------------------------------------
+# Sub-matrix granularity (Sec. 3.1): every weight matrix as equal row blocks, each its own unit
+# ------------------------------------------------------------------------------------------
+
+def _block_scaled(params, wl, nb, seed):
+    """Rescale the row blocks of every weight matrix by different factors, so that a lookup of the
+    wrong block's unit shows."""
+    H, P, R = wl.hidden, wl.proj, wl.R
+    f = rng(seed).choice([0.05, 0.3, 1.0, 4.0], size=nb).astype(np.float32)
+    p = params.copy()
+    off = 0
+
+    def scale(rows, cols):
+        nonlocal off
+        blk = p[off:off + rows * cols].reshape(nb, rows // nb, cols)
+        blk *= f[:, None, None]
+        off += rows * cols
+
+    for l in range(wl.num_layers):
+        for _ in range(4):
+            scale(H, wl.layer_in(l))
+        for _ in range(4):
+            scale(H, R)
+        off += 4 * H
+        if P > 0:
+            scale(P, H)
+    if wl.num_classes > 0:
+        scale(wl.num_classes, R)
+    return p
+
+
+SUB_CASES = [("small", dict(L=2, I=40, H=96, C=12, B=2, T=10), 4), ("layerwise", dict(L=2, I=24, H=48, P=16, C=8, B=9, T=5), 2),
+             ("tc", dict(L=2, I=24, H=64, P=32, C=16, B=70, T=4), 4), ("tc", dict(L=1, I=40, H=96, B=130, T=3), 3),
+             ("layerwise", dict(L=1, I=40, H=12, B=6, T=5), 6)]
+
+
+@pytest.mark.parametrize("path,cfg,nb", SUB_CASES)
+def test_lstm_sub_matrix_units_bit_exact(qnn, path, cfg, nb, monkeypatch):
+    monkeypatch.setenv("QNN_LSTM_PATH", path)
+    wl = _small(**cfg)
+    params, x = wl.make()
+    params = _block_scaled(params, wl, nb, seed=nb)
+    od = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode, nb)
+    ref = oracle.lstm_forward(od, params, x, want_h_all=True)
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode,
+                      weight_blocks=nb)
+    model = qnn.LstmModel(d, gpu(params))
+    B, T, _ = x.shape
+    ha = torch.empty((wl.num_layers, B, T, wl.R), dtype=torch.float32, device="cuda")
+    hs = torch.zeros((wl.num_layers, B, wl.R), dtype=torch.float32, device="cuda")
+    cs = torch.zeros((wl.num_layers, B, wl.hidden), dtype=torch.float32, device="cuda")
+    qnn.profile_read()
+    qnn.profile_enable(True)
+    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha)
+    qnn.profile_enable(False)
+    kernels = qnn.profile_read()
+    want = {"small": "lstm_small", "tc": "lstm_gates_tc", "layerwise": "lstm_recurrent"}[path]
+    assert want in kernels, kernels
+    assert qnn.device_status() == qnn.QNN_OK
+    got = {"y": y.cpu().numpy(), "h": hs.cpu().numpy(), "c": cs.cpu().numpy(), "h_all": ha.cpu().numpy()}
+    _compare(got, ref, wl)
+    codes, prm = model.weights()
+    c_ref, p_ref = oracle.lstm_quantize_weights(od, params)
+    assert np.array_equal(codes, c_ref) and np.array_equal(prm.view(np.int32), p_ref.view(np.int32))
+
+
+def test_sub_matrix_units_must_divide_the_rows(qnn):
+    d = qnn.lstm_desc(1, 8, 12, 0, 0, weight_blocks=5)  # 12 rows per gate matrix do not split in 5
+    assert qnn.qnn_lstm_param_count(d) == -1
+    h = ctypes.c_void_p()
+    params = torch.zeros(qnn.qnn_lstm_param_count(qnn.lstm_desc(1, 8, 12)), device="cuda")
+    assert qnn.lib().qnn_lstm_model_create(ctypes.byref(d), ctypes.c_void_p(params.data_ptr()),
+                                           ctypes.byref(h)) == qnn.QNN_ERR_INVALID_ARG
