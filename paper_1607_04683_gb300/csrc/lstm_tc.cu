@@ -12,6 +12,7 @@
 //   3. with a projection, m_t is quantized the same way and multiplied with Wp' (eq. 1, eq. 3):
 //      r_t is the layer output and the next step's recurrent input.
 // Every step is a few kernel launches in stream order; the stream orders the steps.
+#include <algorithm>
 #include <cfloat>
 #include <cstdlib>
 #include <cstring>
@@ -78,33 +79,22 @@ __global__ void __launch_bounds__(32 * kQuantRowsPerBlock)
     }
 }
 
-// The same for kp <= 2048 with more parallelism per row: a group of G threads (a power of two,
-// 8 G >= kp) per row, each holding 8 consecutive values in registers, so the row is read once.
+// Row-group quantizer shared by the kernels below: a group of G threads (a power of two) holds a
+// row of len values, 8 consecutive values per thread (v, starting at k0 = 8 t); writes the centered
+// fp16 codes [kp] (zero past len), the unit parameters and the code sum of the row (eq. 2).
 template <int G>
-__global__ void __launch_bounds__(256)
-    quantize_rows_f16_kernel(const float *__restrict__ src, int64_t ld, int rows, int len, int kp,
-                             __half *__restrict__ dst, qnn_qparams *__restrict__ prm, int32_t *__restrict__ rsum,
-                             int *status) {
-    constexpr int RPB = 256 / G;                 // rows per block
-    constexpr int W = G > 32 ? G / 32 : 1;       // warps per row
-    __shared__ float s_mn[8], s_mx[8];
-    __shared__ int s_n[8];
-    grid_dependency_wait();
-    grid_dependents_launch();
-    const int t = threadIdx.x % G, rl = threadIdx.x / G, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int r = blockIdx.x * RPB + rl;
-    const bool rv = r < rows;
+__device__ __forceinline__ void quantize_row_group(const float (&v)[8], int len, int kp, int t, int rl, bool rv, int r,
+                                                   __half *__restrict__ dst, qnn_qparams *__restrict__ prm,
+                                                   int32_t *__restrict__ rsum, int *status, float *s_mn, float *s_mx,
+                                                   int *s_n) {
+    constexpr int W = G > 32 ? G / 32 : 1;  // warps per row
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int k0 = 8 * t;
-    const float *xr = src + (int64_t)(rv ? r : 0) * ld;
-    float v[8];
     float mn = FLT_MAX, mx = -FLT_MAX;
     int bad = 0;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-        const int k = k0 + e;
-        const bool in = rv && k < len;
-        v[e] = in ? xr[k] : 0.0f;
-        if (in) {
+        if (rv && k0 + e < len) {
             bad |= !isfinite(v[e]);
             mn = fminf(mn, v[e]);
             mx = fmaxf(mx, v[e]);
@@ -165,6 +155,90 @@ __global__ void __launch_bounds__(256)
     }
 }
 
+// Rows of fp32 values (row r at src + r*ld) -> centered fp16 codes for kp <= 2048: a group of G
+// threads (8 G >= kp) per row, each holding 8 consecutive values, so the row is read once.
+template <int G>
+__global__ void __launch_bounds__(256)
+    quantize_rows_f16_kernel(const float *__restrict__ src, int64_t ld, int rows, int len, int kp,
+                             __half *__restrict__ dst, qnn_qparams *__restrict__ prm, int32_t *__restrict__ rsum,
+                             int *status) {
+    constexpr int RPB = 256 / G;  // rows per block
+    __shared__ float s_mn[8], s_mx[8];
+    __shared__ int s_n[8];
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int t = threadIdx.x % G, rl = threadIdx.x / G;
+    const int r = blockIdx.x * RPB + rl;
+    const bool rv = r < rows;
+    const int k0 = 8 * t;
+    const float *xr = src + (int64_t)(rv ? r : 0) * ld;
+    float v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = (rv && k0 + e < len) ? xr[k0 + e] : 0.0f;
+    quantize_row_group<G>(v, len, kp, t, rl, rv, r, dst, prm, rsum, status, s_mn, s_mx, s_n);
+}
+
+// Arguments of the projection's finishing kernel (one recurrent step of an LSTMP layer).
+struct FinishArgs {
+    const int32_t *part;       // [splits][B][ldpart] split-K partial sums of the centered product
+    int splits;
+    int64_t ldpart;
+    const qnn_qparams *prm_m;  // [B] units of the m_t rows (the product's activations)
+    const int32_t *rs_m;       // [B] their code sums
+    const qnn_qparams *wp_p;   // Wp units, rows_per_unit rows each
+    const int32_t *wp_sum;     // [P] Wp row code sums
+    int rows_per_unit;
+    int K;                     // H, the product's true reduction length
+    float *out;                // r_t: row b at out + b * ldo
+    int64_t ldo;
+    int rows, P;
+    int quantize;              // also quantize r_t for the next step
+    int kp;                    // round_up(P, 64)
+    __half *dst;               // next step's codes [B][kp], params and sums
+    qnn_qparams *prm;
+    int32_t *rsum;
+    int *status;
+};
+
+// Adds the split-K slices, applies eq. (1)'s offsets and eq. (3)'s recovery (the same integer
+// and the same two roundings as the product kernels' epilogues) to give r_t, writes it as the
+// layer output, and quantizes it as the next step's recurrent input.
+template <int G>
+__global__ void __launch_bounds__(256) proj_finish_kernel(const FinishArgs a) {
+    constexpr int RPB = 256 / G;
+    __shared__ float s_mn[8], s_mx[8];
+    __shared__ int s_n[8];
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int t = threadIdx.x % G, rl = threadIdx.x / G;
+    const int r = blockIdx.x * RPB + rl;
+    const bool rv = r < a.rows;
+    const int k0 = 8 * t;
+    float v[8];
+    int za = 0, ra = 0;
+    float Qa = 1.0f;
+    if (rv) {
+        const qnn_qparams pm = a.prm_m[r];
+        za = pm.z, Qa = pm.Q, ra = a.rs_m[r];
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const int n = k0 + e;
+        v[e] = 0.0f;
+        if (rv && n < a.P) {
+            int P = 0;
+            for (int s = 0; s < a.splits; ++s) P += a.part[((int64_t)s * a.rows + r) * a.ldpart + n];
+            const int cs = a.wp_sum[n];
+            const qnn_qparams qw = a.wp_p[n / a.rows_per_unit];
+            const int acc = P + 128 * (ra + cs) - 16384 * a.K;  // raw code product
+            v[e] = recover_product(offset_product(acc, za, qw.z, ra, cs, a.K), Qa, qw.Q);
+            a.out[(int64_t)r * a.ldo + n] = v[e];
+        }
+    }
+    if (!a.quantize) return;
+    quantize_row_group<G>(v, a.P, a.kp, t, rl, rv, r, a.dst, a.prm, a.rsum, a.status, s_mn, s_mx, s_n);
+}
+
 // The four Wh gate matrices (u8 codes, row g*H + j, ld bytes) -> centered fp16 rows in 8-cell
 // groups: row 32*G + 8*g + jj holds gate g of cell 8*G + jj; rows of cells >= H are zero.
 __global__ void interleave_gates_kernel(const uint8_t *__restrict__ codes, int64_t ld, int H, int K, int kp,
@@ -216,6 +290,41 @@ qnn_status launch_quantize_rows_f16(const float *src, int64_t ld, int64_t rows, 
     }
     QNN_CUDA_TRY(e);
     return QNN_OK;
+}
+
+// Launches the projection's finishing kernel (P <= 2048 values per row); with `pdl` as a
+// programmatic dependent launch.
+qnn_status launch_proj_finish(const FinishArgs &fa, bool pdl, cudaStream_t st) {
+    ProfScope prof("proj_finish", st);
+    int g = 8;
+    while (g * 8 < fa.P) g *= 2;
+    cudaLaunchConfig_t cfg = {};
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    auto grid_for = [&](int rpb) { return dim3((unsigned)((fa.rows + rpb - 1) / rpb)); };
+    cudaError_t e;
+    switch (g) {
+        case 8: cfg.gridDim = grid_for(32); e = cudaLaunchKernelEx(&cfg, proj_finish_kernel<8>, fa); break;
+        case 16: cfg.gridDim = grid_for(16); e = cudaLaunchKernelEx(&cfg, proj_finish_kernel<16>, fa); break;
+        case 32: cfg.gridDim = grid_for(8); e = cudaLaunchKernelEx(&cfg, proj_finish_kernel<32>, fa); break;
+        case 64: cfg.gridDim = grid_for(4); e = cudaLaunchKernelEx(&cfg, proj_finish_kernel<64>, fa); break;
+        case 128: cfg.gridDim = grid_for(2); e = cudaLaunchKernelEx(&cfg, proj_finish_kernel<128>, fa); break;
+        case 256: cfg.gridDim = grid_for(1); e = cudaLaunchKernelEx(&cfg, proj_finish_kernel<256>, fa); break;
+        default: return QNN_ERR_INVALID_ARG;
+    }
+    QNN_CUDA_TRY(e);
+    return QNN_OK;
+}
+
+// Split-K slices of the projection (see tc_partial): at most this many, so the workspace is bounded.
+int64_t max_proj_splits(const qnn_lstm_model *m) {
+    const int64_t kb = round_up(m->H, 64) / 64;
+    return std::max<int64_t>((kb + 15) / 16, 8);
 }
 
 // Programmatic dependent launches between the recurrence's kernels (QNN_PDL=0 turns them off).
@@ -277,8 +386,10 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
 
 size_t tc_work_bytes(const qnn_lstm_model *m, int64_t B) {
     const int64_t kh = round_up(m->R, 64), kpj = m->P > 0 ? round_up(m->H, 64) : 0;
+    const int64_t part = m->P > 0 ? max_proj_splits(m) * B * m->P * 4 : 0;
     return (size_t)round_up(B * kh * 2, 256) + (size_t)round_up(B * kpj * 2, 256) +
-           2 * (size_t)round_up(B * (int64_t)sizeof(qnn_qparams), 256) + 2 * (size_t)round_up(B * 4, 256);
+           2 * (size_t)round_up(B * (int64_t)sizeof(qnn_qparams), 256) + 2 * (size_t)round_up(B * 4, 256) +
+           (size_t)round_up(part, 256);
 }
 
 qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
@@ -299,27 +410,43 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     int32_t *rs = reinterpret_cast<int32_t *>(w);
     w += round_up(B * 4, 256);
     int32_t *rs_m = reinterpret_cast<int32_t *>(w);
+    w += round_up(B * 4, 256);
+    int32_t *part = reinterpret_cast<int32_t *>(w);
 
     int *status = nullptr;
     QNN_TRY(status_word(&status));
     TcOperands gates, proj;
     static const int gate_bn[] = {128, 64, 32};
     QNN_TRY(tc_operands(&gates, a16, B, tl.wh16, 4 * H8, kh, tc_choose_bn(B, 4 * H8, gate_bn, 3)));
-    if (P > 0) QNN_TRY(tc_operands(&proj, m16, B, tl.wp16, P, kpj, tc_pick_bn(B, P, kpj)));
+    // the projection: split-K partial sums, finished (offsets, recovery, next step's quantization)
+    // by one row kernel when P <= 2048; else one tcgen05 product with its own epilogue per step
+    const bool split_proj = P > 0 && P <= 2048;
+    int splits = 0;
+    if (P > 0) {
+        QNN_TRY(tc_operands(&proj, m16, B, tl.wp16, P, kpj, split_proj ? 128 : tc_pick_bn(B, P, kpj)));
+        if (split_proj) splits = tc_partial_splits(proj, (int)max_proj_splits(m));
+    }
     // the steps' kernels chain by programmatic dependent launches (see tc_gemm.h); the first one of
     // the layer follows ordinary stream order
     gates.pdl = proj.pdl = pdl_enabled();
+    QNN_TRY(launch_quantize_rows_f16(h0, R, B, R, kh, a16, prm, rs, status, false, st));
     for (int64_t t = 0; t < T; ++t) {
-        const float *src = t == 0 ? h0 : out + (t - 1) * R;
-        const int64_t ld = t == 0 ? R : T * R;
-        QNN_TRY(launch_quantize_rows_f16(src, ld, B, R, kh, a16, prm, rs, status, t > 0 && gates.pdl, st));
+        if (t > 0 && !split_proj)
+            QNN_TRY(launch_quantize_rows_f16(out + (t - 1) * R, T * R, B, R, kh, a16, prm, rs, status, gates.pdl, st));
         TcLstmOut o{px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R, (int)H,
                     (int)m->S, (int)(H / m->S)};
         QNN_TRY(tc_lstm_gates(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, st));
         if (P > 0) {
             QNN_TRY(launch_quantize_rows_f16(mbuf, H, B, H, kpj, m16, prm_m, rs_m, status, gates.pdl, st));
-            QNN_TRY(tc_linear(proj, prm_m, 1, rs_m, H, ly.wp.params, P / m->S, ly.wp.sums, nullptr, out + t * R,
-                              T * R, nullptr, st));
+            if (split_proj) {
+                QNN_TRY(tc_partial(proj, splits, part, P, st));
+                FinishArgs fa{part, splits, P, prm_m, rs_m, ly.wp.params, ly.wp.sums, (int)(P / m->S), (int)H,
+                              out + t * R, T * R, (int)B, (int)P, t + 1 < T, (int)kh, a16, prm, rs, status};
+                QNN_TRY(launch_proj_finish(fa, gates.pdl, st));
+            } else {
+                QNN_TRY(tc_linear(proj, prm_m, 1, rs_m, H, ly.wp.params, P / m->S, ly.wp.sums, nullptr, out + t * R,
+                                  T * R, nullptr, st));
+            }
         }
     }
     return QNN_OK;

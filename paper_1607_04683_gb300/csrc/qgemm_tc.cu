@@ -42,7 +42,9 @@ constexpr unsigned long long TC_WAIT_NS = 2000000000ull;
 // kEpiLstm: the LSTM cell update on gate-interleaved columns, K <= 1024; kEpiLstmEarly the same
 // with the accumulator-independent loads issued before the accumulator wait (a block with a single
 // tile has no earlier epilogue to overlap them with).
-enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiLstmEarly = 3 };
+// kEpiPartial: split-K, each work item (tile, K range of at most 1024) stores its exact centered
+// integer sums P as int32 into its own slice of a partial-sum buffer; a consumer adds the slices.
+enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiLstmEarly = 3, kEpiPartial = 4 };
 
 struct ColConst {  // per-output-column constants of kEpiRow, staged in shared memory per tile
     int cs, zw;
@@ -68,7 +70,7 @@ struct Tile {
     static constexpr int STAGES = EPI == kEpiLinear ? (BN == 256 ? 4 : 6) : (BN == 128 ? 4 : 6);
     static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : 96;
-    static constexpr int EPI_BYTES = EPI == kEpiLstm || EPI == kEpiLstmEarly
+    static constexpr int EPI_BYTES = EPI == kEpiLstm || EPI == kEpiLstmEarly || EPI == kEpiPartial
                                          ? 0
                                          : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
     static constexpr uint32_t IDESC =
@@ -92,6 +94,10 @@ struct TcArgs {
     int KB;     // k-blocks of 64
     int *status;
     TcLstmOut lstm;  // kEpiLstm only
+    int splits;      // K ranges per tile (kEpiPartial; 1 otherwise)
+    int kbs;         // k-blocks per K range
+    int32_t *part;   // kEpiPartial: [splits][M][ldpart] int32
+    int64_t ldpart;
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
@@ -232,6 +238,9 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     const int tiles_n = (int)((args.N + BN - 1) / BN);
     const int64_t tiles_m = (args.M + TBM - 1) / TBM;
     const int64_t tiles = tiles_m * tiles_n;
+    // work items: (tile, K range); one K range per tile except for split-K
+    const int splits = args.splits;
+    const int64_t items = tiles * splits;
     __shared__ int s_abort;
 
     if (threadIdx.x == 0) {
@@ -269,10 +278,11 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         // ---------------- TMA producer ----------------
         if (lane == 0) {
             int64_t g = 0;  // k-blocks issued by this block
-            for (int64_t tile = blockIdx.x; tile < tiles && !s_abort; tile += gridDim.x) {
+            for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
                 int64_t m0, n0;
-                tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
-                for (int kb = 0; kb < KB; ++kb, ++g) {
+                tile_origin(item / splits, tiles_m, tiles_n, BN, m0, n0);
+                const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                for (int kb = kb0; kb < kb1; ++kb, ++g) {
                     const int s = (int)(g % STAGES);
                     if (g >= STAGES && !mb_wait(empty0 + 8 * s, (unsigned)((g / STAGES) - 1) & 1, args.status)) {
                         s_abort = 1;
@@ -289,10 +299,11 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
             int64_t g = 0, gc = 0;  // k-blocks and chunks consumed by this block
-            for (int64_t tile = blockIdx.x; tile < tiles && !s_abort; tile += gridDim.x) {
-                for (int kb = 0; kb < KB; ++kb, ++g) {
+            for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
+                const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                for (int kb = kb0; kb < kb1; ++kb, ++g) {
                     const int s = (int)(g % STAGES);
-                    const int kc = kb % kpc;
+                    const int kc = (kb - kb0) % kpc;
                     const int buf = (int)(gc & 1);
                     if (kc == 0 && gc >= 2 &&
                         !mb_wait(drained0 + 8 * buf, (unsigned)((gc / 2) - 1) & 1, args.status)) {  // buffer free
@@ -313,7 +324,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                                            (kc == 0 && k == 0) ? 0u : 1u);
                     }
                     mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
-                    if (kc == kpc - 1 || kb == KB - 1) {
+                    if (kc == kpc - 1 || kb == kb1 - 1) {
                         mma_commit(chunk0 + 8 * buf);
                         ++gc;
                     }
@@ -532,6 +543,49 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
             ++gc;
         }
+    } else if constexpr (EPI == kEpiPartial) {
+        // ---------------- epilogue (warps 2..17): split-K partial sums ----------------
+        // The item's K range is at most one accumulation chunk, so its fp32 accumulator holds the
+        // exact integer sum of centered products; each lane stores its row's 16-column blocks.
+        const int q = warp & 3;
+        const int part = (warp - 2) >> 2;
+        int64_t gc = 0;
+        bool ok = true;
+        const bool vec = args.ldpart % 4 == 0;
+        for (int64_t item = blockIdx.x; item < items && ok; item += gridDim.x, ++gc) {
+            int64_t m0, n0;
+            tile_origin(item / splits, tiles_m, tiles_n, BN, m0, n0);
+            int32_t *dst = args.part + (item % splits) * args.M * args.ldpart;
+            const int64_t m = m0 + 32 * q + lane;
+            const int buf = (int)(gc & 1);
+            ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll 1
+            for (int j = part; j < BN / 16; j += TL::EPI_WARPS / 4) {
+                uint32_t r[16];
+                tmem_ld16(tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + 16 * j), r);
+                const int64_t nb = n0 + 16 * j;
+                if (m >= args.M || nb >= args.N) continue;
+                int32_t *o = dst + m * args.ldpart + nb;
+                if (vec && nb + 16 <= args.N) {
+#pragma unroll
+                    for (int v4 = 0; v4 < 4; ++v4)
+                        *reinterpret_cast<int4 *>(o + 4 * v4) =
+                            make_int4(f32_integer_to_s32(__uint_as_float(r[4 * v4])),
+                                      f32_integer_to_s32(__uint_as_float(r[4 * v4 + 1])),
+                                      f32_integer_to_s32(__uint_as_float(r[4 * v4 + 2])),
+                                      f32_integer_to_s32(__uint_as_float(r[4 * v4 + 3])));
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i)
+                        if (nb + i < args.N) o[i] = f32_integer_to_s32(__uint_as_float(r[i]));
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+        }
     } else {
         // ---------------- epilogue (warps 2..17): LSTM cell update ----------------
         // Column n of the tile is gate g = (n % 32) / 8 of cell 8 * (n / 32) + n % 8. Each lane owns
@@ -721,9 +775,9 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
                          "%d blocks per SM\n", BN, EPI, TL::THREADS, fa.numRegs, TL::SMEM, n);
         }
     }
-    const int64_t tiles = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN);
+    const int64_t items = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN) * a.splits;
     // persistent: one block per SM (a block holding tensor memory has its SM to itself)
-    const unsigned grid = (unsigned)std::min<int64_t>(tiles, (int64_t)sm_count());
+    const unsigned grid = (unsigned)std::min<int64_t>(items, (int64_t)sm_count());
     ProfScope prof(name, st);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -827,7 +881,7 @@ qnn_status tc_linear(const TcOperands &op, const qnn_qparams *pa, int per_row, c
     int *status = nullptr;
     QNN_TRY(status_word(&status));
     TcArgs a{pa, per_row, rsA, pw, rows_per_block, csW, bias, Y, ldy, acc_out, op.M, op.N, (int)K,
-             (int)(op.kp / TBK), status, TcLstmOut{}};
+             (int)(op.kp / TBK), status, TcLstmOut{}, 1, (int)(op.kp / TBK), nullptr, 0};
     return dispatch_linear(op, a, st);
 }
 
@@ -838,8 +892,32 @@ qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int3
     if (op.N != 4 * ((out.H + 7) / 8 * 8)) return QNN_ERR_INVALID_ARG;
     int *status = nullptr;
     QNN_TRY(status_word(&status));
-    TcArgs a{pa, 1, rsA, pw4, 0, cs, nullptr, nullptr, 0, nullptr, op.M, op.N, (int)K, (int)(op.kp / TBK), status, out};
+    TcArgs a{pa, 1, rsA, pw4, 0, cs, nullptr, nullptr, 0, nullptr, op.M, op.N, (int)K, (int)(op.kp / TBK), status, out,
+             1, (int)(op.kp / TBK), nullptr, 0};
     return dispatch_lstm(op, a, st);
+}
+
+int tc_partial_splits(const TcOperands &op, int max_splits) {
+    const int KB = (int)(op.kp / TBK), kpc = KCHUNK / TBK;
+    const int64_t tiles = ((op.M + TBM - 1) / TBM) * ((op.N + op.bn - 1) / op.bn);
+    // as many K ranges as keep the work items within one wave, but at least one exact chunk each
+    int splits = (int)std::max<int64_t>((KB + kpc - 1) / kpc, sm_count() / tiles);
+    splits = std::max(1, std::min({splits, KB, std::max(max_splits, (KB + kpc - 1) / kpc)}));
+    const int kbs = (KB + splits - 1) / splits;  // equal ranges (the last one shorter)
+    return (KB + kbs - 1) / kbs;
+}
+
+qnn_status tc_partial(const TcOperands &op, int splits, int32_t *part, int64_t ldpart, cudaStream_t st) {
+    const int KB = (int)(op.kp / TBK);
+    if (splits < 1 || splits > KB || (op.bn != 64 && op.bn != 128) || ldpart < op.N) return QNN_ERR_INVALID_ARG;
+    const int kbs = (KB + splits - 1) / splits;
+    if (kbs > KCHUNK / TBK || (KB + kbs - 1) / kbs != splits) return QNN_ERR_INVALID_ARG;  // one exact chunk each
+    int *status = nullptr;
+    QNN_TRY(status_word(&status));
+    TcArgs a{nullptr, 0, nullptr, nullptr, 0, nullptr, nullptr, nullptr, 0, nullptr, op.M, op.N, 0, KB, status,
+             TcLstmOut{}, splits, kbs, part, ldpart};
+    return op.bn == 64 ? launch_tc<64, kEpiPartial>(op, a, "qgemm_tc_partial", st)
+                       : launch_tc<128, kEpiPartial>(op, a, "qgemm_tc_partial", st);
 }
 
 qnn_status launch_center_fp16(const uint8_t *in, int64_t rows, int64_t K, int64_t ldi, __half *out, int64_t ldo,

@@ -59,6 +59,14 @@ struct TcLstmOut {
 qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int32_t *rsA, int64_t K,
                          const qnn_qparams *pw4, const int32_t *cs, const TcLstmOut &out, cudaStream_t st);
 
+// Split-K partial sums of the centered integer product: part[s][m][n] = sum over K range s of
+// (a - 128)(w - 128), int32, ranges of at most 1024 so that each is exact in one accumulator;
+// the slices add up to P = acc - 128 (rsA + csW) + 128^2 K. ldpart >= N (elements).
+// K ranges giving at most one wave of work items (each range one exact chunk; at most
+// max(max_splits, the chunks K needs) ranges).
+int tc_partial_splits(const TcOperands &op, int max_splits);
+qnn_status tc_partial(const TcOperands &op, int splits, int32_t *part, int64_t ldpart, cudaStream_t st);
+
 // u8 codes [rows][ldi] -> centered fp16 [rows][ldo], zero past K.
 qnn_status launch_center_fp16(const uint8_t *in, int64_t rows, int64_t K, int64_t ldi, __half *out, int64_t ldo,
                               cudaStream_t st);
