@@ -213,6 +213,26 @@ __device__ __forceinline__ void tile_origin(int64_t tile, int64_t tiles_m, int t
     n0 = (local / rows) * bn;
 }
 
+// Recovered outputs of one 16-column block of one row that lies in one weight unit (the row
+// terms rt, za + 128 and the divisor Qa Qw hoisted), stored as four 16-byte vectors.
+template <bool BIAS>
+__device__ __forceinline__ void row_block_fast(const uint32_t (&r)[16], const ColConst *cc, long long rt, int za128,
+                                               float den, float *yr) {
+#pragma unroll
+    for (int v4 = 0; v4 < 4; ++v4) {
+        float y[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int i = 4 * v4 + e;
+            const long long S = (long long)f32_integer_to_s32(__uint_as_float(r[i])) + rt + (long long)za128 * cc[i].cs;
+            const float x = s64_to_f32_rn(S);
+            y[e] = __fdiv_rn(x, den);
+            if (BIAS) y[e] = __fadd_rn(y[e], cc[i].bias);
+        }
+        *reinterpret_cast<float4 *>(yr + 4 * v4) = make_float4(y[0], y[1], y[2], y[3]);
+    }
+}
+
 // Persistent tile loop. Warp 0: TMA producer; warp 1: tensor-memory owner and MMA issuer; warps
 // 2.. : epilogue. EPI = kEpiLinear / kEpiRow write the recovered product (plus bias) and
 // optionally the raw int32 accumulator; EPI = kEpiLstm treats the columns as gate-interleaved LSTM
@@ -506,6 +526,13 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 }
                 float *yr = args.Y ? args.Y + m * args.ldy + nb : nullptr;
                 const bool full = vec && nb + 16 <= args.N;
+                if (one_unit && full && !args.acc_out) {  // the usual block: no per-element branches
+                    if (args.bias)
+                        row_block_fast<true>(r, cc + c0, rt, za128, den, yr);
+                    else
+                        row_block_fast<false>(r, cc + c0, rt, za128, den, yr);
+                    continue;
+                }
 #pragma unroll
                 for (int v4 = 0; v4 < 4; ++v4) {
                     float y[4];
@@ -647,6 +674,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         const qnn_qparams qw = args.pw[g * E.ups + unit];
                         rt[g] = (long long)(128 + qw.z) * rs + (long long)K * ((long long)za * qw.z - 16384);
                         den[g] = __fmul_rn(Qa, qw.Q);
+
                     }
                     const float *pxr = E.px + b * E.px_ld + j0;
                     float *cr = E.c + b * (int64_t)H + j0;
@@ -661,7 +689,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         for (int jj = 0; jj < 4; ++jj) {
                             const long long S = (long long)f32_integer_to_s32(__uint_as_float(r[g][jj])) + rt[g] +
                                                 (long long)za128 * csv[jj];
-                            pre[g][jj] = __fadd_rn(pv[jj], __fdiv_rn(s64_to_f32_rn(S), den[g]));
+                            const float xs = s64_to_f32_rn(S);
+                            pre[g][jj] = __fadd_rn(pv[jj], __fdiv_rn(xs, den[g]));
                         }
                     }
                     const float4 c4 = s == s0 ? c0v : *reinterpret_cast<const float4 *>(cr);
