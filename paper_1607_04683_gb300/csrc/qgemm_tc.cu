@@ -63,13 +63,19 @@ struct ColUnit {  // and the weight unit of each column (-1 past N)
 template <int BN, int EPI>
 struct Tile {
     static_assert(EPI == kEpiLinear || BN <= 128, "row and LSTM epilogues take tiles of at most 128 columns");
-    static constexpr int EPI_WARPS = EPI == kEpiLinear ? 8 : 16;
+    // a 96-column LSTM tile has six 4-cell slices per lane quarter: 24 epilogue warps, one slice each
+    static constexpr bool LSTM96 = (EPI == kEpiLstm || EPI == kEpiLstmEarly) && BN == 96;
+    static constexpr int EPI_WARPS = EPI == kEpiLinear ? 8 : (LSTM96 ? 24 : 16);
+    // LSTM: cells per epilogue slice (a 32-column tile has 8 cells: 2-cell slices keep 4 warps busy)
+    static constexpr int CPS = BN == 32 ? 2 : 4;
     static constexpr int THREADS = 32 * (2 + EPI_WARPS);
     static constexpr int B_BYTES = BN * TBK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGES = EPI == kEpiLinear ? (BN == 256 ? 4 : 6) : (BN == 128 ? 4 : 6);
-    static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
-    static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : 96;
+    static constexpr int TMEM_COLS = 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
+    // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
+    // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
+    static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : (LSTM96 ? 72 : 96);
     static constexpr int EPI_BYTES = EPI == kEpiLstm || EPI == kEpiLstmEarly || EPI == kEpiPartial
                                          ? 0
                                          : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
@@ -193,8 +199,36 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         : "r"(taddr));
     tmem_wait_ld();
 }
+// 2 consecutive fp32 columns, without the wait.
+__device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[2]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(taddr));
+}
+// Vector loads and stores of 2 or 4 consecutive (8- or 16-byte aligned) values.
+__device__ __forceinline__ void ld_vec(const float *p, float (&v)[4]) {
+    const float4 a = *reinterpret_cast<const float4 *>(p);
+    v[0] = a.x, v[1] = a.y, v[2] = a.z, v[3] = a.w;
+}
+__device__ __forceinline__ void ld_vec(const float *p, float (&v)[2]) {
+    const float2 a = *reinterpret_cast<const float2 *>(p);
+    v[0] = a.x, v[1] = a.y;
+}
+__device__ __forceinline__ void ld_vec(const int *p, int (&v)[4]) {
+    const int4 a = *reinterpret_cast<const int4 *>(p);
+    v[0] = a.x, v[1] = a.y, v[2] = a.z, v[3] = a.w;
+}
+__device__ __forceinline__ void ld_vec(const int *p, int (&v)[2]) {
+    const int2 a = *reinterpret_cast<const int2 *>(p);
+    v[0] = a.x, v[1] = a.y;
+}
+__device__ __forceinline__ void st_vec(float *p, const float (&v)[4]) {
+    *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+}
+__device__ __forceinline__ void st_vec(float *p, const float (&v)[2]) {
+    *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+}
+
 // 4 consecutive fp32 columns, without the wait (the caller waits once for several loads).
-__device__ __forceinline__ void tmem_ld4_nowait(uint32_t taddr, uint32_t (&r)[4]) {
+__device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[4]) {
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                  : "r"(taddr));
@@ -614,11 +648,14 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
         }
     } else {
-        // ---------------- epilogue (warps 2..17): LSTM cell update ----------------
+        // ---------------- epilogue: LSTM cell update ----------------
         // Column n of the tile is gate g = (n % 32) / 8 of cell 8 * (n / 32) + n % 8. Each lane owns
-        // one batch row; the four warps of a lane quarter take 4-cell slices in turn, reading the
+        // one batch row; the warps of a lane quarter take slices of CPS cells in turn, reading the
         // four gates of their cells from tensor memory, so a thread has everything for eq. (1)/(3)
-        // and the cell update of 4 cells.
+        // and the cell update of CPS cells.
+        constexpr int CPS = TL::CPS;
+        constexpr int SLICES = BN / (4 * CPS);   // slices per tile
+        constexpr int SPG = 8 / CPS;             // slices per 8-cell group
         const int q = warp & 3;
         const int eh = (warp - 2) >> 2;
         const int K = args.K;
@@ -644,24 +681,24 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             // this warp's first slice: the input products and cell state do not depend on the
             // accumulator, so they may be loaded before waiting for it
             const int s0 = EPI == kEpiLstmEarly ? eh : -1;
-            float4 px0[4], c0v = make_float4(0.f, 0.f, 0.f, 0.f);
-            const int j00 = (int)(n0 / 4) + (eh >> 1) * 8 + (eh & 1) * 4;
-            if (EPI == kEpiLstmEarly && eh < BN / 16 && bv && j00 < H) {
+            float px0[4][CPS], c0v[CPS];
+            const int j00 = (int)(n0 / 4) + (eh / SPG) * 8 + (eh % SPG) * CPS;
+            if (EPI == kEpiLstmEarly && eh < SLICES && bv && j00 < H) {
 #pragma unroll
-                for (int g = 0; g < 4; ++g) px0[g] = *reinterpret_cast<const float4 *>(E.px + b * E.px_ld + j00 + (int64_t)g * H);
-                c0v = *reinterpret_cast<const float4 *>(E.c + b * (int64_t)H + j00);
+                for (int g = 0; g < 4; ++g) ld_vec(E.px + b * E.px_ld + j00 + (int64_t)g * H, px0[g]);
+                ld_vec(E.c + b * (int64_t)H + j00, c0v);
             }
             ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll 1
-            for (int s = eh; s < BN / 16; s += TL::EPI_WARPS / 4) {
-                const int gi = s >> 1, part = s & 1;
-                const int j0 = (int)(n0 / 4) + gi * 8 + part * 4;  // H is a multiple of 4: all 4 valid or none
-                uint32_t r[4][4];
-                const uint32_t ta = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + gi * 32 + part * 4);
+            for (int s = eh; s < SLICES; s += TL::EPI_WARPS / 4) {
+                const int gi = s / SPG, part = s % SPG;
+                const int j0 = (int)(n0 / 4) + gi * 8 + part * CPS;  // H is a multiple of 4: all CPS valid or none
+                uint32_t r[4][CPS];
+                const uint32_t ta = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + gi * 32 + part * CPS);
 #pragma unroll
-                for (int g = 0; g < 4; ++g) tmem_ld4_nowait(ta + 8 * g, r[g]);
+                for (int g = 0; g < 4; ++g) tmem_ld_nowait(ta + 8 * g, r[g]);
                 tmem_wait_ld();
                 if (bv && j0 < H) {
                     // eq. (1) expanded around the centered product P: S = P + rt[g] + (128 + za) csW,
@@ -674,31 +711,39 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         const qnn_qparams qw = args.pw[g * E.ups + unit];
                         rt[g] = (long long)(128 + qw.z) * rs + (long long)K * ((long long)za * qw.z - 16384);
                         den[g] = __fmul_rn(Qa, qw.Q);
-
                     }
                     const float *pxr = E.px + b * E.px_ld + j0;
                     float *cr = E.c + b * (int64_t)H + j0;
-                    float pre[4][4];
+                    float pre[4][CPS];
 #pragma unroll
                     for (int g = 0; g < 4; ++g) {
-                        const float4 v = s == s0 ? px0[g] : *reinterpret_cast<const float4 *>(pxr + (int64_t)g * H);
-                        const int4 cs = *reinterpret_cast<const int4 *>(args.csW + g * H + j0);
-                        const int csv[4] = {cs.x, cs.y, cs.z, cs.w};
-                        const float pv[4] = {v.x, v.y, v.z, v.w};
+                        float pv[CPS];
+                        int csv[CPS];
+                        if (s == s0) {
 #pragma unroll
-                        for (int jj = 0; jj < 4; ++jj) {
+                            for (int jj = 0; jj < CPS; ++jj) pv[jj] = px0[g][jj];
+                        } else {
+                            ld_vec(pxr + (int64_t)g * H, pv);
+                        }
+                        ld_vec(args.csW + g * H + j0, csv);
+#pragma unroll
+                        for (int jj = 0; jj < CPS; ++jj) {
                             const long long S = (long long)f32_integer_to_s32(__uint_as_float(r[g][jj])) + rt[g] +
                                                 (long long)za128 * csv[jj];
-                            const float xs = s64_to_f32_rn(S);
-                            pre[g][jj] = __fadd_rn(pv[jj], __fdiv_rn(xs, den[g]));
+                            pre[g][jj] = __fadd_rn(pv[jj], __fdiv_rn(s64_to_f32_rn(S), den[g]));
                         }
                     }
-                    const float4 c4 = s == s0 ? c0v : *reinterpret_cast<const float4 *>(cr);
-                    float cv[4] = {c4.x, c4.y, c4.z, c4.w}, mv[4];
+                    float cv[CPS], mv[CPS];
+                    if (s == s0) {
 #pragma unroll
-                    for (int jj = 0; jj < 4; ++jj) lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
-                    *reinterpret_cast<float4 *>(cr) = make_float4(cv[0], cv[1], cv[2], cv[3]);
-                    *reinterpret_cast<float4 *>(E.h + b * E.h_ld + j0) = make_float4(mv[0], mv[1], mv[2], mv[3]);
+                        for (int jj = 0; jj < CPS; ++jj) cv[jj] = c0v[jj];
+                    } else {
+                        ld_vec(cr, cv);
+                    }
+#pragma unroll
+                    for (int jj = 0; jj < CPS; ++jj) lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
+                    st_vec(cr, cv);
+                    st_vec(E.h + b * E.h_ld + j0, mv);
                 }
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -844,6 +889,7 @@ qnn_status dispatch_lstm(const TcOperands &op, const TcArgs &a, cudaStream_t st)
         switch (op.bn) {
             case 32: return launch_tc<32, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
             case 64: return launch_tc<64, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
+            case 96: return launch_tc<96, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
             case 128: return launch_tc<128, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
             default: return QNN_ERR_INVALID_ARG;
         }
@@ -851,6 +897,7 @@ qnn_status dispatch_lstm(const TcOperands &op, const TcArgs &a, cudaStream_t st)
     switch (op.bn) {
         case 32: return launch_tc<32, kEpiLstm>(op, a, "lstm_gates_tc", st);
         case 64: return launch_tc<64, kEpiLstm>(op, a, "lstm_gates_tc", st);
+        case 96: return launch_tc<96, kEpiLstm>(op, a, "lstm_gates_tc", st);
         case 128: return launch_tc<128, kEpiLstm>(op, a, "lstm_gates_tc", st);
         default: return QNN_ERR_INVALID_ARG;
     }
@@ -894,7 +941,7 @@ int tc_pick_bn(int64_t M, int64_t N, int64_t kp) {
 }
 
 qnn_status tc_operands(TcOperands *op, const __half *A16, int64_t M, const __half *W16, int64_t N, int64_t kp, int bn) {
-    if (bn != 32 && bn != 64 && bn != 128 && bn != 256) return QNN_ERR_INVALID_ARG;
+    if (bn != 32 && bn != 64 && bn != 96 && bn != 128 && bn != 256) return QNN_ERR_INVALID_ARG;
     if (kp <= 0 || kp % TBK != 0 || M <= 0 || N <= 0) return QNN_ERR_INVALID_ARG;
     QNN_TRY(make_map(&op->a, A16, M, kp, TBM));
     QNN_TRY(make_map(&op->w, W16, N, kp, bn));

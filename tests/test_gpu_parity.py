@@ -365,7 +365,7 @@ TC_CASES = [dict(L=1, I=40, H=128, B=5, T=6), dict(L=2, I=40, H=100, C=37, B=130
             dict(L=3, I=5, H=8, B=3, T=4, mu=0.5), dict(L=1, I=40, H=800, B=300, T=2, w=0.05)]
 
 
-@pytest.mark.parametrize("bn", ["32", "64", "128"])
+@pytest.mark.parametrize("bn", ["32", "64", "96", "128"])
 @pytest.mark.parametrize("cfg", TC_CASES)
 def test_tc_recurrence_bit_exact(qnn, cfg, bn, monkeypatch):
     wl = _small(**cfg)
