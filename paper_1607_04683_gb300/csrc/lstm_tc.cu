@@ -221,16 +221,30 @@ __global__ void __launch_bounds__(256) proj_finish_kernel(const FinishArgs a) {
         const qnn_qparams pm = a.prm_m[r];
         za = pm.z, Qa = pm.Q, ra = a.rs_m[r];
     }
+    // the exact centered sums of this thread's 8 outputs: slices added in int32 (16-byte loads when
+    // the row of 8 lies inside P and the slices are 16-byte aligned)
+    int Psum[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    if (rv && k0 + 8 <= a.P && a.ldpart % 4 == 0) {
+        for (int s = 0; s < a.splits; ++s) {
+            const int4 *src = reinterpret_cast<const int4 *>(a.part + ((int64_t)s * a.rows + r) * a.ldpart + k0);
+            const int4 u = src[0], w = src[1];
+            Psum[0] += u.x, Psum[1] += u.y, Psum[2] += u.z, Psum[3] += u.w;
+            Psum[4] += w.x, Psum[5] += w.y, Psum[6] += w.z, Psum[7] += w.w;
+        }
+    } else if (rv) {
+        for (int s = 0; s < a.splits; ++s)
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                if (k0 + e < a.P) Psum[e] += a.part[((int64_t)s * a.rows + r) * a.ldpart + k0 + e];
+    }
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
         const int n = k0 + e;
         v[e] = 0.0f;
         if (rv && n < a.P) {
-            int P = 0;
-            for (int s = 0; s < a.splits; ++s) P += a.part[((int64_t)s * a.rows + r) * a.ldpart + n];
             const int cs = a.wp_sum[n];
             const qnn_qparams qw = a.wp_p[n / a.rows_per_unit];
-            const int acc = P + 128 * (ra + cs) - 16384 * a.K;  // raw code product
+            const int acc = Psum[e] + 128 * (ra + cs) - 16384 * a.K;  // raw code product
             v[e] = recover_product(offset_product(acc, za, qw.z, ra, cs, a.K), Qa, qw.Q);
             a.out[(int64_t)r * a.ldo + n] = v[e];
         }

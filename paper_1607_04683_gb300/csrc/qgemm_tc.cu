@@ -71,7 +71,9 @@ struct Tile {
     static constexpr int THREADS = 32 * (2 + EPI_WARPS);
     static constexpr int B_BYTES = BN * TBK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = EPI == kEpiLinear ? (BN == 256 ? 4 : 6) : (BN == 128 ? 4 : 6);
+    static constexpr int STAGES = EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
+                                  : EPI == kEpiPartial ? 6  // one K range per item: keep it all in flight
+                                                       : (BN == 128 ? 4 : 6);
     static constexpr int TMEM_COLS = 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
     // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
