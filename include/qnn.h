@@ -238,6 +238,13 @@ qnn_status qnn_measure_peak(int kind, double *tops);
  * QNN_ERR_INVALID_ARG for n < 0 or null/host pointers with n > 0. Asynchronous on `stream`. */
 qnn_status qnn_selftest_s64_to_f32(const int64_t *in, float *out, int64_t n, void *stream);
 
+/* Diagnostic (no counterpart in the paper): runs one warp that waits, through the bounded wait of
+ * the tensor-core kernels, on a barrier nothing completes, for limit_ns (1 us .. 1 s). The wait
+ * gives up and records QNN_ERR_TIMEOUT in the device status word (read it with qnn_device_status);
+ * the context stays usable. Synchronous on `stream`. Returns QNN_OK when the wait gave up as
+ * designed, QNN_ERR_INVALID_ARG for a limit out of range. */
+qnn_status qnn_selftest_wait_timeout(int64_t limit_ns, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

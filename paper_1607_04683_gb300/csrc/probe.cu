@@ -50,6 +50,19 @@ __global__ void __launch_bounds__(256) dp4a_peak_kernel(int iters, int *sink) {
     if (s == 0x7fffffff) sink[0] = s;
 }
 
+// A wait nothing ends: one warp waits on an mbarrier that no thread arrives at, through the same
+// bounded wait the tensor-core kernels use, with a short limit.
+__global__ void wait_timeout_kernel(int *status, unsigned long long limit_ns, int *result) {
+    __shared__ __align__(8) unsigned long long bar;
+    const uint32_t b = static_cast<uint32_t>(__cvta_generic_to_shared(&bar));
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(b) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncwarp();
+    const bool completed = mbar_wait_bounded(b, 0, status, limit_ns);
+    if (threadIdx.x == 0) *result = completed ? 1 : 2;
+}
 }  // namespace
 }  // namespace qnn
 
@@ -107,4 +120,20 @@ extern "C" qnn_status qnn_selftest_s64_to_f32(const int64_t *in, float *out, int
     qnn::s64_to_f32_kernel<<<blocks, 256, 0, qnn::as_stream(stream)>>>(in, out, n);
     QNN_CUDA_TRY(cudaGetLastError());
     return QNN_OK;
+}
+
+extern "C" qnn_status qnn_selftest_wait_timeout(int64_t limit_ns, void *stream) {
+    if (limit_ns < 1000 || limit_ns > 1000000000) return QNN_ERR_INVALID_ARG;
+    int *status = nullptr, *result = nullptr;
+    QNN_TRY(qnn::status_word(&status));
+    void *scratch = nullptr;
+    QNN_TRY(qnn::scratch(qnn::kScratchReduce, 256, &scratch));
+    result = reinterpret_cast<int *>(scratch);
+    cudaStream_t st = qnn::as_stream(stream);
+    qnn::wait_timeout_kernel<<<1, 32, 0, st>>>(status, (unsigned long long)limit_ns, result);
+    QNN_CUDA_TRY(cudaGetLastError());
+    int r = 0;
+    QNN_CUDA_TRY(cudaMemcpyAsync(&r, result, sizeof(int), cudaMemcpyDeviceToHost, st));
+    QNN_CUDA_TRY(cudaStreamSynchronize(st));
+    return r == 2 ? QNN_OK : QNN_ERR_CUDA;  // 2: the wait gave up, as it must
 }

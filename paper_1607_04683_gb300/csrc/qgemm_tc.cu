@@ -109,41 +109,16 @@ struct TcArgs {
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
-__device__ __forceinline__ unsigned long long gtime() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
-    return t;
-}
+__device__ __forceinline__ unsigned long long gtime() { return global_timer_ns(); }
 __device__ __forceinline__ void mb_init(uint32_t b, unsigned n) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(b), "r"(n) : "memory");
 }
 __device__ __forceinline__ void mb_expect(uint32_t b, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(b), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ bool mb_try(uint32_t b, unsigned parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(ok)
-        : "r"(b), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
 // Bounded wait; false (and QNN_ERR_TIMEOUT recorded) if the phase did not complete in time.
 __device__ __forceinline__ bool mb_wait(uint32_t b, unsigned parity, int *status) {
-    if (mb_try(b, parity)) return true;
-    const unsigned long long t0 = gtime();
-    int spins = 0;
-    while (!mb_try(b, parity)) {
-        if (++spins >= 256) {
-            spins = 0;
-            if (gtime() - t0 > TC_WAIT_NS) {
-                record_status(status, QNN_ERR_TIMEOUT);
-                return false;
-            }
-        }
-    }
-    return true;
+    return mbar_wait_bounded(b, parity, status, TC_WAIT_NS);
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {

@@ -151,6 +151,42 @@ __device__ __forceinline__ void lstm_cell(float pi, float pf, float pg, float po
     m = lstm_cell_update(ig, fg, gg, og, c);
 }
 
+// Device clock in nanoseconds (%globaltimer).
+__device__ __forceinline__ unsigned long long global_timer_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Wait for the phase with the given parity of a shared-memory mbarrier, for at most limit_ns: on
+// time-out, record QNN_ERR_TIMEOUT and return false (the caller then skips ahead, so the kernel
+// ends and the host reads the status instead of finding the GPU hung).
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, unsigned parity, int *status,
+                                                  unsigned long long limit_ns) {
+    auto try_wait = [&]() {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        return ok != 0;
+    };
+    if (try_wait()) return true;
+    const unsigned long long t0 = global_timer_ns();
+    int spins = 0;
+    while (!try_wait()) {
+        if (++spins >= 256) {
+            spins = 0;
+            if (global_timer_ns() - t0 > limit_ns) {
+                record_status(status, QNN_ERR_TIMEOUT);
+                return false;
+            }
+        }
+    }
+    return true;
+}
+
 // Programmatic dependent launch: a kernel launched with the programmatic stream serialization
 // attribute may start while the previous kernel of its stream is still running. The wait returns
 // once that kernel has completed and its memory operations are visible (at once without such a

@@ -33,7 +33,7 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmul", "qnn_lstm_param_count",
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
            "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static",
-           "qnn_selftest_s64_to_f32", "qnn_stack_frames")
+           "qnn_selftest_s64_to_f32", "qnn_stack_frames", "qnn_selftest_wait_timeout")
 
 
 class QnnError(RuntimeError):
@@ -86,6 +86,8 @@ def lib():
         L.qnn_measure_peak.restype = i32
         L.qnn_selftest_s64_to_f32.argtypes = [P, P, i64, P]
         L.qnn_stack_frames.argtypes = [P, i64, i64, i64, i32, i32, P, P]
+        L.qnn_selftest_wait_timeout.argtypes = [i64, P]
+        L.qnn_selftest_wait_timeout.restype = i32
         L.qnn_stack_frames.restype = i32
         L.qnn_selftest_s64_to_f32.restype = i32
         L.qnn_quantize_matrix_static.argtypes = [P, i64, i64, i64, P, i64, P, P, P, P]
@@ -113,6 +115,11 @@ def selftest_s64_to_f32(values):
     _check(lib().qnn_selftest_s64_to_f32(values.data_ptr(), out.data_ptr(), values.numel(),
                                          torch.cuda.current_stream().cuda_stream), "qnn_selftest_s64_to_f32")
     return out
+
+
+def selftest_wait_timeout(limit_ns: int, stream=None):
+    """A bounded device wait that nothing ends: raises unless it gave up as designed."""
+    _check(lib().qnn_selftest_wait_timeout(int(limit_ns), _stream(stream)), "qnn_selftest_wait_timeout")
 
 
 def profile_read() -> dict:
