@@ -51,6 +51,23 @@ def parse():
     return ap.parse_args()
 
 
+def max_over_ranks(ms: float, world: int, device=None) -> float:
+    """The slowest rank's time: every rank contributes its own, all receive the maximum."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, max_ms: float, world: int) -> float:
+    """Weak scaling: every rank runs its own copy of the workload (independent sequences; no data
+    exchange), so the job processes world x units in the slowest rank's time."""
+    return world * units_per_rank / (max_ms / 1e3)
+
+
 def dist_info():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -311,13 +328,9 @@ def run_ours(args, wl, rank, world, local):
     torch.cuda.synchronize()
     qnn.profile_enable(False)
     prof = qnn.profile_read()
-    total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(step_ms), world, dev)
     frames_per_step = wl.batch * wl.frames
-    value = world * frames_per_step * args.steps / (total_ms / 1e3)
+    value = whole_job_rate(frames_per_step * args.steps, total_ms, world)
 
     # ---- end to end: pinned host buffers through the C ABI, copies inside the timed region ----
     x_host = torch.from_numpy(x).pin_memory()
@@ -336,11 +349,8 @@ def run_ours(args, wl, rank, world, local):
         b.synchronize()
         e2e_ms += a.elapsed_time(b)
     barrier()
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_value = world * frames_per_step * args.steps / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
+    e2e_value = whole_job_rate(frames_per_step * args.steps, e2e_ms, world)
     ok = qnn.device_status() == qnn.QNN_OK
     if not ok:
         raise RuntimeError("device status reported an error during the timed steps")
