@@ -456,6 +456,7 @@ def run_sweep(args):
         Y = torch.empty((shape.M, shape.N), dtype=torch.float32, device="cuda")
         t_mm = timed(lambda: qnn.qnn_qmatmul(ca, pa, 0, ra, cw, pw, cs, out=Y))
         t_q = timed(lambda: qnn.qnn_quantize(Ag, qnn.PER_MATRIX))
+        t_qr = timed(lambda: qnn.qnn_quantize(Ag, qnn.PER_ROW))
 
         def both():
             c, p, r = qnn.qnn_quantize(Ag, qnn.PER_MATRIX)
@@ -472,9 +473,28 @@ def run_sweep(args):
             "f16_tensor_peak_tflops": peaks["bf16_tflops"],
             "qmatmul_gbs": mm_bytes / t_mm / 1e9,
             "fp32_in_tops": ops / t_all / 1e12, "quantize_ms": t_q * 1e3,
-            "quantize_gbs_alg": 5.0 * shape.M * shape.K / t_q / 1e9, "hbm_peak_gbs": peaks["hbm_gbs"],
+            "quantize_gbs_alg": 5.0 * shape.M * shape.K / t_q / 1e9,
+            "quantize_rows_gbs_alg": (5.0 * shape.M * shape.K + 20.0 * shape.M) / t_qr / 1e9,
+            "hbm_peak_gbs": peaks["hbm_gbs"],
             "peak_kind": peak_kind, "l2": "flushed"}), flush=True)
         del Ag, Wg, cw, ca, Y
+        torch.cuda.empty_cache()
+    if args.shape:
+        return 0
+    # the on-the-fly quantizer alone, per-row units, on activation matrices shaped like the LSTM
+    # layers' inputs (T*B frames x width; all larger than L2)
+    gen = torch.Generator(device="cuda").manual_seed(7)
+    for rows, cols, what in ((1024000, 512, "LSTMP 5x2048p512 layer input, T=1000 B=1024"),
+                             (128000, 500, "LSTM 5x500 layer input, T=500 B=256"),
+                             (131072, 2048, "rows of 2048 (two passes)")):
+        X = torch.randn((rows, cols), device="cuda", generator=gen) * 1.7 + 0.3
+        t_qr = timed(lambda: qnn.qnn_quantize(X, qnn.PER_ROW))
+        alg = 5.0 * rows * cols + 20.0 * rows
+        print(json.dumps({"sweep": "quantize", "rows": rows, "cols": cols, "granularity": "per row",
+                          "what": what, "ms": t_qr * 1e3, "gbs_alg": alg / t_qr / 1e9,
+                          "frac_of_hbm": alg / t_qr / 1e9 / peaks["hbm_gbs"], "hbm_peak_gbs": peaks["hbm_gbs"],
+                          "peak_kind": peak_kind, "l2": "flushed"}), flush=True)
+        del X
         torch.cuda.empty_cache()
     return 0
 

@@ -2,8 +2,9 @@
 //
 // Two passes over each unit: a range pass (exact fp32 min/max, warp shuffles; non-finite values
 // flagged) and a code pass (eq. 2 with the unit's Q and z, four codes per 32-bit store, row code
-// sums). Per-row units (one frame of one sequence) take one warp per row; the second pass re-reads
-// the row from L1/L2. A per-matrix unit first reduces block partials into a small scratch array;
+// sums). Per-row units (one frame of one sequence) take one warp per row; rows of up to 1024
+// values stay in the warp's registers between the passes (read once), longer ones are re-read
+// from L1/L2. A per-matrix unit first reduces block partials into a small scratch array;
 // the last block to finish folds them into the unit's parameters, then a second launch writes codes.
 #include <cfloat>
 #include <cstdlib>
@@ -107,6 +108,83 @@ __global__ void __launch_bounds__(kRowWarps * 32) quantize_rows_kernel(const flo
     }
 }
 
+// Per-row units of at most 1024 values (16-byte aligned input rows): the warp holds its row in
+// registers, NV float4 per lane, all loads issued before any is used, so the row is read once and
+// the code pass needs no second read.
+template <int NV>
+__global__ void __launch_bounds__(kRowWarps * 32) quantize_rows_reg_kernel(const float *__restrict__ x, int64_t rows,
+                                                                          int cols, int64_t ldx,
+                                                                          uint8_t *__restrict__ codes, int64_t ldc,
+                                                                          qnn_qparams *__restrict__ params,
+                                                                          int32_t *__restrict__ sums, int *status,
+                                                                          bool pack) {
+    const int64_t row = (int64_t)blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (row >= rows) return;
+    const int lane = threadIdx.x & 31;
+    const float *xr = x + row * ldx;
+    float4 v[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int k = 4 * (lane + 32 * i);
+        if (k + 4 <= cols) {
+            v[i] = __ldg(reinterpret_cast<const float4 *>(xr + k));
+        } else {  // ragged end of the row
+            v[i].x = k < cols ? __ldg(xr + k) : 0.0f;
+            v[i].y = k + 1 < cols ? __ldg(xr + k + 1) : 0.0f;
+            v[i].z = k + 2 < cols ? __ldg(xr + k + 2) : 0.0f;
+            v[i].w = k + 3 < cols ? __ldg(xr + k + 3) : 0.0f;
+        }
+    }
+    float mn = FLT_MAX, mx = -FLT_MAX;
+    bool bad = false;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int k = 4 * (lane + 32 * i);
+        const float e[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (k + j < cols) {
+                bad |= !isfinite(e[j]);
+                mn = fminf(mn, e[j]);
+                mx = fmaxf(mx, e[j]);
+            }
+    }
+    mn = warp_min(mn);
+    mx = warp_max(mx);
+    if (__any_sync(0xffffffffu, bad)) {
+        if (lane == 0) record_status(status, QNN_ERR_NONFINITE);
+        mn = 0.0f;
+        mx = 0.0f;
+    }
+    const qnn_qparams p = params_from_range(mn, mx);
+    uint8_t *cr = codes + row * ldc;
+    int s = 0;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int k = 4 * (lane + 32 * i);
+        if (k >= cols) continue;
+        const uint32_t a = quant_code(v[i].x, p.Q, p.z), b = quant_code(v[i].y, p.Q, p.z),
+                       c = quant_code(v[i].z, p.Q, p.z), d = quant_code(v[i].w, p.Q, p.z);
+        if (pack && k + 4 <= cols) {  // 4-byte aligned code rows: one store for four codes
+            s += (int)(a + b + c + d);
+            *reinterpret_cast<uint32_t *>(cr + k) = a | (b << 8) | (c << 16) | (d << 24);
+        } else {
+            const uint32_t q4[4] = {a, b, c, d};
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (k + j < cols) {
+                    s += (int)q4[j];
+                    cr[k + j] = (uint8_t)q4[j];
+                }
+        }
+    }
+    s = warp_sum(s);
+    if (lane == 0) {
+        params[row] = p;
+        if (sums) sums[row] = s;
+    }
+}
+
 // Per-matrix pass 1: block partial ranges; the last block folds them into params[0].
 template <bool kVec>
 __global__ void __launch_bounds__(kRowWarps * 32) matrix_range_kernel(const float *__restrict__ x, int64_t rows,
@@ -197,7 +275,18 @@ qnn_status launch_quantize_rows(const float *x, int64_t rows, int64_t cols, int6
     QNN_TRY(status_word(&status));
     dim3 grid((unsigned)((rows + kRowWarps - 1) / kRowWarps));
     ProfScope prof("quantize_rows", st);
-    if (vec_ok(x, ldx, codes, ldc))
+    const int nv = (int)((cols + 127) / 128);  // float4 per lane for a register-resident row
+    const bool x_ok = ((reinterpret_cast<uintptr_t>(x) & 15) == 0) && (ldx % 4 == 0);
+    if (x_ok && nv <= 8) {
+        const bool pack = ((reinterpret_cast<uintptr_t>(codes) & 3) == 0) && (ldc % 4 == 0);
+        const int r = nv <= 1 ? 1 : nv <= 2 ? 2 : nv <= 4 ? 4 : 8;
+        switch (r) {
+            case 1: quantize_rows_reg_kernel<1><<<grid, kRowWarps * 32, 0, st>>>(x, rows, (int)cols, ldx, codes, ldc, params, sums, status, pack); break;
+            case 2: quantize_rows_reg_kernel<2><<<grid, kRowWarps * 32, 0, st>>>(x, rows, (int)cols, ldx, codes, ldc, params, sums, status, pack); break;
+            case 4: quantize_rows_reg_kernel<4><<<grid, kRowWarps * 32, 0, st>>>(x, rows, (int)cols, ldx, codes, ldc, params, sums, status, pack); break;
+            default: quantize_rows_reg_kernel<8><<<grid, kRowWarps * 32, 0, st>>>(x, rows, (int)cols, ldx, codes, ldc, params, sums, status, pack); break;
+        }
+    } else if (vec_ok(x, ldx, codes, ldc))
         quantize_rows_kernel<true><<<grid, kRowWarps * 32, 0, st>>>(x, rows, (int)cols, ldx, codes, ldc, params, sums, status);
     else
         quantize_rows_kernel<false><<<grid, kRowWarps * 32, 0, st>>>(x, rows, (int)cols, ldx, codes, ldc, params, sums, status);

@@ -78,6 +78,22 @@ def test_quantize_strided_and_degenerate_rows(qnn):
         assert np.array_equal(p[f], p_ref[f]), f
 
 
+@pytest.mark.parametrize("cols,ld", [(190, 256), (1022, 1024), (1024, 1028), (1025, 1028), (509, 512), (2, 4)])
+def test_quantize_per_row_aligned_ragged(qnn, cols, ld):
+    # 16-byte aligned rows whose length is not a multiple of 4 (ragged last float4), at and past
+    # the 1024-value register-resident limit
+    r = rng(cols * 7 + ld)
+    big = (r.normal(-0.2, 2.0, (37, ld)) * r.uniform(0.1, 5, (37, 1))).astype(np.float32)
+    codes, params, sums = qnn.qnn_quantize(gpu(big)[:, :cols], qnn.PER_ROW)
+    assert qnn.device_status() == qnn.QNN_OK
+    c_ref, p_ref, s_ref = oracle.quantize(np.ascontiguousarray(big[:, :cols]), oracle.PER_ROW)
+    assert np.array_equal(codes.cpu().numpy(), c_ref)
+    assert np.array_equal(sums.cpu().numpy(), s_ref)
+    p = qnn.params_view(params)
+    for f in ("vmin", "vmax", "Q", "z"):
+        assert np.array_equal(p[f], p_ref[f]), f
+
+
 def test_quantize_large_matrix_per_matrix(qnn):
     # config-4 size activation: 16384 x 8192, per-matrix unit; codes checked on sampled rows.
     shape = inputs.QmatmulShape(16384, 8192, 8192)
