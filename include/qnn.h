@@ -176,6 +176,47 @@ qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_
                             float *c_state, float *h_all, void *stream);
 
 /*
+ * Streaming server mode — frame-at-a-time inference with a resident kernel (the embedded,
+ * frame-by-frame setting of Sec. 1 and Sec. 3.1, where inputs are quantized on the fly as they
+ * arrive). One launch of the batch-of-few dataflow kernel stays resident for `chunk` frames and
+ * takes each frame as soon as the host has written it into host-mapped memory; the output blocks
+ * finish the softmax in the kernel and write each frame's posteriors straight to host-mapped
+ * memory, flagging the frame when it is complete. The next chunk's launch is queued when its
+ * first frame is pushed, with the state (h, c) carried from the previous launch on the device,
+ * so the results equal qnn_lstm_forward on the whole sequence (the recurrence bit for bit; the
+ * posteriors to within the rounding of the softmax's sum order).
+ *
+ * qnn_lstm_stream_open — B sequences (1 <= B <= 4) of model m (no projection, H <= 512, R and I
+ *   <= 512, output layer absent or quantized; the model's frame stacking is not applied: push
+ *   network input rows of m's input width). chunk: frames per launch (1 .. 65536). idle_seconds
+ *   (0.001 .. 3600): every wait of the kernel gives up after this long, so a stream left without
+ *   input for longer ends with QNN_ERR_TIMEOUT (reopen it to continue). Allocates pinned
+ *   host-mapped buffers of 2 chunk B (8 I + 4 out) bytes and device buffers on the current
+ *   device, and creates its own CUDA stream. Errors: QNN_ERR_INVALID_ARG (a size or the model out
+ *   of range), QNN_ERR_NO_COOP (the kernel's clusters cannot all be resident), QNN_ERR_CUDA.
+ *   The model must outlive the session.
+ * qnn_lstm_stream_push — appends n frames of every sequence: x is host memory [B][n][I]
+ *   (sequence-major, as for qnn_lstm_forward), read during the call only. At most `chunk` frames
+ *   may be pushed ahead of those pulled (QNN_ERR_INVALID_ARG otherwise, nothing pushed). Returns
+ *   without waiting for the GPU.
+ * qnn_lstm_stream_pull — waits (at most timeout_seconds) for the next n frames and copies them
+ *   into y, host memory [B][n][C] posteriors (or [B][n][R] top-layer outputs without an output
+ *   layer). n must not exceed the frames pushed and not yet pulled (QNN_ERR_INVALID_ARG).
+ *   QNN_ERR_TIMEOUT if the frames are not ready in time or the kernel gave up (see idle_seconds);
+ *   the session is then unusable except for qnn_lstm_stream_close.
+ * qnn_lstm_stream_close — completes the current launch with zero frames (their outputs are
+ *   dropped), waits for it, frees the session and returns the first error the kernel recorded
+ *   (QNN_ERR_NONFINITE for a non-finite input, QNN_ERR_TIMEOUT) or QNN_OK.
+ * A session's calls must not overlap in time (one host thread at a time).
+ */
+typedef struct qnn_lstm_stream qnn_lstm_stream;
+qnn_status qnn_lstm_stream_open(qnn_lstm_model *m, int64_t B, int64_t chunk, double idle_seconds,
+                                qnn_lstm_stream **out);
+qnn_status qnn_lstm_stream_push(qnn_lstm_stream *s, const float *x, int64_t n);
+qnn_status qnn_lstm_stream_pull(qnn_lstm_stream *s, float *y, int64_t n, double timeout_seconds);
+qnn_status qnn_lstm_stream_close(qnn_lstm_stream *s);
+
+/*
  * qnn_stack_frames — the frontend of Sec. 4: features of n consecutive frames are stacked (the frame
  * and n - 1 frames of right context) and only every stride-th stacked frame is kept.
  *   x   [B][T][I] fp32, device memory, caller-owned.

@@ -65,6 +65,29 @@ namespace qnn {
 // Arguments as for qnn_lstm_forward.
 qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
                               float *c_state, float *h_all, cudaStream_t st, bool *used);
+// Streaming with the batch-of-few kernel (stream.cu): one launch serves T frames that the host
+// supplies while it runs. Buffers: xs [B][T][I] tagged input rows (host-mapped), out [B][T][C]
+// posteriors (or [B][T][R] top-layer outputs without an output layer; host-mapped), done
+// [T][writer blocks] frame flags (host-mapped), hx [L][B][T][R] and smx [B][T][nout][2] tagged
+// device words (zeroed once; tags are launch epochs, never 0), state in h0/c0, out to h_fin/c_fin.
+struct SmallStreamArgs {
+    const unsigned long long *xs = nullptr;
+    float *out = nullptr;
+    unsigned *done = nullptr;
+    unsigned long long *hx = nullptr, *smx = nullptr;
+    const float *h0 = nullptr, *c0 = nullptr;
+    float *h_fin = nullptr, *c_fin = nullptr;
+    int *status = nullptr, *abort_flag = nullptr;
+    unsigned epoch = 0;
+    int64_t B = 0, T = 0;
+    unsigned long long wait_ns = 0;
+};
+// Whether model m streams at batch B on that kernel (QNN_ERR_INVALID_ARG: shape not supported;
+// QNN_ERR_NO_COOP: its clusters cannot all be resident), the number of blocks that flag each frame,
+// and the number of output blocks.
+qnn_status small_stream_plan(const qnn_lstm_model *m, int64_t B, int *writer_blocks, int *nout);
+qnn_status small_stream_launch(const qnn_lstm_model *m, const SmallStreamArgs &s, cudaStream_t st);
+
 // Which forward path to take, from the QNN_LSTM_PATH environment variable: "layerwise" (the
 // persistent integer-MMA recurrence), "tc" (the tensor-core recurrence), "small" or unset/"auto"
 // (small when it qualifies, else tc for batches of at least kTcMinBatch, else layerwise).

@@ -94,6 +94,14 @@ struct SmallArgs {
     unsigned epoch;
     int L, I, H, R, C, B, T, CS;
     int ups, cpu, opu;  // weight units per matrix; cells per gate unit; output rows per Wo unit
+    unsigned long long wait_ns;  // limit of every wait
+    // streaming (null otherwise): the first layer polls xs instead of reading x; the output blocks
+    // finish the softmax in the kernel and write probs; each writer block flags every frame in done
+    const unsigned long long *xs;  // [B][T][I] input rows tagged like hx, in host-mapped memory
+    float *probs;                  // [B][T][C] posteriors (host-mapped)
+    unsigned long long *smx;       // [B][T][nout][2] tagged (max, sum) softmax partials per output block
+    unsigned *done;                // [T][writer blocks]: the launch's epoch once the block's rows of frame t are out
+    int nout;                      // output blocks (output clusters x CS)
 };
 
 // ---- shared memory layout ---------------------------------------------------------------------
@@ -115,6 +123,8 @@ struct Smem {
     int acc_x[2][kMaxB][kRows];         // int32 sums [frame parity][seq][row]
     int acc_h[2][kMaxB][kRows];
     RowMeta meta_x[2][kMaxB], meta_h[2][kMaxB];
+    float red_m[kPW][kMaxB], red_s[kPW][kMaxB];  // in-kernel softmax: per-warp partials
+    float2 sm_fin[kMaxB];                        // (max, sum) of the whole output row
     uint8_t wx[kRows][kMaxK];            // Wx rows of this block (local row order)
     unsigned long long bar_full[kRing], bar_empty[kRing], bar_h[2], bar_ax[2], bar_ah[2], bar_ep[2];
 };
@@ -192,6 +202,15 @@ __device__ __forceinline__ unsigned long long ld_tag(const unsigned long long *p
 __device__ __forceinline__ void st_tag(unsigned long long *p, unsigned long long v) {
     asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
+// Host-mapped words written by the host (inputs) or read by it (frame flags): system scope.
+__device__ __forceinline__ unsigned long long ld_tag_sys(const unsigned long long *p) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.sys.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_flag_sys(unsigned *p, unsigned v) {
+    asm volatile("st.release.sys.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
 __device__ __forceinline__ void named_bar(int id, int count) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
@@ -207,14 +226,22 @@ struct Deadline {
         if (++spins < kSpinCheck) return false;
         spins = 0;
         if (*(volatile int *)a->abort_flag) return true;
-        if (now_ns() - t0 > kWaitNs) {
+        if (now_ns() - t0 > a->wait_ns) {
             record_status(a->status, QNN_ERR_TIMEOUT);
             atomicExch(a->abort_flag, 1);
+            __threadfence();  // the flag is visible before anything computed after the give-up
             return true;
         }
         return false;
     }
 };
+
+// Whether some wait of the launch has given up (after a fence, so that data which depends on a
+// give-up is never taken for good).
+__device__ __forceinline__ bool aborted(const SmallArgs &a) {
+    __threadfence();
+    return *(volatile int *)a.abort_flag != 0;
+}
 
 __device__ __forceinline__ void wait_cta(const SmallArgs &a, uint32_t bar, unsigned parity) {
     if (mbar_try(bar, parity)) return;
@@ -370,7 +397,12 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
     if (warp == kLoaderWarp) {
         // ---------------- loader ----------------
         const unsigned long long *src = nullptr;
-        if (!(is_layer && l == 0)) src = a.hx + (int64_t)(is_layer ? l - 1 : a.L - 1) * B * T * R;
+        int64_t src_ld = R;
+        const bool sys = is_layer && l == 0;  // streamed input rows, written by the host
+        if (!(is_layer && l == 0))
+            src = a.hx + (int64_t)(is_layer ? l - 1 : a.L - 1) * B * T * R;
+        else if (a.xs)
+            src = a.xs, src_ld = a.I;
         for (int t = 0; t < T; ++t) {
             const int slot = t % kRing;
             if (t >= kRing) wait_cta(a, empty0 + 8 * slot, ((t / kRing) - 1) & 1);
@@ -388,12 +420,13 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                         mx = fmaxf(mx, v);
                     }
                 } else {
-                    const unsigned long long *hr = src + ((int64_t)b * T + t) * R;
+                    const unsigned long long *hr = src + ((int64_t)b * T + t) * src_ld;
+                    auto ld = [&](const unsigned long long *p) { return sys ? ld_tag_sys(p) : ld_tag(p); };
                     unsigned long long v[16];
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
                         const int k = lane + 32 * i;
-                        v[i] = k < kin ? ld_tag(hr + k) : ((unsigned long long)a.epoch << 32);
+                        v[i] = k < kin ? ld(hr + k) : ((unsigned long long)a.epoch << 32);
                     }
                     Deadline d{&a, now_ns(), 0};
                     while (true) {
@@ -402,10 +435,11 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                         for (int i = 0; i < 16; ++i) ready &= (unsigned)(v[i] >> 32) == a.epoch;
                         if (__all_sync(0xffffffffu, ready)) break;
                         if (__any_sync(0xffffffffu, d.expired())) break;
+                        if (sys) __nanosleep(64);  // host-mapped input: fewer polls across the host link
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             const int k = lane + 32 * i;
-                            if (k < kin && (unsigned)(v[i] >> 32) != a.epoch) v[i] = ld_tag(hr + k);
+                            if (k < kin && (unsigned)(v[i] >> 32) != a.epoch) v[i] = ld(hr + k);
                         }
                     }
 #pragma unroll
@@ -459,6 +493,91 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 o_b = a.bo[n];
             }
         }
+        // Streaming: the softmax of frame t over the rows of every output block. Each block reduces
+        // its rows to (m_b, s_b) = (max l, sum E(l - m_b)), publishes them as tagged words, gathers
+        // every block's pair, and merges them the same way in every block: M = max m_b,
+        // sum = sum_b s_b E(m_b - M); a row's posterior is E(l - M) / sum. The block then flags the
+        // frame for the host.
+        auto softmax_out = [&](int t, const float (&lg)[kMaxB]) {
+            const bool mine = row_writer && o_n >= 0;
+            const int ob = (cid - a.L) * CS + (int)rank;
+            const unsigned long long tag = (unsigned long long)a.epoch << 32;
+#pragma unroll
+            for (int b = 0; b < kMaxB; ++b) {
+                if (b >= B) break;
+                const float m = warp_max(mine ? lg[b] : -FLT_MAX);
+                if (lane == 0) S.red_m[warp][b] = m;
+            }
+            named_bar(1, kPT);
+            float bm[kMaxB];
+#pragma unroll
+            for (int b = 0; b < kMaxB; ++b) {
+                bm[b] = -FLT_MAX;
+                if (b >= B) break;
+                for (int w = 0; w < kPW; ++w) bm[b] = fmaxf(bm[b], S.red_m[w][b]);
+                const float e = warp_sum_f(mine ? pexp(__fsub_rn(lg[b], bm[b])) : 0.0f);
+                if (lane == 0) S.red_s[warp][b] = e;
+            }
+            named_bar(1, kPT);
+            if (warp == 0) {
+#pragma unroll
+                for (int b = 0; b < kMaxB; ++b) {
+                    if (b >= B) break;
+                    unsigned long long *row = a.smx + ((int64_t)b * T + t) * a.nout * 2;
+                    if (lane == 0) {
+                        float sum = 0.0f;
+                        for (int w = 0; w < kPW; ++w) sum = __fadd_rn(sum, S.red_s[w][b]);
+                        st_tag(row + 2 * ob, tag | __float_as_uint(bm[b]));
+                        st_tag(row + 2 * ob + 1, tag | __float_as_uint(sum));
+                    }
+                    // lane i gathers the pairs of blocks i, i + 32, ...: first wait for them and take
+                    // the maximum, then read them again (now present) for the sum
+                    const int rounds = (a.nout + 31) / 32;
+                    float M = -FLT_MAX;
+#pragma unroll 1
+                    for (int q = 0; q < rounds; ++q) {
+                        const int i = lane + 32 * q;
+                        unsigned long long mv = tag, sv = tag;  // absent blocks: never waited for
+                        if (i < a.nout) mv = ld_tag(row + 2 * i), sv = ld_tag(row + 2 * i + 1);
+                        Deadline d{&a, now_ns(), 0};
+                        while (true) {
+                            const bool ready = (unsigned)(mv >> 32) == a.epoch && (unsigned)(sv >> 32) == a.epoch;
+                            if (__all_sync(0xffffffffu, ready)) break;
+                            if (__any_sync(0xffffffffu, d.expired())) break;
+                            if (i < a.nout && (unsigned)(mv >> 32) != a.epoch) mv = ld_tag(row + 2 * i);
+                            if (i < a.nout && (unsigned)(sv >> 32) != a.epoch) sv = ld_tag(row + 2 * i + 1);
+                        }
+                        if (i < a.nout) M = fmaxf(M, __uint_as_float((unsigned)mv));
+                    }
+                    M = warp_max(M);
+                    float part = 0.0f;
+#pragma unroll 1
+                    for (int q = 0; q < rounds; ++q) {
+                        const int i = lane + 32 * q;
+                        if (i < a.nout) {
+                            const float mi = __uint_as_float((unsigned)ld_tag(row + 2 * i));
+                            const float si = __uint_as_float((unsigned)ld_tag(row + 2 * i + 1));
+                            part = __fadd_rn(part, __fmul_rn(si, pexp(__fsub_rn(mi, M))));
+                        }
+                    }
+                    part = warp_sum_f(part);  // xor butterfly: the same sum in every lane and block
+                    if (lane == 0) S.sm_fin[b] = make_float2(M, part);
+                }
+            }
+            named_bar(1, kPT);
+#pragma unroll
+            for (int b = 0; b < kMaxB; ++b) {
+                if (b >= B) break;
+                if (mine) {
+                    const float2 f = S.sm_fin[b];
+                    a.probs[((int64_t)b * T + t) * a.C + o_n] = __fdiv_rn(pexp(__fsub_rn(lg[b], f.x)), f.y);
+                }
+            }
+            if (mine) __threadfence_system();
+            named_bar(1, kPT);
+            // a frame computed after some wait gave up is not flagged (its values may be stale)
+            if (tid == 0 && !aborted(a)) st_flag_sys(a.done + (int64_t)t * a.nout + ob, a.epoch);
+        };
         // X phase of frame t: ring -> codes -> products (layer: Wx sums to the epilogue; output
         // layer: logits).
         auto x_phase = [&](int t) {
@@ -471,28 +590,35 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
             }
             named_bar(1, kPT);
             if (tid == 0) mbar_arrive(empty0 + 8 * slot);
-            for (int b = 0; b < B; ++b) {
-                int rs = 0;
-                int s;
-                if (is_layer) {
-                    s = dot8([&](int r) { return *reinterpret_cast<const uint4 *>(&S.wx[lr0 + r][lane * 16]); },
+            if (is_layer) {
+                for (int b = 0; b < B; ++b) {
+                    int rs = 0;
+                    const int s =
+                        dot8([&](int r) { return *reinterpret_cast<const uint4 *>(&S.wx[lr0 + r][lane * 16]); },
                              S.codes_x[b], warp == 0, rs);
                     if (row_writer) S.acc_x[par][b][my_row] = s;
                     if (tid == 0) S.meta_x[par][b].rs = rs;
-                } else {
-                    s = dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
-                             S.codes_x[b], true, rs);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(axb0 + 8 * par);
+            } else {
+                float lg[kMaxB];
+#pragma unroll
+                for (int b = 0; b < kMaxB; ++b) {
+                    lg[b] = 0.0f;
+                    if (b >= B) break;
+                    int rs = 0;
+                    const int s = dot8([&](int r) { return make_uint4(wr[r][0], wr[r][1], wr[r][2], wr[r][3]); },
+                                       S.codes_x[b], true, rs);
                     if (row_writer && o_n >= 0) {
                         const RowMeta mt = S.meta_x[par][b];
                         const qnn_qparams po = a.wo_p[o_n / a.opu];
                         const long long Sv = offset_product(s, mt.za, po.z, rs, o_cs, R);
-                        a.logits[((int64_t)b * T + t) * a.C + o_n] = __fadd_rn(recover_product(Sv, mt.Qa, po.Q), o_b);
+                        lg[b] = __fadd_rn(recover_product(Sv, mt.Qa, po.Q), o_b);
+                        if (a.logits) a.logits[((int64_t)b * T + t) * a.C + o_n] = lg[b];
                     }
                 }
-            }
-            if (is_layer) {
-                __syncwarp();
-                if (lane == 0) mbar_arrive(axb0 + 8 * par);
+                if (a.probs) softmax_out(t, lg);
             }
         };
         if (!is_layer) {
@@ -624,6 +750,11 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                     if (a.ytop && l == a.L - 1) a.ytop[((int64_t)b * T + t) * R + j] = h;
                 }
             }
+            if (a.done && a.C == 0 && l == a.L - 1) {  // streaming without an output layer: h_t is the output
+                if (g == 0 && jv) __threadfence_system();
+                named_bar(2, kET);
+                if (et == 0 && !aborted(a)) st_flag_sys(a.done + (int64_t)t * CS + rank, a.epoch);
+            }
             __syncwarp();
             if (lane == 0) mbar_arrive(saddr(&S.bar_ep[par]));  // gate arithmetic of frame t done
         }
@@ -647,7 +778,115 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
 
 int g_small_cfg_dev = -1;
 
+// Launch geometry of the kernel for model m at batch B; false when the model or batch does not
+// fit this path (then nothing is set).
+struct SmallGeom {
+    int CS = 0, clusters = 0, nout = 0;
+};
+bool small_geometry(const qnn_lstm_model *m, int64_t B, SmallGeom *g) {
+    const int64_t L = m->L, I = m->I, H = m->H, C = m->C, R = m->R;
+    if (m->P != 0 || B < 1 || B > kMaxB || L > kMaxLayers || I > kMaxK || R > kMaxK || H > kCellsPerBlock * kMaxCS)
+        return false;
+    if (C > 0 && m->d.output_mode != QNN_OUT_QUANT) return false;
+    g->CS = (int)((H + kCellsPerBlock - 1) / kCellsPerBlock);
+    const int out_blocks = C > 0 ? (int)((C + kRows - 1) / kRows) : 0;
+    const int out_clusters = (out_blocks + g->CS - 1) / g->CS;
+    g->clusters = (int)L + out_clusters;
+    g->nout = out_clusters * g->CS;
+    return true;
+}
+
+// Sets the kernel's attributes (once per device) and fills the cluster launch configuration;
+// *fits tells whether all clusters can be resident at once (the dataflow between them needs it).
+qnn_status small_config(const SmallGeom &g, cudaStream_t st, cudaLaunchConfig_t *cfg, cudaLaunchAttribute *attr,
+                        bool *fits) {
+    const size_t smem = sizeof(Smem);
+    int dev = 0;
+    QNN_CUDA_TRY(cudaGetDevice(&dev));
+    if (g_small_cfg_dev != dev) {
+        QNN_CUDA_TRY(cudaFuncSetAttribute(lstm_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        QNN_CUDA_TRY(cudaFuncSetAttribute(lstm_small_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
+        g_small_cfg_dev = dev;
+    }
+    *cfg = cudaLaunchConfig_t{};
+    cfg->gridDim = dim3((unsigned)(g.clusters * g.CS));
+    cfg->blockDim = dim3(kSThreads);
+    cfg->dynamicSmemBytes = smem;
+    cfg->stream = st;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)g.CS;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg->attrs = attr;
+    cfg->numAttrs = 1;
+    int max_clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, lstm_small_kernel, cfg) != cudaSuccess) {
+        cudaGetLastError();
+        *fits = false;
+        return QNN_OK;
+    }
+    *fits = max_clusters >= g.clusters;
+    return QNN_OK;
+}
+
+// The model's weights, units and shapes into the kernel arguments.
+void small_model_args(const qnn_lstm_model *m, const SmallGeom &g, int64_t B, int64_t T, SmallArgs *a) {
+    for (int64_t l = 0; l < m->L; ++l) {
+        const LayerDev &ly = m->layers[l];
+        a->layer[l] = SmallLayer{ly.wx.codes, ly.wx.sums, ly.wx.params, ly.wh.codes, ly.wh.sums, ly.wh.params,
+                                 ly.bias, (int)ly.wx.ld, (int)ly.wh.ld, (int)ly.kin};
+    }
+    if (m->C > 0) {
+        a->wo = m->wo.codes, a->wo_sum = m->wo.sums, a->wo_p = m->wo.params, a->bo = m->bo, a->ldo = (int)m->wo.ld;
+    }
+    a->L = (int)m->L, a->I = (int)m->I, a->H = (int)m->H, a->R = (int)m->R, a->C = (int)m->C;
+    a->B = (int)B, a->T = (int)T, a->CS = g.CS, a->nout = g.nout;
+    a->ups = (int)m->S, a->cpu = (int)(m->H / m->S), a->opu = m->C > 0 ? (int)(m->C / m->S) : 1;
+    a->wait_ns = kWaitNs;
+}
+
 }  // namespace
+
+qnn_status small_stream_plan(const qnn_lstm_model *m, int64_t B, int *writer_blocks, int *nout) {
+    SmallGeom g;
+    if (!small_geometry(m, B, &g)) return QNN_ERR_INVALID_ARG;
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute attr[1];
+    bool fits = false;
+    QNN_TRY(small_config(g, nullptr, &cfg, attr, &fits));
+    if (!fits) return QNN_ERR_NO_COOP;
+    *nout = g.nout;
+    *writer_blocks = m->C > 0 ? g.nout : g.CS;
+    return QNN_OK;
+}
+
+qnn_status small_stream_launch(const qnn_lstm_model *m, const SmallStreamArgs &s, cudaStream_t st) {
+    SmallGeom g;
+    if (!small_geometry(m, s.B, &g)) return QNN_ERR_INVALID_ARG;
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute attr[1];
+    bool fits = false;
+    QNN_TRY(small_config(g, st, &cfg, attr, &fits));
+    if (!fits) return QNN_ERR_NO_COOP;
+    SmallArgs a{};
+    small_model_args(m, g, s.B, s.T, &a);
+    a.xs = s.xs;
+    a.hx = s.hx;
+    a.smx = s.smx;
+    a.done = s.done;
+    if (m->C > 0)
+        a.probs = s.out;
+    else
+        a.ytop = s.out;
+    a.h0 = s.h0, a.c0 = s.c0, a.h_fin = s.h_fin, a.c_fin = s.c_fin;
+    a.status = s.status;
+    a.abort_flag = s.abort_flag;
+    a.epoch = s.epoch;
+    a.wait_ns = s.wait_ns;
+    ProfScope prof("lstm_small_stream", st);
+    QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, lstm_small_kernel, a));
+    return QNN_OK;
+}
 
 PathChoice path_choice() {
     const char *v = std::getenv("QNN_LSTM_PATH");
@@ -662,40 +901,13 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
                               float *c_state, float *h_all, cudaStream_t st, bool *used) {
     *used = false;
     const int64_t L = m->L, I = m->I, H = m->H, C = m->C, R = m->R;
-    if (m->P != 0 || B > kMaxB || L > kMaxLayers || I > kMaxK || R > kMaxK || H > kCellsPerBlock * kMaxCS) return QNN_OK;
-    if (C > 0 && m->d.output_mode != QNN_OUT_QUANT) return QNN_OK;
-    if (T > (int64_t)INT32_MAX / 4) return QNN_OK;
-    const int CS = (int)((H + kCellsPerBlock - 1) / kCellsPerBlock);
-    const int out_blocks = C > 0 ? (int)((C + kRows - 1) / kRows) : 0;
-    const int out_clusters = (out_blocks + CS - 1) / CS;
-    const int clusters = (int)L + out_clusters;
-    const size_t smem = sizeof(Smem);
-
-    int dev = 0;
-    QNN_CUDA_TRY(cudaGetDevice(&dev));
-    if (g_small_cfg_dev != dev) {
-        QNN_CUDA_TRY(cudaFuncSetAttribute(lstm_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        QNN_CUDA_TRY(cudaFuncSetAttribute(lstm_small_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
-        g_small_cfg_dev = dev;
-    }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(clusters * CS));
-    cfg.blockDim = dim3(kSThreads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = st;
+    SmallGeom geo;
+    if (!small_geometry(m, B, &geo) || T > (int64_t)INT32_MAX / 4) return QNN_OK;
+    cudaLaunchConfig_t cfg;
     cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = (unsigned)CS;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int max_clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, lstm_small_kernel, &cfg) != cudaSuccess) {
-        cudaGetLastError();
-        return QNN_OK;
-    }
-    if (max_clusters < clusters) return QNN_OK;  // cannot be co-resident: layer-by-layer path
+    bool fits = false;
+    QNN_TRY(small_config(geo, st, &cfg, attr, &fits));
+    if (!fits) return QNN_OK;  // cannot be co-resident: layer-by-layer path
 
     // workspace: staging, tagged layer outputs, logits, state
     const bool x_dev = is_device_ptr(x), y_dev = is_device_ptr(y);
@@ -734,14 +946,7 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
     }
     char *ws = reinterpret_cast<char *>(m->sws);
     SmallArgs a{};
-    for (int64_t l = 0; l < L; ++l) {
-        const LayerDev &ly = m->layers[l];
-        a.layer[l] = SmallLayer{ly.wx.codes, ly.wx.sums, ly.wx.params, ly.wh.codes, ly.wh.sums, ly.wh.params,
-                                ly.bias, (int)ly.wx.ld, (int)ly.wh.ld, (int)ly.kin};
-    }
-    if (C > 0) {
-        a.wo = m->wo.codes, a.wo_sum = m->wo.sums, a.wo_p = m->wo.params, a.bo = m->bo, a.ldo = (int)m->wo.ld;
-    }
+    small_model_args(m, geo, B, T, &a);
     const float *xd = x;
     if (!x_dev) {
         QNN_CUDA_TRY(cudaMemcpyAsync(ws + o_x, x, sizeof(float) * rows * I, cudaMemcpyHostToDevice, st));
@@ -771,8 +976,6 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
     a.status = status;
     a.abort_flag = reinterpret_cast<int *>(ws + o_flag);
     a.epoch = m->epoch;
-    a.L = (int)L, a.I = (int)I, a.H = (int)H, a.R = (int)R, a.C = (int)C, a.B = (int)B, a.T = (int)T, a.CS = CS;
-    a.ups = (int)m->S, a.cpu = (int)(H / m->S), a.opu = C > 0 ? (int)(C / m->S) : 1;
     {
         ProfScope prof("lstm_small", st);
         QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, lstm_small_kernel, a));

@@ -33,7 +33,8 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmul", "qnn_lstm_param_count",
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
            "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static",
-           "qnn_selftest_s64_to_f32", "qnn_stack_frames", "qnn_selftest_wait_timeout")
+           "qnn_selftest_s64_to_f32", "qnn_stack_frames", "qnn_selftest_wait_timeout", "qnn_lstm_stream_open",
+           "qnn_lstm_stream_push", "qnn_lstm_stream_pull", "qnn_lstm_stream_close")
 
 
 class QnnError(RuntimeError):
@@ -90,6 +91,14 @@ def lib():
         L.qnn_selftest_wait_timeout.restype = i32
         L.qnn_stack_frames.restype = i32
         L.qnn_selftest_s64_to_f32.restype = i32
+        L.qnn_lstm_stream_open.argtypes = [P, i64, i64, C.c_double, C.POINTER(P)]
+        L.qnn_lstm_stream_open.restype = i32
+        L.qnn_lstm_stream_push.argtypes = [P, P, i64]
+        L.qnn_lstm_stream_push.restype = i32
+        L.qnn_lstm_stream_pull.argtypes = [P, P, i64, C.c_double]
+        L.qnn_lstm_stream_pull.restype = i32
+        L.qnn_lstm_stream_close.argtypes = [P]
+        L.qnn_lstm_stream_close.restype = i32
         L.qnn_quantize_matrix_static.argtypes = [P, i64, i64, i64, P, i64, P, P, P, P]
         L.qnn_quantize_matrix_static.restype = i32
         _lib = L
@@ -268,3 +277,38 @@ class LstmModel:
         _check(lib().qnn_lstm_forward(self._h, _p(x), B, x.shape[1], _p(y), _p(h_state), _p(c_state), _p(h_all),
                                       _stream(stream)), "qnn_lstm_forward")
         return y
+
+
+class LstmStream:
+    """Streaming server mode (qnn_lstm_stream_*): B sequences fed frame by frame to a resident
+    kernel; push() appends frames [B, n, I], pull() returns the next frames' outputs [B, n, out]
+    (posteriors, or top-layer outputs without an output layer). Host numpy arrays only."""
+
+    def __init__(self, model: LstmModel, B: int, chunk: int = 1024, idle_seconds: float = 10.0):
+        self.model, self.B = model, B
+        d = model.desc
+        self.I = d.input_dim * max(d.stack, 1)
+        self.out_dim = d.num_classes if d.num_classes > 0 else model.R
+        h = C.c_void_p()
+        _check(lib().qnn_lstm_stream_open(model._h, B, chunk, idle_seconds, C.byref(h)), "qnn_lstm_stream_open")
+        self._h = h
+
+    def push(self, x: np.ndarray):
+        x = np.ascontiguousarray(x, dtype=np.float32)
+        assert x.ndim == 3 and x.shape[0] == self.B and x.shape[2] == self.I
+        _check(lib().qnn_lstm_stream_push(self._h, _p(x), x.shape[1]), "qnn_lstm_stream_push")
+
+    def pull(self, n: int, timeout: float = 10.0) -> np.ndarray:
+        y = np.empty((self.B, n, self.out_dim), np.float32)
+        _check(lib().qnn_lstm_stream_pull(self._h, _p(y), n, timeout), "qnn_lstm_stream_pull")
+        return y
+
+    def close(self) -> int:
+        """Ends the session; returns the first status the kernel recorded (QNN_OK if none)."""
+        st = QNN_OK
+        if getattr(self, "_h", None) and _lib is not None:
+            st = _lib.qnn_lstm_stream_close(self._h)
+            self._h = None
+        return st
+
+    __del__ = close

@@ -67,3 +67,9 @@ def test_argument_errors_need_no_gpu(qlib):
     assert qlib.qnn_lstm_model_create(C.byref(qnn.lstm_desc(0, 1, 1)), None, C.byref(h)) == qnn.QNN_ERR_INVALID_ARG
     for args in ((-1, 3, 4, 8, 3), (1, 0, 4, 8, 3), (1, 3, 0, 8, 3), (1, 3, 4, 0, 3), (1, 3, 4, 8, 0)):
         assert qlib.qnn_stack_frames(None, *args, None, None) == qnn.QNN_ERR_INVALID_ARG
+    # streaming session calls: null handles and out-of-range sizes
+    s = C.c_void_p()
+    assert qlib.qnn_lstm_stream_open(None, 1, 8, 1.0, C.byref(s)) == qnn.QNN_ERR_INVALID_ARG
+    assert qlib.qnn_lstm_stream_push(None, None, 1) == qnn.QNN_ERR_INVALID_ARG
+    assert qlib.qnn_lstm_stream_pull(None, None, 1, 1.0) == qnn.QNN_ERR_INVALID_ARG
+    assert qlib.qnn_lstm_stream_close(None) == qnn.QNN_ERR_INVALID_ARG
