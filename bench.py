@@ -44,6 +44,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="standalone quantized matmul sweep instead")
     ap.add_argument("--shape", default="", help="with --sweep: one shape M,N,K only")
+    ap.add_argument("--stream", action="store_true",
+                    help="streaming server mode instead: per-frame latency and burst rate of a resident session")
     ap.add_argument("--frames", type=int, default=0,
                     help="profiling aid: run only the first N frames of the workload (same per-launch shapes)")
     ap.add_argument("--layers", type=int, default=0,
@@ -499,10 +501,74 @@ def run_sweep(args):
     return 0
 
 
+def run_stream(args):
+    """Streaming server mode on the batch-1 workload's model (5 x 500 cells, 2000 classes): a
+    session pushes one frame and pulls its posteriors before the next (round-trip latency seen by
+    the host, wall clock), then pushes and pulls bursts of 64 frames (sustained rate). Inputs from
+    host memory, outputs to host memory; one JSON line per measurement."""
+    import numpy as np
+    import torch
+
+    from paper_1607_04683_gb300 import build as qbuild, qnn
+    qbuild.build()
+    torch.cuda.set_device(0)
+    wl = inputs.LSTM_5x500_B1
+    params, x = wl.make()
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, torch.from_numpy(params).cuda())
+    T = x.shape[1]
+    chunk = 1024
+    # for comparison, the same frame-by-frame use through the batch call: one qnn_lstm_forward of
+    # one frame per step, state carried on the device, input and output in pinned host memory
+    # (measured before the session opens: its resident kernel holds the SMs this call needs)
+    hs = torch.zeros((wl.num_layers, 1, wl.R), dtype=torch.float32, device="cuda")
+    cs = torch.zeros((wl.num_layers, 1, wl.hidden), dtype=torch.float32, device="cuda")
+    xh = torch.from_numpy(x).pin_memory()
+    yh = torch.empty((1, 1, wl.num_classes), dtype=torch.float32).pin_memory()
+    cur = torch.cuda.current_stream()
+    lat_f = []
+    for t in range(T):
+        t0 = time.perf_counter()
+        model.forward(xh[:, t:t + 1], y=yh, h_state=hs, c_state=cs)
+        cur.synchronize()
+        lat_f.append(time.perf_counter() - t0)
+    lat_f = np.array(lat_f[20:]) * 1e6
+    print(json.dumps({"bench": "stream", "mode": "frame by frame through qnn_lstm_forward (1 frame per call)",
+                      "model": wl.name, "frames": int(lat_f.size), "latency_us_median": float(np.median(lat_f)),
+                      "latency_us_p99": float(np.percentile(lat_f, 99))}), flush=True)
+    s = qnn.LstmStream(model, 1, chunk=chunk, idle_seconds=10.0)
+    lat = []
+    for t in range(T):
+        t0 = time.perf_counter()
+        s.push(x[:, t:t + 1])
+        s.pull(1)
+        lat.append(time.perf_counter() - t0)
+    lat = np.array(lat[20:]) * 1e6  # past the first launch's start
+    print(json.dumps({"bench": "stream", "mode": "frame by frame (push 1, pull 1)", "model": wl.name,
+                      "frames": int(lat.size), "latency_us_median": float(np.median(lat)),
+                      "latency_us_p99": float(np.percentile(lat, 99)), "latency_us_min": float(lat.min()),
+                      "chunk": chunk, "io": "host memory (host-mapped buffers)"}), flush=True)
+    burst = 64
+    reps = 40
+    t0 = time.perf_counter()
+    for i in range(reps):
+        xs = x[:, (i * burst) % (T - burst):(i * burst) % (T - burst) + burst]
+        s.push(xs)
+        s.pull(burst)
+    dt = time.perf_counter() - t0
+    st = s.close()
+    print(json.dumps({"bench": "stream", "mode": f"bursts of {burst} frames", "model": wl.name,
+                      "frames": burst * reps, "frames_per_s": burst * reps / dt, "status": int(st),
+                      "chunk": chunk}), flush=True)
+    return 0 if st == qnn.QNN_OK else 1
+
+
 def main():
     args = parse()
     if args.sweep:
         return run_sweep(args)
+    if args.stream:
+        return run_stream(args)
     rank, world, local = dist_info()
     wl = inputs.LSTM_WORKLOADS[args.workload]
     if args.frames or args.layers:  # a cut of the named workload (its name says so)

@@ -24,6 +24,8 @@
 //   E  the epilogue warps apply eq. 1's offsets, recover, add the bias, apply
 //      the gates and the cell update, send their new h values and range to every block of the
 //      cluster, and write them tagged to global memory for the next layer.
+// (Streaming launches, whose inputs arrive one at a time, take H before X within each frame: the
+// Wh product of frame t is done while x_t is still awaited.)
 // A layer's recurrence only waits on its own cluster; consecutive layers run one frame apart. Every
 // wait is bounded in time: one that gives up records QNN_ERR_TIMEOUT and raises an abort flag,
 // after which all waits return at once, so every block runs its loop to the end (outputs then
@@ -102,6 +104,9 @@ struct SmallArgs {
     unsigned long long *smx;       // [B][T][nout][2] tagged (max, sum) softmax partials per output block
     unsigned *done;                // [T][writer blocks]: the launch's epoch once the block's rows of frame t are out
     int nout;                      // output blocks (output clusters x CS)
+    int h_first;                   // order of a frame's products: Wh h_{t-1} before Wx x_t (latency, for
+                                   // inputs that arrive one at a time) instead of Wx x_{t+1} right after
+                                   // Wh h_{t-1} (throughput: it overlaps the cluster exchange)
 };
 
 // ---- shared memory layout ---------------------------------------------------------------------
@@ -627,7 +632,7 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 named_bar(1, kPT);  // codes_x is rewritten next frame
             }
         } else {
-            if (T > 0) x_phase(0);
+            if (T > 0 && !a.h_first) x_phase(0);
             for (int t = 0; t < T; ++t) {
                 const int par = t & 1, pb = (t - 1) & 1;
                 if (t > 0) {
@@ -667,8 +672,12 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
                 __syncwarp();
                 if (lane == 0) mbar_arrive(ahb0 + 8 * par);
                 // X phase of the next frame overlaps the cluster exchange of this one
-                if (kXAfterEpilogue) wait_cta(a, saddr(&S.bar_ep[par]), (t >> 1) & 1);
-                if (t + 1 < T) x_phase(t + 1);
+                if (a.h_first) {
+                    x_phase(t);  // h_{t-1} was known before x_t arrived: only Wx x_t is left after it
+                } else {
+                    if (kXAfterEpilogue) wait_cta(a, saddr(&S.bar_ep[par]), (t >> 1) & 1);
+                    if (t + 1 < T) x_phase(t + 1);
+                }
             }
         }
     } else if (is_layer) {
@@ -883,6 +892,7 @@ qnn_status small_stream_launch(const qnn_lstm_model *m, const SmallStreamArgs &s
     a.abort_flag = s.abort_flag;
     a.epoch = s.epoch;
     a.wait_ns = s.wait_ns;
+    a.h_first = 1;
     ProfScope prof("lstm_small_stream", st);
     QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, lstm_small_kernel, a));
     return QNN_OK;
