@@ -385,6 +385,14 @@ def run_ours(args, wl, rank, world, local):
                     "alg_bytes_per_launch": small_bytes_per_launch(wl), "hbm_frac":
                         small_bytes_per_launch(wl) / avg_s / 1e9 / peaks["hbm_gbs"],
                     "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
+        # a frame of a layer is a chain of dependent steps: its time against the measured floor of
+        # the kernel's per-frame synchronisation (cluster exchange + hand-over, no arithmetic)
+        cs = (wl.hidden + 31) // 32
+        floor_us = qnn.measure_exchange_floor(cs, 20000)
+        us_frame = avg_s * 1e6 / wl.frames
+        roofline["latency"] = {"us_per_frame": us_frame, "floor_us_per_frame": floor_us,
+                               "frac": floor_us / us_frame, "cluster_blocks": cs,
+                               "floor_kind": "measured (qnn_measure_exchange_floor)"}
     elif kname == "lstm_gates_tc":
         # one recurrent step of one layer: the tcgen05 gate product with the LSTM cell in its
         # epilogue; reported against HBM with the step's algorithmic bytes, plus its tensor rate

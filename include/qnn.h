@@ -273,6 +273,16 @@ qnn_status qnn_profile_read(int capacity, const char **names, double *total_ms, 
  * Register-only loops on every SM; synchronous; the best of three timed runs. */
 qnn_status qnn_measure_peak(int kind, double *tops);
 
+/* Measures the latency floor of the batch-of-few recurrence (no counterpart in the paper): the
+ * time per round, in microseconds, of that kernel's per-frame synchronisation skeleton with all
+ * arithmetic removed, on one cluster of cluster_size (1 .. 16) blocks: product warps wait for the
+ * cluster-wide exchange of the previous frame's outputs (distributed shared memory stores completing
+ * on a transaction-count barrier) and hand over to the epilogue warps, which send their values to
+ * every block of the cluster. A layer of that kernel cannot take less per frame. rounds: 1 ..
+ * 10^6 rounds per launch; synchronous; best of three launches; QNN_ERR_NO_COOP if the cluster
+ * cannot be launched, QNN_ERR_TIMEOUT if a (bounded) wait gave up. */
+qnn_status qnn_measure_exchange_floor(int32_t cluster_size, int32_t rounds, double *us_per_round);
+
 /* Diagnostic (no counterpart in the paper): out[i] = in[i] rounded to the nearest fp32 value, ties
  * to even, by the conversion the recovery of eq. (3) uses on the device for the exact int64 sums
  * S of eq. (1). in [n] int64 and out [n] float are device buffers owned by the caller; errors:

@@ -223,8 +223,10 @@ __device__ __forceinline__ void named_bar(int id, int count) {
 // Bounded waits. A wait that gives up records QNN_ERR_TIMEOUT and raises the abort flag; every
 // later wait then returns within kSpinCheck polls. Waits never make a warp leave its loop, so all
 // warps keep executing the same sequence of named barriers and the launch always runs to its end.
-struct Deadline {
-    const SmallArgs *a;
+// (A: any argument block with status, abort_flag and wait_ns.)
+template <typename A>
+struct DeadlineT {
+    const A *a;
     unsigned long long t0;
     int spins;
     __device__ bool expired() {
@@ -240,6 +242,7 @@ struct Deadline {
         return false;
     }
 };
+using Deadline = DeadlineT<SmallArgs>;
 
 // Whether some wait of the launch has given up (after a fence, so that data which depends on a
 // give-up is never taken for good).
@@ -248,16 +251,18 @@ __device__ __forceinline__ bool aborted(const SmallArgs &a) {
     return *(volatile int *)a.abort_flag != 0;
 }
 
-__device__ __forceinline__ void wait_cta(const SmallArgs &a, uint32_t bar, unsigned parity) {
+template <typename A>
+__device__ __forceinline__ void wait_cta(const A &a, uint32_t bar, unsigned parity) {
     if (mbar_try(bar, parity)) return;
-    Deadline d{&a, now_ns(), 0};
+    DeadlineT<A> d{&a, now_ns(), 0};
     while (!mbar_try(bar, parity))
         if (d.expired()) return;
 }
 
-__device__ __forceinline__ void wait_cluster(const SmallArgs &a, uint32_t bar, unsigned parity) {
+template <typename A>
+__device__ __forceinline__ void wait_cluster(const A &a, uint32_t bar, unsigned parity) {
     if (mbar_try_cluster(bar, parity)) return;
-    Deadline d{&a, now_ns(), 0};
+    DeadlineT<A> d{&a, now_ns(), 0};
     while (!mbar_try_cluster(bar, parity))
         if (d.expired()) return;
 }
@@ -785,6 +790,73 @@ __global__ void __launch_bounds__(kSThreads, 1) lstm_small_kernel(const __grid_c
     cluster_sync();
 }
 
+// ---- latency floor probe --------------------------------------------------------------------------
+// The per-frame synchronisation skeleton of one layer cluster of lstm_small_kernel with the
+// arithmetic taken out: per round, the 16 product warps of every block wait for the cluster
+// exchange (transaction-count mbarrier), re-arm it and hand over to the 4 epilogue warps (local
+// mbarrier); the epilogue warps send their 40 bytes to every block of the cluster (st.async),
+// which completes the next round's exchange. Its time per round is the floor under the time per
+// frame of a layer, whatever the products and the gate arithmetic cost.
+struct FloorArgs {
+    int rounds;
+    int *status;
+    int *abort_flag;
+    unsigned long long wait_ns;
+};
+
+__global__ void __launch_bounds__(kSThreads, 1) exchange_floor_kernel(const __grid_constant__ FloorArgs f) {
+    __shared__ __align__(16) float hbuf[2][kMaxK];
+    __shared__ __align__(16) float2 hmm[2][kHParts];
+    __shared__ __align__(8) unsigned long long bar_h[2], bar_a[2];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
+    uint32_t CS;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(CS));
+    const uint32_t rank = cluster_rank();
+    const uint32_t hb0 = saddr(&bar_h[0]), ab0 = saddr(&bar_a[0]);
+    const uint32_t bytes = CS * kEW * kHBytes;
+    if (tid == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(hb0 + 8 * i, 1);
+            mbar_init(ab0 + 8 * i, kPW);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        mbar_arrive_expect(hb0, bytes);
+        if (f.rounds > 1) mbar_arrive_expect(hb0 + 8, bytes);
+    }
+    __syncthreads();
+    cluster_sync();
+    if (warp < kPW) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(ab0);  // round 0 may start
+        for (int t = 0; t < f.rounds; ++t) {
+            const int par = t & 1;
+            wait_cluster(f, hb0 + 8 * par, (t >> 1) & 1);
+            if (tid == 0 && t + 2 < f.rounds) mbar_arrive_expect(hb0 + 8 * par, bytes);
+            __syncwarp();
+            if (lane == 0 && t + 1 < f.rounds) mbar_arrive(ab0 + 8 * (par ^ 1));
+        }
+    } else if (warp < kPW + kEW) {
+        const int ew = warp - kPW;
+        const uint32_t hbuf_l = saddr(&hbuf[0][0]), hmm_l = saddr(&hmm[0][0]);
+        for (int t = 0; t < f.rounds; ++t) {
+            const int par = t & 1;
+            wait_cta(f, ab0 + 8 * par, (t >> 1) & 1);
+            if (lane < (int)CS) {
+                const float v = (float)t;
+                const uint32_t rbar = map_rank(hb0 + 8 * par, lane);
+                const uint32_t dst = map_rank(hbuf_l + 4u * (uint32_t)(par * kMaxK + rank * kCellsPerBlock + 8 * ew), lane);
+                st_async_v4(dst, make_float4(v, v, v, v), rbar);
+                st_async_v4(dst + 16u, make_float4(v, v, v, v), rbar);
+                st_async_v2(map_rank(hmm_l + 8u * (uint32_t)(par * kHParts + rank * kEW + ew), lane), v, v, rbar);
+            }
+        }
+    }
+    __syncwarp();
+    if (*(volatile int *)f.abort_flag)
+        for (int i = 0; i < 100; ++i) __nanosleep(100000);
+    cluster_sync();
+}
+
 int g_small_cfg_dev = -1;
 
 // Launch geometry of the kernel for model m at batch B; false when the model or batch does not
@@ -1003,3 +1075,53 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
 }
 
 }  // namespace qnn
+
+// Time per round of the batch-of-few kernel's per-frame synchronisation skeleton on one cluster of
+// cluster_size blocks (exchange_floor_kernel). Synchronous; best of three timed launches.
+extern "C" qnn_status qnn_measure_exchange_floor(int32_t cluster_size, int32_t rounds, double *us_per_round) {
+    using namespace qnn;
+    if (!us_per_round || cluster_size < 1 || cluster_size > kMaxCS || rounds < 1 || rounds > 1000000)
+        return QNN_ERR_INVALID_ARG;
+    QNN_CUDA_TRY(cudaFuncSetAttribute(exchange_floor_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)cluster_size);
+    cfg.blockDim = dim3(kSThreads);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)cluster_size;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int max_clusters = 0;
+    QNN_CUDA_TRY(cudaOccupancyMaxActiveClusters(&max_clusters, exchange_floor_kernel, &cfg));
+    if (max_clusters < 1) return QNN_ERR_NO_COOP;
+    int *words = nullptr;  // status, abort flag
+    QNN_CUDA_TRY(cudaMalloc(&words, 2 * sizeof(int)));
+    QNN_CUDA_TRY(cudaMemset(words, 0, 2 * sizeof(int)));
+    FloorArgs f{rounds, words, words + 1, kWaitNs};
+    cudaEvent_t e0, e1;
+    QNN_CUDA_TRY(cudaEventCreate(&e0));
+    QNN_CUDA_TRY(cudaEventCreate(&e1));
+    double best = 1e30;
+    qnn_status result = QNN_OK;
+    for (int rep = 0; rep < 4 && result == QNN_OK; ++rep) {
+        if (cudaEventRecord(e0) != cudaSuccess || cudaLaunchKernelEx(&cfg, exchange_floor_kernel, f) != cudaSuccess ||
+            cudaEventRecord(e1) != cudaSuccess || cudaEventSynchronize(e1) != cudaSuccess) {
+            result = QNN_ERR_CUDA;
+            break;
+        }
+        float ms = 0.0f;
+        cudaEventElapsedTime(&ms, e0, e1);
+        if (rep > 0) best = std::min(best, 1e3 * ms / rounds);
+    }
+    int st = 0;
+    if (result == QNN_OK && cudaMemcpy(&st, words, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+        result = QNN_ERR_CUDA;
+    if (result == QNN_OK && st != 0) result = (qnn_status)st;
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    cudaFree(words);
+    if (result == QNN_OK) *us_per_round = best;
+    return result;
+}

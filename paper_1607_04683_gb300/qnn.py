@@ -34,7 +34,7 @@ EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmu
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
            "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static",
            "qnn_selftest_s64_to_f32", "qnn_stack_frames", "qnn_selftest_wait_timeout", "qnn_lstm_stream_open",
-           "qnn_lstm_stream_push", "qnn_lstm_stream_pull", "qnn_lstm_stream_close")
+           "qnn_lstm_stream_push", "qnn_lstm_stream_pull", "qnn_lstm_stream_close", "qnn_measure_exchange_floor")
 
 
 class QnnError(RuntimeError):
@@ -91,6 +91,8 @@ def lib():
         L.qnn_selftest_wait_timeout.restype = i32
         L.qnn_stack_frames.restype = i32
         L.qnn_selftest_s64_to_f32.restype = i32
+        L.qnn_measure_exchange_floor.argtypes = [i32, i32, C.POINTER(C.c_double)]
+        L.qnn_measure_exchange_floor.restype = i32
         L.qnn_lstm_stream_open.argtypes = [P, i64, i64, C.c_double, C.POINTER(P)]
         L.qnn_lstm_stream_open.restype = i32
         L.qnn_lstm_stream_push.argtypes = [P, P, i64]
@@ -113,6 +115,14 @@ def measure_peak(kind: int) -> float:
     """Measured peak TOPS of an integer datapath: 0 = mma.sync u8 tensor-core MMA, 1 = dp4a."""
     v = C.c_double(0.0)
     _check(lib().qnn_measure_peak(kind, C.byref(v)), "qnn_measure_peak")
+    return v.value
+
+
+def measure_exchange_floor(cluster_size: int, rounds: int = 20000) -> float:
+    """Microseconds per round of the batch-of-few recurrence's per-frame synchronisation skeleton
+    (no arithmetic) on one cluster of cluster_size blocks: the floor under a layer's time per frame."""
+    v = C.c_double(0.0)
+    _check(lib().qnn_measure_exchange_floor(cluster_size, rounds, C.byref(v)), "qnn_measure_exchange_floor")
     return v.value
 
 
