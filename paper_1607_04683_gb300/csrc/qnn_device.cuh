@@ -160,31 +160,33 @@ __device__ __forceinline__ unsigned long long global_timer_ns() {
 
 // Wait for the phase with the given parity of a shared-memory mbarrier, for at most limit_ns: on
 // time-out, record QNN_ERR_TIMEOUT and return false (the caller then skips ahead, so the kernel
-// ends and the host reads the status instead of finding the GPU hung).
+// ends and the host reads the status instead of finding the GPU hung). After a first test, each
+// further test lets the thread be suspended until the phase completes, for at most kSuspendNs
+// (mbarrier.try_wait's suspend-time hint), so a warp that waits long issues a few instructions per
+// microsecond instead of spinning against the warps that do the work.
+constexpr unsigned kSuspendNs = 1000;
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, unsigned parity, int *status,
                                                   unsigned long long limit_ns) {
-    auto try_wait = [&]() {
-        uint32_t ok;
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-            : "=r"(ok)
-            : "r"(bar), "r"(parity)
-            : "memory");
-        return ok != 0;
-    };
-    if (try_wait()) return true;
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    if (ok) return true;
     const unsigned long long t0 = global_timer_ns();
-    int spins = 0;
-    while (!try_wait()) {
-        if (++spins >= 256) {
-            spins = 0;
-            if (global_timer_ns() - t0 > limit_ns) {
-                record_status(status, QNN_ERR_TIMEOUT);
-                return false;
-            }
+    while (true) {
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity), "r"(kSuspendNs)
+            : "memory");
+        if (ok) return true;
+        if (global_timer_ns() - t0 > limit_ns) {
+            record_status(status, QNN_ERR_TIMEOUT);
+            return false;
         }
     }
-    return true;
 }
 
 // Programmatic dependent launch: a kernel launched with the programmatic stream serialization
