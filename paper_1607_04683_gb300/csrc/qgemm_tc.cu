@@ -106,6 +106,8 @@ struct TcArgs {
     int kbs;         // k-blocks per K range
     int32_t *part;   // kEpiPartial: [splits][M][ldpart] int32
     int64_t ldpart;
+    int w_static;    // W was written before the previous kernel of the stream started (model weights):
+                     // its first tiles may load before the programmatic-launch wait
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
@@ -297,6 +299,24 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem_base = *tmem_slot;
+    // Static weights: the producer starts the W tiles of its first stages before the wait below
+    // (the A tiles, outputs of the previous kernel, follow after it); their barriers expect both.
+    int w_early = 0;
+    if (warp == 0 && lane == 0) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapA)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapW)) : "memory");
+        if (args.w_static && blockIdx.x < items) {
+            int64_t m0, n0;
+            tile_origin(blockIdx.x / splits, tiles_m, tiles_n, BN, m0, n0);
+            const int kb0 = (int)(blockIdx.x % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+            w_early = min(STAGES, kb1 - kb0);
+            for (int j = 0; j < w_early; ++j) {
+                const uint32_t sb = su32(smem + j * TL::STAGE_BYTES) + A_BYTES;
+                mb_expect(full0 + 8 * j, TL::STAGE_BYTES);
+                tma_load_2d(sb, &mapW, full0 + 8 * j, (kb0 + j) * TBK, n0);
+            }
+        }
+    }
     // With a programmatic dependent launch the setup above overlaps the previous kernel of the
     // stream; its outputs (this kernel's operands) are complete and visible after this wait.
     grid_dependency_wait();
@@ -320,6 +340,10 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         break;
                     }
                     const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
+                    if (g < w_early) {  // W already on its way (expect set with it)
+                        tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
+                        continue;
+                    }
                     mb_expect(full0 + 8 * s, TL::STAGE_BYTES);
                     tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
                     tma_load_2d(sb, &mapW, full0 + 8 * s, kb * TBK, n0);
@@ -946,7 +970,7 @@ qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int3
     int *status = nullptr;
     QNN_TRY(status_word(&status));
     TcArgs a{pa, 1, rsA, pw4, 0, cs, nullptr, nullptr, 0, nullptr, op.M, op.N, (int)K, (int)(op.kp / TBK), status, out,
-             1, (int)(op.kp / TBK), nullptr, 0};
+             1, (int)(op.kp / TBK), nullptr, 0, 1};
     return dispatch_lstm(op, a, st);
 }
 
@@ -968,7 +992,7 @@ qnn_status tc_partial(const TcOperands &op, int splits, int32_t *part, int64_t l
     int *status = nullptr;
     QNN_TRY(status_word(&status));
     TcArgs a{nullptr, 0, nullptr, nullptr, 0, nullptr, nullptr, nullptr, 0, nullptr, op.M, op.N, 0, KB, status,
-             TcLstmOut{}, splits, kbs, part, ldpart};
+             TcLstmOut{}, splits, kbs, part, ldpart, 1};
     return op.bn == 64 ? launch_tc<64, kEpiPartial>(op, a, "qgemm_tc_partial", st)
                        : launch_tc<128, kEpiPartial>(op, a, "qgemm_tc_partial", st);
 }
