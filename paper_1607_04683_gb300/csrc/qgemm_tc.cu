@@ -39,12 +39,12 @@ constexpr unsigned long long TC_WAIT_NS = 2000000000ull;
 
 // kEpiLinear: recovered product, any K (chunked drains), outputs staged through shared memory.
 // kEpiRow: recovered product for K <= 1024, one output row per lane, two blocks per SM.
-// kEpiLstm: the LSTM cell update on gate-interleaved columns, K <= 1024; kEpiLstmEarly the same
-// with the accumulator-independent loads issued before the accumulator wait (a block with a single
-// tile has no earlier epilogue to overlap them with).
+// kEpiLstm: the LSTM cell update on gate-interleaved columns, K <= 1024. (Issuing its input-product
+// and cell-state loads before the accumulator wait was measured slower even for single-tile grids:
+// those HBM loads delay the tile's TMA stream.)
 // kEpiPartial: split-K, each work item (tile, K range of at most 1024) stores its exact centered
 // integer sums P as int32 into its own slice of a partial-sum buffer; a consumer adds the slices.
-enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiLstmEarly = 3, kEpiPartial = 4 };
+enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiPartial = 4 };
 
 struct ColConst {  // per-output-column constants of kEpiRow, staged in shared memory per tile
     int cs, zw;
@@ -64,7 +64,7 @@ template <int BN, int EPI>
 struct Tile {
     static_assert(EPI == kEpiLinear || BN <= 128, "row and LSTM epilogues take tiles of at most 128 columns");
     // a 96-column LSTM tile has six 4-cell slices per lane quarter: 24 epilogue warps, one slice each
-    static constexpr bool LSTM96 = (EPI == kEpiLstm || EPI == kEpiLstmEarly) && BN == 96;
+    static constexpr bool LSTM96 = EPI == kEpiLstm && BN == 96;
     static constexpr int EPI_WARPS = EPI == kEpiLinear ? 8 : (LSTM96 ? 24 : 16);
     // LSTM: cells per epilogue slice (a 32-column tile has 8 cells: 2-cell slices keep 4 warps busy)
     static constexpr int CPS = BN == 32 ? 2 : 4;
@@ -78,7 +78,7 @@ struct Tile {
     // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : (LSTM96 ? 72 : 96);
-    static constexpr int EPI_BYTES = EPI == kEpiLstm || EPI == kEpiLstmEarly || EPI == kEpiPartial
+    static constexpr int EPI_BYTES = EPI == kEpiLstm || EPI == kEpiPartial
                                          ? 0
                                          : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
     static constexpr uint32_t IDESC =
@@ -679,16 +679,6 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             }
             const int za128 = 128 + za;
             const int buf = (int)(gc & 1);
-            // this warp's first slice: the input products and cell state do not depend on the
-            // accumulator, so they may be loaded before waiting for it
-            const int s0 = EPI == kEpiLstmEarly ? eh : -1;
-            float px0[4][CPS], c0v[CPS];
-            const int j00 = (int)(n0 / 4) + (eh / SPG) * 8 + (eh % SPG) * CPS;
-            if (EPI == kEpiLstmEarly && eh < SLICES && bv && j00 < H) {
-#pragma unroll
-                for (int g = 0; g < 4; ++g) ld_vec(E.px + b * E.px_ld + j00 + (int64_t)g * H, px0[g]);
-                ld_vec(E.c + b * (int64_t)H + j00, c0v);
-            }
             ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -720,12 +710,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     for (int g = 0; g < 4; ++g) {
                         float pv[CPS];
                         int csv[CPS];
-                        if (s == s0) {
-#pragma unroll
-                            for (int jj = 0; jj < CPS; ++jj) pv[jj] = px0[g][jj];
-                        } else {
-                            ld_vec(pxr + (int64_t)g * H, pv);
-                        }
+                        ld_vec(pxr + (int64_t)g * H, pv);
                         ld_vec(args.csW + g * H + j0, csv);
 #pragma unroll
                         for (int jj = 0; jj < CPS; ++jj) {
@@ -735,12 +720,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         }
                     }
                     float cv[CPS], mv[CPS];
-                    if (s == s0) {
-#pragma unroll
-                        for (int jj = 0; jj < CPS; ++jj) cv[jj] = c0v[jj];
-                    } else {
-                        ld_vec(cr, cv);
-                    }
+                    ld_vec(cr, cv);
 #pragma unroll
                     for (int jj = 0; jj < CPS; ++jj) lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
                     st_vec(cr, cv);
@@ -885,16 +865,6 @@ qnn_status dispatch_linear(const TcOperands &op, const TcArgs &a, cudaStream_t s
 }
 
 qnn_status dispatch_lstm(const TcOperands &op, const TcArgs &a, cudaStream_t st) {
-    const int64_t tiles = ((a.M + TBM - 1) / TBM) * ((a.N + op.bn - 1) / op.bn);
-    if (tiles <= sm_count()) {
-        switch (op.bn) {
-            case 32: return launch_tc<32, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
-            case 64: return launch_tc<64, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
-            case 96: return launch_tc<96, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
-            case 128: return launch_tc<128, kEpiLstmEarly>(op, a, "lstm_gates_tc", st);
-            default: return QNN_ERR_INVALID_ARG;
-        }
-    }
     switch (op.bn) {
         case 32: return launch_tc<32, kEpiLstm>(op, a, "lstm_gates_tc", st);
         case 64: return launch_tc<64, kEpiLstm>(op, a, "lstm_gates_tc", st);
