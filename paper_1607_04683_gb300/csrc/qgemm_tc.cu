@@ -70,10 +70,17 @@ struct Tile {
     static constexpr int CPS = BN == 32 ? 2 : 4;
     static constexpr int THREADS = 32 * (2 + EPI_WARPS);
     static constexpr int B_BYTES = BN * TBK * 2;
-    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
-                                  : EPI == kEpiPartial ? 6  // one K range per item: keep it all in flight
-                                                       : (BN == 128 ? 4 : 6);
+    // a pipeline stage carries KPS consecutive k-blocks (A sub-tiles first, then the W sub-tiles):
+    // the operand stream advances by stages at a pace that hardly depends on their size, so narrow
+    // LSTM tiles (small stages, one tile per SM) take two k-blocks a stage; wider tiles keep more,
+    // smaller stages in flight (measured both ways on GB300)
+    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 2 : 1;
+    static constexpr int SUB_BYTES = A_BYTES + B_BYTES;
+    static constexpr int STAGE_BYTES = KPS * SUB_BYTES;
+    static constexpr int STAGES = (EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
+                                   : EPI == kEpiPartial ? 6  // one K range per item: keep it all in flight
+                                                        : (BN == 128 ? 4 : 6)) /
+                                  KPS;
     static constexpr int TMEM_COLS = 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
     // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
@@ -309,11 +316,22 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             int64_t m0, n0;
             tile_origin(blockIdx.x / splits, tiles_m, tiles_n, BN, m0, n0);
             const int kb0 = (int)(blockIdx.x % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
-            w_early = min(STAGES, kb1 - kb0);
-            for (int j = 0; j < w_early; ++j) {
-                const uint32_t sb = su32(smem + j * TL::STAGE_BYTES) + A_BYTES;
-                mb_expect(full0 + 8 * j, TL::STAGE_BYTES);
-                tma_load_2d(sb, &mapW, full0 + 8 * j, (kb0 + j) * TBK, n0);
+            if constexpr (TL::KPS == 1) {
+                w_early = min(STAGES, kb1 - kb0);
+                for (int j = 0; j < w_early; ++j) {
+                    const uint32_t sb = su32(smem + j * TL::STAGE_BYTES) + A_BYTES;
+                    mb_expect(full0 + 8 * j, TL::STAGE_BYTES);
+                    tma_load_2d(sb, &mapW, full0 + 8 * j, (kb0 + j) * TBK, n0);
+                }
+            } else {
+                w_early = min(STAGES, (kb1 - kb0 + TL::KPS - 1) / TL::KPS);
+                for (int j = 0; j < w_early; ++j) {
+                    const int kbj = kb0 + j * TL::KPS, nv = min(TL::KPS, kb1 - kbj);
+                    const uint32_t sb = su32(smem + j * TL::STAGE_BYTES) + TL::KPS * A_BYTES;
+                    mb_expect(full0 + 8 * j, (uint32_t)(nv * TL::SUB_BYTES));
+                    for (int v = 0; v < nv; ++v)
+                        tma_load_2d(sb + v * TL::B_BYTES, &mapW, full0 + 8 * j, (kbj + v) * TBK, n0);
+                }
             }
         }
     }
@@ -327,64 +345,165 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     // epilogue overlaps the next tile's MMAs.
     if (warp == 0) {
         // ---------------- TMA producer ----------------
-        if (lane == 0) {
-            int64_t g = 0;  // k-blocks issued by this block
-            for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
-                int64_t m0, n0;
-                tile_origin(item / splits, tiles_m, tiles_n, BN, m0, n0);
-                const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
-                for (int kb = kb0; kb < kb1; ++kb, ++g) {
-                    const int s = (int)(g % STAGES);
-                    if (g >= STAGES && !mb_wait(empty0 + 8 * s, (unsigned)((g / STAGES) - 1) & 1, args.status)) {
-                        s_abort = 1;
-                        break;
-                    }
-                    const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
-                    if (g < w_early) {  // W already on its way (expect set with it)
+        if constexpr (TL::KPS == 1) {
+            if (lane == 0) {
+                int64_t g = 0;  // k-blocks issued by this block
+                for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
+                    int64_t m0, n0;
+                    tile_origin(item / splits, tiles_m, tiles_n, BN, m0, n0);
+                    const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                    for (int kb = kb0; kb < kb1; ++kb, ++g) {
+                        const int s = (int)(g % STAGES);
+                        if (g >= STAGES && !mb_wait(empty0 + 8 * s, (unsigned)((g / STAGES) - 1) & 1, args.status)) {
+                            s_abort = 1;
+                            break;
+                        }
+                        const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
+                        if (g < w_early) {  // W already on its way (expect set with it)
+                            tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
+                            continue;
+                        }
+                        mb_expect(full0 + 8 * s, TL::STAGE_BYTES);
                         tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
-                        continue;
+                        tma_load_2d(sb, &mapW, full0 + 8 * s, kb * TBK, n0);
                     }
-                    mb_expect(full0 + 8 * s, TL::STAGE_BYTES);
-                    tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
-                    tma_load_2d(sb, &mapW, full0 + 8 * s, kb * TBK, n0);
+                }
+            }
+        } else {
+            if (lane == 0) {
+                // One thread issues every copy; its loop is on the critical path of the operand stream,
+                // so the ring position (slot, phase, shared-memory address) advances incrementally in
+                // 32-bit registers instead of being derived from a 64-bit counter every stage.
+                const uint32_t ring0 = su32(smem);
+                int slot = 0, issued = 0;  // ring slot; stages issued (saturating at STAGES)
+                unsigned phase = 0;        // parity of the slot's current use
+                uint32_t st_addr = ring0, bar_full = full0, bar_empty = empty0;
+                for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
+                    int64_t m0l, n0l;
+                    tile_origin(item / splits, tiles_m, tiles_n, BN, m0l, n0l);
+                    const int m0 = (int)m0l, n0 = (int)n0l;
+                    const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                    for (int kb = kb0; kb < kb1; kb += TL::KPS) {
+                        if (issued >= STAGES && !mb_wait(bar_empty, phase ^ 1u, args.status)) {
+                            s_abort = 1;
+                            break;
+                        }
+                        const int nv = min(TL::KPS, kb1 - kb);  // k-blocks in this stage (the last may be short)
+                        const uint32_t sb = st_addr + TL::KPS * A_BYTES;
+                        const bool w_sent = issued < w_early;   // W already on its way (expect set with it)
+                        if (!w_sent) mb_expect(bar_full, (uint32_t)(nv * TL::SUB_BYTES));
+    #pragma unroll
+                        for (int v = 0; v < TL::KPS; ++v) {
+                            if (v >= nv) break;
+                            tma_load_2d(st_addr + v * A_BYTES, &mapA, bar_full, (kb + v) * TBK, m0);
+                            if (!w_sent) tma_load_2d(sb + v * TL::B_BYTES, &mapW, bar_full, (kb + v) * TBK, n0);
+                        }
+                        if (issued < STAGES) ++issued;
+                        if (++slot == STAGES) {
+                            slot = 0;
+                            phase ^= 1u;
+                            st_addr = ring0, bar_full = full0, bar_empty = empty0;
+                        } else {
+                            st_addr += TL::STAGE_BYTES, bar_full += 8, bar_empty += 8;
+                        }
+                    }
                 }
             }
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
-        if (lane == 0) {
-            int64_t g = 0, gc = 0;  // k-blocks and chunks consumed by this block
-            for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
-                const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
-                for (int kb = kb0; kb < kb1; ++kb, ++g) {
-                    const int s = (int)(g % STAGES);
-                    const int kc = (kb - kb0) % kpc;
-                    const int buf = (int)(gc & 1);
-                    if (kc == 0 && gc >= 2 &&
-                        !mb_wait(drained0 + 8 * buf, (unsigned)((gc / 2) - 1) & 1, args.status)) {  // buffer free
-                        s_abort = 1;
-                        break;
+        if constexpr (TL::KPS == 1) {
+            if (lane == 0) {
+                int64_t g = 0, gc = 0;  // k-blocks and chunks consumed by this block
+                for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
+                    const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                    for (int kb = kb0; kb < kb1; ++kb, ++g) {
+                        const int s = (int)(g % STAGES);
+                        const int kc = (kb - kb0) % kpc;
+                        const int buf = (int)(gc & 1);
+                        if (kc == 0 && gc >= 2 &&
+                            !mb_wait(drained0 + 8 * buf, (unsigned)((gc / 2) - 1) & 1, args.status)) {  // buffer free
+                            s_abort = 1;
+                            break;
+                        }
+                        if (!mb_wait(full0 + 8 * s, (unsigned)(g / STAGES) & 1, args.status)) {
+                            s_abort = 1;
+                            break;
+                        }
+                        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                        const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
+                        const uint32_t tmem_d = tmem_base + (uint32_t)(buf * BN);
+    #pragma unroll
+                        for (int k = 0; k < TBK / 16; ++k) {
+                            // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
+                            mma_f16<TL::IDESC>(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k),
+                                               (kc == 0 && k == 0) ? 0u : 1u);
+                        }
+                        mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
+                        if (kc == kpc - 1 || kb == kb1 - 1) {
+                            mma_commit(chunk0 + 8 * buf);
+                            ++gc;
+                        }
                     }
-                    if (!mb_wait(full0 + 8 * s, (unsigned)(g / STAGES) & 1, args.status)) {
-                        s_abort = 1;
-                        break;
-                    }
-                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                    const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
-                    const uint32_t tmem_d = tmem_base + (uint32_t)(buf * BN);
-#pragma unroll
-                    for (int k = 0; k < TBK / 16; ++k) {
-                        // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
-                        mma_f16<TL::IDESC>(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k),
-                                           (kc == 0 && k == 0) ? 0u : 1u);
-                    }
-                    mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
-                    if (kc == kpc - 1 || kb == kb1 - 1) {
-                        mma_commit(chunk0 + 8 * buf);
-                        ++gc;
-                    }
+                    if (s_abort) break;
                 }
-                if (s_abort) break;
+            }
+        } else {
+            if (lane == 0) {
+                // The same incremental ring position as the producer's; the shared-memory descriptors of
+                // a stage are its base descriptor plus the byte offset / 16 in the address field (the
+                // address stays below 2^18, so the 14-bit field never carries).
+                const uint32_t ring0 = su32(smem);
+                int slot = 0;
+                unsigned phase = 0;
+                uint32_t st_addr = ring0, bar_full = full0, bar_empty = empty0;
+                int64_t gc = 0;  // chunks accumulated by this block
+                for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
+                    const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                    int kc = 0;  // position of the stage in its K chunk (chunks hold whole stages)
+                    for (int kb = kb0; kb < kb1; kb += TL::KPS) {
+                        const int nv = min(TL::KPS, kb1 - kb);
+                        const int buf = (int)(gc & 1);
+                        if (kc == 0 && gc >= 2 &&
+                            !mb_wait(drained0 + 8 * buf, (unsigned)((gc / 2) - 1) & 1, args.status)) {  // buffer free
+                            s_abort = 1;
+                            break;
+                        }
+                        if (!mb_wait(bar_full, phase, args.status)) {
+                            s_abort = 1;
+                            break;
+                        }
+                        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                        const uint64_t da = smem_desc(st_addr), db = smem_desc(st_addr + TL::KPS * A_BYTES);
+                        const uint32_t tmem_d = tmem_base + (uint32_t)(buf * BN);
+    #pragma unroll
+                        for (int v = 0; v < TL::KPS; ++v) {
+                            if (v >= nv) break;
+    #pragma unroll
+                            for (int k = 0; k < TBK / 16; ++k) {
+                                // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
+                                mma_f16<TL::IDESC>(tmem_d, da + (uint64_t)((v * A_BYTES + 32 * k) >> 4),
+                                                   db + (uint64_t)((v * TL::B_BYTES + 32 * k) >> 4),
+                                                   (kc == 0 && v == 0 && k == 0) ? 0u : 1u);
+                            }
+                        }
+                        mma_commit(bar_empty);  // frees the stage when these MMAs have read it
+                        kc += nv;
+                        if (kc >= kpc || kb + nv >= kb1) {
+                            mma_commit(chunk0 + 8 * buf);
+                            ++gc;
+                            kc = 0;
+                        }
+                        if (++slot == STAGES) {
+                            slot = 0;
+                            phase ^= 1u;
+                            st_addr = ring0, bar_full = full0, bar_empty = empty0;
+                        } else {
+                            st_addr += TL::STAGE_BYTES, bar_full += 8, bar_empty += 8;
+                        }
+                    }
+                    if (s_abort) break;
+                }
             }
         }
     } else if constexpr (EPI == kEpiLinear) {
