@@ -72,15 +72,15 @@ struct Tile {
     static constexpr int B_BYTES = BN * TBK * 2;
     // a pipeline stage carries KPS consecutive k-blocks (A sub-tiles first, then the W sub-tiles):
     // the operand stream advances by stages at a pace that hardly depends on their size, so narrow
-    // LSTM tiles (small stages, one tile per SM) take two k-blocks a stage; wider tiles keep more,
-    // smaller stages in flight (measured both ways on GB300)
-    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 2 : 1;
+    // LSTM tiles (small stages, one tile per SM) take four k-blocks a stage (two stages in flight);
+    // wider tiles keep more, smaller stages in flight (measured each way on GB300)
+    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 4 : 1;
     static constexpr int SUB_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGE_BYTES = KPS * SUB_BYTES;
-    static constexpr int STAGES = (EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
-                                   : EPI == kEpiPartial ? 6  // one K range per item: keep it all in flight
-                                                        : (BN == 128 ? 4 : 6)) /
-                                  KPS;
+    static constexpr int BASE_STAGES = EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
+                                       : EPI == kEpiPartial ? 6  // one K range per item: keep it all in flight
+                                                            : (BN == 128 ? 4 : 6);
+    static constexpr int STAGES = BASE_STAGES / KPS < 2 ? 2 : BASE_STAGES / KPS;
     static constexpr int TMEM_COLS = 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
     // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
