@@ -74,7 +74,7 @@ struct Tile {
     // the operand stream advances by stages at a pace that hardly depends on their size, so narrow
     // LSTM tiles (small stages, one tile per SM) take four k-blocks a stage (two stages in flight);
     // wider tiles keep more, smaller stages in flight (measured each way on GB300)
-    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 4 : 1;
+    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 4 : (EPI == kEpiPartial ? 2 : 1);
     static constexpr int SUB_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGE_BYTES = KPS * SUB_BYTES;
     static constexpr int BASE_STAGES = EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
