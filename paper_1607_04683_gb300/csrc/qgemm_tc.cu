@@ -71,10 +71,11 @@ struct Tile {
     static constexpr int THREADS = 32 * (2 + EPI_WARPS);
     static constexpr int B_BYTES = BN * TBK * 2;
     // a pipeline stage carries KPS consecutive k-blocks (A sub-tiles first, then the W sub-tiles):
-    // the operand stream advances by stages at a pace that hardly depends on their size, so narrow
-    // LSTM tiles (small stages, one tile per SM) take four k-blocks a stage (two stages in flight);
-    // wider tiles keep more, smaller stages in flight (measured each way on GB300)
-    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 4 : (EPI == kEpiPartial ? 2 : 1);
+    // the operand stream advances by stages at a pace that hardly depends on their size, so short
+    // reductions (K <= 1024) take several k-blocks a stage: four for narrow LSTM tiles (two stages in
+    // flight), two for row tiles and split-K items; the long-K linear tiles and the 96-column LSTM
+    // tiles keep more, smaller stages in flight (each choice measured on GB300)
+    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 4 : ((EPI == kEpiPartial || EPI == kEpiRow) ? 2 : 1);
     static constexpr int SUB_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGE_BYTES = KPS * SUB_BYTES;
     static constexpr int BASE_STAGES = EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
