@@ -398,6 +398,20 @@ def test_tc_recurrence_bit_exact(qnn, cfg, bn, monkeypatch):
     _compare(got, ref, wl)
 
 
+@pytest.mark.parametrize("bn", ["32", "96"])
+def test_tc_recurrence_large_weight_offsets(qnn, bn, monkeypatch):
+    # every weight shifted by +20: weight ranges far from zero give offsets z of about 32000, so
+    # K |a' + za| |w' + zw| exceeds 2^31 and the gate epilogue sums S in 64 bits
+    wl = _small(L=1, I=40, H=128, B=70, T=3, w=0.08)
+    params, x = wl.make()
+    params = (params + np.float32(20.0)).astype(np.float32)
+    ref = _oracle(wl, params, x, want_h_all=True)
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    monkeypatch.setenv("QNN_TC_BN", bn)
+    got = _gpu_forward(qnn, wl, params, x)
+    _compare(got, ref, wl)
+
+
 def test_tc_recurrence_state_round_trip(qnn, monkeypatch):
     """Streaming: two calls on halves of the frames give the single call's outputs and state."""
     monkeypatch.setenv("QNN_LSTM_PATH", "tc")
