@@ -75,20 +75,29 @@ struct Tile {
     // reductions (K <= 1024) take several k-blocks a stage: four for narrow LSTM tiles (two stages in
     // flight), two for row tiles and split-K items; the long-K linear tiles and the 96-column LSTM
     // tiles keep more, smaller stages in flight (each choice measured on GB300)
-    static constexpr int KPS = (EPI == kEpiLstm && BN <= 64) ? 4 : ((EPI == kEpiPartial || EPI == kEpiRow) ? 2 : 1);
+    static constexpr int KPS = EPI == kEpiLstm ? (BN <= 32 ? 4 : (BN == 64 ? 2 : 1))
+                                               : ((EPI == kEpiPartial || EPI == kEpiRow) ? 2 : 1);
     static constexpr int SUB_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGE_BYTES = KPS * SUB_BYTES;
     static constexpr int BASE_STAGES = EPI == kEpiLinear    ? (BN == 256 ? 4 : 6)
                                        : EPI == kEpiPartial ? 6  // one K range per item: keep it all in flight
                                                             : (BN == 128 ? 4 : 6);
-    static constexpr int STAGES = BASE_STAGES / KPS < 2 ? 2 : BASE_STAGES / KPS;
+    // LSTM: the tile's input products px (4 gates x 128 rows x BN/4 cells) and cell state c (128 x
+    // BN/4), fp32, double-buffered in shared memory after the stages
+    static constexpr int PX_BOX = TBM * (BN / 4) * 4;  // one gate's px box, bytes
+    static constexpr int LSTM_BUF = 5 * PX_BOX;        // 4 px boxes + the c box
+    static constexpr int EPI_BYTES = EPI == kEpiLstm      ? 2 * LSTM_BUF
+                                     : EPI == kEpiPartial ? 0
+                                                          : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
+    static constexpr int SMEM_CAP = 227 * 1024 - 1024 - 256;  // dynamic shared memory left for stages + EPI_BYTES
+    static constexpr int FIT_STAGES = (SMEM_CAP - EPI_BYTES) / STAGE_BYTES;
+    static constexpr int WANT_STAGES = BASE_STAGES / KPS < 2 ? 2 : BASE_STAGES / KPS;
+    static constexpr int STAGES = WANT_STAGES < FIT_STAGES ? WANT_STAGES : FIT_STAGES;
+    static_assert(STAGES >= 2, "at least two pipeline stages must fit");
     static constexpr int TMEM_COLS = 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
     // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : (LSTM96 ? 72 : 96);
-    static constexpr int EPI_BYTES = EPI == kEpiLstm || EPI == kEpiPartial
-                                         ? 0
-                                         : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
     static constexpr uint32_t IDESC =
         (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TBM >> 4) << 24);
     static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + EPI_BYTES + 256;
@@ -262,6 +271,7 @@ __device__ __forceinline__ void row_block_fast(const uint32_t (&r)[16], const Co
 template <int BN, int EPI>
 __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN, EPI>::MAX_REGS))
     qgemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapW,
+                    const __grid_constant__ CUtensorMap mapPX, const __grid_constant__ CUtensorMap mapC,
                     const TcArgs args) {
     using TL = Tile<BN, EPI>;
     constexpr int STAGES = TL::STAGES;
@@ -269,9 +279,11 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     // 1024-byte alignment for the swizzled tiles
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + STAGES * TL::STAGE_BYTES + TL::EPI_BYTES);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 4);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * STAGES + 8);
     const uint32_t full0 = su32(bars), empty0 = su32(bars + STAGES), chunk0 = su32(bars + 2 * STAGES),
                    drained0 = su32(bars + 2 * STAGES + 2);
+    // LSTM only: px/c buffer i loaded (pxfull0 + 8 i) and released by every epilogue warp (pxempty0 + 8 i)
+    const uint32_t pxfull0 = su32(bars + 2 * STAGES + 4), pxempty0 = su32(bars + 2 * STAGES + 6);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int KB = args.KB;
     const int kpc = KCHUNK / TBK;  // k-blocks per chunk (16)
@@ -293,6 +305,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         for (int i = 0; i < 2; ++i) {
             mb_init(chunk0 + 8 * i, 1);      // MMA -> epilogue: chunk accumulated in buffer i
             mb_init(drained0 + 8 * i, TL::EPI_WARPS);  // epilogue -> MMA: buffer i read out by every epilogue warp
+            mb_init(pxfull0 + 8 * i, 1);
+            mb_init(pxempty0 + 8 * i, TL::EPI_WARPS);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -782,11 +796,35 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         const int K = args.K;
         const TcLstmOut &E = args.lstm;
         const int H = E.H;
+        // px and c of a tile come into shared memory by TMA, two tiles ahead: buffer i % 2 holds
+        // the block's i-th tile; one thread (warp 2, lane 0) refills a buffer once every epilogue
+        // warp has released it, so the loads overlap the arithmetic of the tile in between
+        constexpr int CW = BN / 4;  // cells per tile
+        float *const pxs0 = reinterpret_cast<float *>(smem + STAGES * TL::STAGE_BYTES);
+        const bool issuer = warp == 2 && lane == 0;
+        auto issue_px = [&](int64_t t_issue, int pbuf) {
+            int64_t m1, n1;
+            tile_origin(t_issue, tiles_m, tiles_n, BN, m1, n1);
+            const uint32_t bar = pxfull0 + 8 * pbuf;
+            const uint32_t dst = su32(pxs0) + (uint32_t)(pbuf * TL::LSTM_BUF);
+            mb_expect(bar, (uint32_t)TL::LSTM_BUF);
+#pragma unroll
+            for (int g = 0; g < 4; ++g)
+                tma_load_2d(dst + g * TL::PX_BOX, &mapPX, bar, g * H + (int)(n1 / 4), (int)m1);
+            tma_load_2d(dst + 4 * TL::PX_BOX, &mapC, bar, (int)(n1 / 4), (int)m1);
+        };
+        if (issuer) {
+            if (blockIdx.x < tiles) issue_px(blockIdx.x, 0);
+            if (blockIdx.x + gridDim.x < tiles) issue_px(blockIdx.x + gridDim.x, 1);
+        }
         int64_t gc = 0;
         bool ok = true;
         for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
             int64_t m0, n0;
             tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
+            const int pbuf = (int)(gc & 1);  // this tile's px/c buffer (gc counts the block's tiles)
+            const float *pxb = pxs0 + pbuf * (TL::LSTM_BUF / 4);
+            const int rl = 32 * q + lane;    // row within the tile
             const int64_t b = m0 + 32 * q + lane;
             const bool bv = b < args.M;
             int za = 0, rs = 0;
@@ -799,7 +837,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             }
             const int za128 = 128 + za;
             const int buf = (int)(gc & 1);
-            ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status));
+            ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status) &&
+                                             mb_wait(pxfull0 + 8 * pbuf, (unsigned)(gc / 2) & 1, args.status));
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll 1
@@ -831,14 +870,15 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         if (BN <= 64)
                             fits &= (long long)K * amax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31);
                     }
-                    const float *pxr = E.px + b * E.px_ld + j0;
+                    const int jt = j0 - (int)(n0 / 4);  // cell within the tile
+                    const float *pxr = pxb + rl * CW + jt;
                     float *cr = E.c + b * (int64_t)H + j0;
                     float pre[4][CPS];
 #pragma unroll
                     for (int g = 0; g < 4; ++g) {
                         float pv[CPS];
                         int csv[CPS];
-                        ld_vec(pxr + (int64_t)g * H, pv);
+                        ld_vec(pxr + g * (TL::PX_BOX / 4), pv);
                         ld_vec(args.csW + g * H + j0, csv);
 #pragma unroll
                         for (int jj = 0; jj < CPS; ++jj) {
@@ -854,7 +894,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         }
                     }
                     float cv[CPS], mv[CPS];
-                    ld_vec(cr, cv);
+                    ld_vec(pxb + 4 * (TL::PX_BOX / 4) + rl * CW + jt, cv);
 #pragma unroll
                     for (int jj = 0; jj < CPS; ++jj) lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
                     st_vec(cr, cv);
@@ -863,9 +903,17 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
-            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+            if (lane == 0) {
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(pxempty0 + 8 * pbuf) : "memory");
+            }
+            // refill the buffer with the tile two ahead once every epilogue warp has released it
+            if (issuer && tile + 2 * (int64_t)gridDim.x < tiles &&
+                mb_wait(pxempty0 + 8 * pbuf, (unsigned)(gc / 2) & 1, args.status))
+                issue_px(tile + 2 * (int64_t)gridDim.x, pbuf);
             ++gc;
         }
+        if (!ok) s_abort = 1;  // copies may still be in flight: the block waits for them before leaving
     }
     __syncwarp();
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -919,6 +967,23 @@ qnn_status get_encode(PFN_cuTensorMapEncodeTiled_v12000 *out) {
     return QNN_OK;
 }
 
+// 2-D fp32 tensor: rows of `cols` values, `ld` values apart (ld a multiple of 4, base 16-byte
+// aligned), boxes of box_cols x box_rows, no swizzle (rows of the box land box_cols * 4 bytes apart).
+qnn_status make_map_f32(CUtensorMap *map, const float *base, int64_t rows, int64_t cols, int64_t ld, int box_cols,
+                        int box_rows) {
+    if ((reinterpret_cast<uintptr_t>(base) & 15) || ld % 4 || box_cols % 4) return QNN_ERR_INVALID_ARG;
+    PFN_cuTensorMapEncodeTiled_v12000 enc = nullptr;
+    QNN_TRY(get_encode(&enc));
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)(ld * 4)};
+    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(base), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? QNN_OK : QNN_ERR_CUDA;
+}
+
 // 2-D fp16 tensor [rows][ld] (ld a multiple of 64), boxes of 64 x box_rows, 128-byte swizzle.
 qnn_status make_map(CUtensorMap *map, const __half *base, int64_t rows, int64_t ld, int box_rows) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = nullptr;
@@ -943,7 +1008,8 @@ size_t tc_scratch_bytes(int64_t M, int64_t N, int64_t K) {
 namespace {
 
 template <int BN, int EPI>
-qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cudaStream_t st) {
+qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cudaStream_t st,
+                     const CUtensorMap *map_px = nullptr, const CUtensorMap *map_c = nullptr) {
     using TL = Tile<BN, EPI>;
     static int configured = -1;
     int dev = 0;
@@ -978,7 +1044,9 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = op.pdl ? 1 : 0;
-    QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, qgemm_tc_kernel<BN, EPI>, op.a, op.w, a));
+    // the px and c maps are read by the LSTM epilogue only (the others get A's map, unused)
+    QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, qgemm_tc_kernel<BN, EPI>, op.a, op.w, map_px ? *map_px : op.a,
+                                    map_c ? *map_c : op.a, a));
     return QNN_OK;
 }
 
@@ -999,11 +1067,16 @@ qnn_status dispatch_linear(const TcOperands &op, const TcArgs &a, cudaStream_t s
 }
 
 qnn_status dispatch_lstm(const TcOperands &op, const TcArgs &a, cudaStream_t st) {
+    // the epilogue's px (B rows of 4H, px_ld apart) and c (B x H) tiles, 128 rows x bn / 4 cells
+    const TcLstmOut &E = a.lstm;
+    CUtensorMap map_px, map_c;
+    QNN_TRY(make_map_f32(&map_px, E.px, a.M, 4 * (int64_t)E.H, E.px_ld, op.bn / 4, TBM));
+    QNN_TRY(make_map_f32(&map_c, E.c, a.M, E.H, E.H, op.bn / 4, TBM));
     switch (op.bn) {
-        case 32: return launch_tc<32, kEpiLstm>(op, a, "lstm_gates_tc", st);
-        case 64: return launch_tc<64, kEpiLstm>(op, a, "lstm_gates_tc", st);
-        case 96: return launch_tc<96, kEpiLstm>(op, a, "lstm_gates_tc", st);
-        case 128: return launch_tc<128, kEpiLstm>(op, a, "lstm_gates_tc", st);
+        case 32: return launch_tc<32, kEpiLstm>(op, a, "lstm_gates_tc", st, &map_px, &map_c);
+        case 64: return launch_tc<64, kEpiLstm>(op, a, "lstm_gates_tc", st, &map_px, &map_c);
+        case 96: return launch_tc<96, kEpiLstm>(op, a, "lstm_gates_tc", st, &map_px, &map_c);
+        case 128: return launch_tc<128, kEpiLstm>(op, a, "lstm_gates_tc", st, &map_px, &map_c);
         default: return QNN_ERR_INVALID_ARG;
     }
 }
