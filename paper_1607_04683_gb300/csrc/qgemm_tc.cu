@@ -855,20 +855,18 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     // with the weight unit of the slice's cells (one per gate matrix, or per block)
                     // S sums K products (a' + za)(w' + zw) of magnitude at most amax * wmax, so when
                     // K amax wmax < 2^31 it fits in 32 bits and wrapping 32-bit arithmetic gives it
-                    // exactly (the usual case: offsets within [-255, 255]); otherwise 64-bit. (Narrow
-                    // tiles only: at 72 registers the 96-column tile measured slower with it.)
+                    // exactly (the usual case: offsets within [-255, 255]); otherwise 64-bit
                     long long rt[4];
                     float den[4];
                     const int unit = j0 / E.cpu;
                     const long long amax = max(abs(za), abs(za + 255));
-                    bool fits = BN <= 64;
+                    bool fits = true;
 #pragma unroll
                     for (int g = 0; g < 4; ++g) {
                         const qnn_qparams qw = args.pw[g * E.ups + unit];
                         rt[g] = (long long)(128 + qw.z) * rs + (long long)K * ((long long)za * qw.z - 16384);
                         den[g] = __fmul_rn(Qa, qw.Q);
-                        if (BN <= 64)
-                            fits &= (long long)K * amax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31);
+                        fits &= (long long)K * amax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31);
                     }
                     const int jt = j0 - (int)(n0 / 4);  // cell within the tile
                     const float *pxr = pxb + rl * CW + jt;
@@ -884,7 +882,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         for (int jj = 0; jj < CPS; ++jj) {
                             const int P = f32_integer_to_s32(__uint_as_float(r[g][jj]));
                             float x;
-                            if (BN <= 64 && fits) {
+                            if (fits) {
                                 const uint32_t u = (uint32_t)P + (uint32_t)rt[g] + (uint32_t)za128 * (uint32_t)csv[jj];
                                 x = __int2float_rn((int)u);
                             } else {
