@@ -99,6 +99,10 @@ def test_tc_large_offsets_bit_exact(qnn, K, monkeypatch):
         assert qnn.device_status() == qnn.QNN_OK
         assert np.array_equal(acc.cpu().numpy(), ref["acc"]), path
         assert np.array_equal(Y.cpu().numpy(), ref["y"]), path
+        # without the raw accumulator the full 16-column blocks take the fast recovery: 32-bit sums
+        # for the ordinary rows, 64-bit ones for the large-offset rows
+        Y2, _ = qnn.qnn_qmatmul(gpu(ca), qnn.params_tensor(pa), 1, gpu(ra), gpu(cw), qnn.params_tensor(pw), gpu(cs))
+        assert np.array_equal(Y2.cpu().numpy(), ref["y"]), path
 
 
 def test_s64_to_f32_rounds_to_nearest_even(qnn):
