@@ -929,20 +929,45 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     }
 }
 
-// u8 codes -> centered fp16 (c - 128), rows padded with zeros to ldo (a multiple of 64).
+// Two codes (bytes lo and hi of w selected by sel) as two centered fp16 values c - 128: the byte
+// placed under the exponent pattern 0x64 is the fp16 value 1024 + c (exact), and 1024 + 128 is
+// then subtracted (exact: integers below 2048).
+__device__ __forceinline__ uint32_t center2(uint32_t w, uint32_t sel) {
+    const uint32_t bits = __byte_perm(w, 0x64646464u, sel);
+    const __half2 v = __hsub2(*reinterpret_cast<const __half2 *>(&bits), __halves2half2(__ushort_as_half(0x6480),
+                                                                                      __ushort_as_half(0x6480)));
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+// u8 codes -> centered fp16 (c - 128), rows padded with zeros to ldo (a multiple of 64). A thread
+// converts 16 codes: one 16-byte load and two 16-byte stores when the row is 16-byte aligned and
+// the 16 codes lie inside K, element by element otherwise (ragged tail, padding, unaligned rows).
 __global__ void center_fp16_kernel(const uint8_t *__restrict__ in, int64_t rows, int K, int64_t ldi,
                                    __half *__restrict__ out, int ldo) {
-    const int64_t total = rows * (int64_t)(ldo / 8);
+    const int per_row = ldo / 16;
+    const int64_t total = rows * (int64_t)per_row;
+    const bool vec = (reinterpret_cast<uintptr_t>(in) & 15) == 0 && ldi % 16 == 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t r = i / (ldo / 8);
-        const int k0 = (int)(i % (ldo / 8)) * 8;
-        __align__(16) __half v[8];
+        const int64_t r = i / per_row;
+        const int k0 = (int)(i - r * per_row) * 16;
+        uint4 o[2];
+        if (vec && k0 + 16 <= K) {
+            const uint4 w = *reinterpret_cast<const uint4 *>(in + r * ldi + k0);
+            o[0] = make_uint4(center2(w.x, 0x4140u), center2(w.x, 0x4342u), center2(w.y, 0x4140u), center2(w.y, 0x4342u));
+            o[1] = make_uint4(center2(w.z, 0x4140u), center2(w.z, 0x4342u), center2(w.w, 0x4140u), center2(w.w, 0x4342u));
+        } else {
+            __align__(16) __half v[16];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const int k = k0 + e;
-            v[e] = k < K ? __int2half_rn((int)in[r * ldi + k] - 128) : __int2half_rn(0);
+            for (int e = 0; e < 16; ++e) {
+                const int k = k0 + e;
+                v[e] = k < K ? __int2half_rn((int)in[r * ldi + k] - 128) : __int2half_rn(0);
+            }
+            o[0] = reinterpret_cast<const uint4 *>(v)[0];
+            o[1] = reinterpret_cast<const uint4 *>(v)[1];
         }
-        *reinterpret_cast<uint4 *>(out + r * ldo + k0) = *reinterpret_cast<const uint4 *>(v);
+        uint4 *dst = reinterpret_cast<uint4 *>(out + r * ldo + k0);
+        dst[0] = o[0];
+        dst[1] = o[1];
     }
 }
 
@@ -1175,9 +1200,9 @@ qnn_status tc_partial(const TcOperands &op, int splits, int32_t *part, int64_t l
 qnn_status launch_center_fp16(const uint8_t *in, int64_t rows, int64_t K, int64_t ldi, __half *out, int64_t ldo,
                               cudaStream_t st) {
     if (rows == 0) return QNN_OK;
-    const int64_t tot = rows * (ldo / 8);
-    center_fp16_kernel<<<(unsigned)std::min<int64_t>((tot + 255) / 256, 65535 * 4), 256, 0, st>>>(in, rows, (int)K, ldi,
-                                                                                                  out, (int)ldo);
+    const int64_t tot = rows * (ldo / 16);
+    center_fp16_kernel<<<(unsigned)std::min<int64_t>((tot + 255) / 256, (int64_t)sm_count() * 16), 256, 0, st>>>(
+        in, rows, (int)K, ldi, out, (int)ldo);
     QNN_CUDA_TRY(cudaGetLastError());
     return QNN_OK;
 }
