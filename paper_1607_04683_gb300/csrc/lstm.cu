@@ -821,6 +821,8 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
                         (choice == PathChoice::kTc || (choice == PathChoice::kAuto && B >= kTcMinBatch));
     if (choice == PathChoice::kTc && !use_tc) return QNN_ERR_INVALID_ARG;
     if (use_tc) QNN_TRY(tc_prepare(m));
+    // the tensor-core recurrence computes each step's input product in its gate kernel (no px)
+    const bool fused = use_tc && tc_input_fused(m);
     const FwdPlan plan = plan_recurrent(m, B);
 
     // workspace layout
@@ -835,7 +837,8 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const size_t o_codes = acct(rows * ld_in);
     const size_t o_prm = acct(rows * sizeof(qnn_qparams));
     const size_t o_rs = acct(rows * 4);
-    const size_t o_px = acct(rows * 4 * H * 4);
+    const size_t o_px = acct(fused ? 0 : rows * 4 * H * 4);
+    const size_t o_x16 = acct(fused ? tc_xwork_bytes(m, rows) : 0);
     const size_t o_seq0 = acct(rows * R * 4);
     const size_t o_seq1 = acct(rows * R * 4);
     const size_t o_h0 = acct(B * R * 4 * L);
@@ -895,11 +898,13 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     int64_t kin = I;
     for (int64_t l = 0; l < L; ++l) {
         const LayerDev &ly = m->layers[l];
-        // 1. quantize every frame of the layer input (one unit per row)
-        QNN_TRY(launch_quantize_rows(in, rows, kin, kin, codes, ld_in, prm, rs, st));
-        // 2. batched input product, recovered, plus bias
-        QNN_TRY(launch_qgemm(codes, ld_in, prm, QNN_PER_ROW, rs, rows, kin, ly.wx.codes, ly.wx.ld, ly.wx.params,
-                             H / m->S, ly.wx.sums, 4 * H, ly.bias, px, 4 * H, nullptr, st));
+        if (!fused) {
+            // 1. quantize every frame of the layer input (one unit per row)
+            QNN_TRY(launch_quantize_rows(in, rows, kin, kin, codes, ld_in, prm, rs, st));
+            // 2. batched input product, recovered, plus bias
+            QNN_TRY(launch_qgemm(codes, ld_in, prm, QNN_PER_ROW, rs, rows, kin, ly.wx.codes, ly.wx.ld, ly.wx.params,
+                                 H / m->S, ly.wx.sums, 4 * H, ly.bias, px, 4 * H, nullptr, st));
+        }
         // 3. recurrence
         float *outl = (ha_dev ? h_all + l * rows * R : seq[l & 1]);
         if (c_state)
@@ -907,7 +912,10 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
         else
             QNN_CUDA_TRY(cudaMemsetAsync(cbuf, 0, B * H * 4, st));
         if (use_tc) {
-            QNN_TRY(tc_layer_recurrence(m, l, px, h0 + l * B * R, cbuf, outl, mbuf, B, T, ws + o_tc, st));
+            TcFusedInput fx;
+            fx.in = in, fx.kin = kin, fx.x16 = reinterpret_cast<__half *>(ws + o_x16), fx.prm = prm, fx.rs = rs;
+            QNN_TRY(tc_layer_recurrence(m, l, fused ? nullptr : px, h0 + l * B * R, cbuf, outl, mbuf, B, T,
+                                        ws + o_tc, st, fused ? &fx : nullptr));
         } else {
             QNN_CUDA_TRY(cudaMemsetAsync(bar, 0, 256, st));
             RecArgs a{};

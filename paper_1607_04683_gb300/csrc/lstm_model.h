@@ -27,7 +27,19 @@ struct LayerDev {
 struct TcLayer {  // fp16 centered weight copies for the tensor-core recurrence (lstm_tc.cu)
     __half *wh16 = nullptr;  // [4 * round_up(H, 8)][kh]: gate rows interleaved in 8-cell groups
     __half *wp16 = nullptr;  // [P][kp] (P > 0)
-    int64_t kh = 0, kp = 0;
+    __half *wx16 = nullptr;  // [4 * round_up(H, 8)][kx], interleaved like wh16 (kx <= 1024)
+    int64_t kh = 0, kp = 0, kx = 0;
+};
+
+// The layer input of a recurrence whose input product is fused into the gate kernel: in [B*T][kin]
+// fp32 (row b T + t), and workspace for its centered fp16 codes x16 [B*T][round_up(kin, 64)], row
+// units prm [B*T] and code sums rs [B*T].
+struct TcFusedInput {
+    const float *in = nullptr;
+    int64_t kin = 0;
+    __half *x16 = nullptr;
+    qnn_qparams *prm = nullptr;
+    int32_t *rs = nullptr;
 };
 
 }  // namespace qnn
@@ -104,6 +116,13 @@ qnn_status tc_prepare(qnn_lstm_model *m);
 size_t tc_work_bytes(const qnn_lstm_model *m, int64_t B);
 // The T recurrent steps of layer l: px [B*T][4H] (row b*T + t) recovered input products plus bias,
 // h0 [B][R], cbuf [B][H] cell state in/out, out [B][T][R] layer outputs, mbuf [B][H] (P > 0).
+// With fx the step's input product is computed in the gate kernel from fx->in (px unused);
+// otherwise px holds it.
 qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
-                               float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st);
+                               float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st,
+                               const TcFusedInput *fx = nullptr);
+// Whether every layer's input product can be fused into its gate kernel (input width <= 1024; the
+// environment variable QNN_TC_FUSE_X=0 turns it off), and the workspace for the layer input's codes.
+bool tc_input_fused(const qnn_lstm_model *m);
+size_t tc_xwork_bytes(const qnn_lstm_model *m, int64_t rows);
 }  // namespace qnn

@@ -361,6 +361,8 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
     for (int64_t l = 0; l < m->L; ++l) {
         bytes += (size_t)round_up(4 * H8 * kh * 2, 256);
         if (P > 0) bytes += (size_t)round_up(P * kpj * 2, 256);
+        const int64_t kx = round_up(m->layers[l].kin, 64);
+        if (kx <= 1024) bytes += (size_t)round_up(4 * H8 * kx * 2, 256);  // Wx for the fused input product
     }
     void *buf = nullptr;
     QNN_CUDA_TRY(cudaMalloc(&buf, bytes));
@@ -378,6 +380,19 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
         if (cudaGetLastError() != cudaSuccess) {
             cudaFree(buf);
             return QNN_ERR_CUDA;
+        }
+        const int64_t kx = round_up(ly.kin, 64);
+        if (kx <= 1024) {
+            tl.kx = kx;
+            tl.wx16 = reinterpret_cast<__half *>(p);
+            p += round_up(4 * H8 * kx * 2, 256);
+            const int64_t totx = 4 * H8 * (kx / 8);
+            interleave_gates_kernel<<<(unsigned)((totx + 255) / 256), 256>>>(ly.wx.codes, ly.wx.ld, (int)H, (int)ly.kin,
+                                                                             (int)kx, tl.wx16);
+            if (cudaGetLastError() != cudaSuccess) {
+                cudaFree(buf);
+                return QNN_ERR_CUDA;
+            }
         }
         if (P > 0) {
             tl.kp = kpj;
@@ -406,8 +421,23 @@ size_t tc_work_bytes(const qnn_lstm_model *m, int64_t B) {
            (size_t)round_up(part, 256);
 }
 
+bool tc_input_fused(const qnn_lstm_model *m) {
+    const char *v = std::getenv("QNN_TC_FUSE_X");
+    if (v && std::strcmp(v, "0") == 0) return false;
+    for (int64_t l = 0; l < m->L; ++l)
+        if (round_up(m->layers[l].kin, 64) > 1024) return false;
+    return true;
+}
+
+size_t tc_xwork_bytes(const qnn_lstm_model *m, int64_t rows) {
+    int64_t kx = 0;
+    for (int64_t l = 0; l < m->L; ++l) kx = std::max(kx, round_up(m->layers[l].kin, 64));
+    return (size_t)round_up(rows * kx * 2, 256);
+}
+
 qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
-                               float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st) {
+                               float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st,
+                               const TcFusedInput *fx) {
     const LayerDev &ly = m->layers[l];
     const TcLayer &tl = m->tc_layers[l];
     const int64_t H = m->H, R = m->R, P = m->P, H8 = round_up(H, 8);
@@ -443,13 +473,27 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     // the steps' kernels chain by programmatic dependent launches (see tc_gemm.h); the first one of
     // the layer follows ordinary stream order
     gates.pdl = proj.pdl = pdl_enabled();
+    // fused input product: every frame of the layer input quantized once (rows b T + t, centered fp16)
+    TcLstmInput xin;
+    if (fx) {
+        if (!tl.wx16 || tl.kx != round_up(fx->kin, 64)) return QNN_ERR_INVALID_ARG;
+        QNN_TRY(launch_quantize_rows_f16(fx->in, fx->kin, B * T, (int)fx->kin, (int)tl.kx, fx->x16, fx->prm, fx->rs,
+                                         status, false, st));
+        xin.x_pitch = T * tl.kx, xin.kx = tl.kx, xin.K_x = (int)fx->kin, xin.stride = T;
+        xin.wx16 = tl.wx16, xin.pw4 = ly.wx.params, xin.cs = ly.wx.sums, xin.bias = ly.bias;
+    }
     QNN_TRY(launch_quantize_rows_f16(h0, R, B, R, kh, a16, prm, rs, status, false, st));
     for (int64_t t = 0; t < T; ++t) {
         if (t > 0 && !split_proj)
             QNN_TRY(launch_quantize_rows_f16(out + (t - 1) * R, T * R, B, R, kh, a16, prm, rs, status, gates.pdl, st));
-        TcLstmOut o{px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R, (int)H,
-                    (int)m->S, (int)(H / m->S)};
-        QNN_TRY(tc_lstm_gates(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, st));
+        TcLstmOut o{fx ? nullptr : px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R,
+                    (int)H, (int)m->S, (int)(H / m->S)};
+        if (fx) {
+            xin.x16 = fx->x16 + t * tl.kx, xin.pa = fx->prm + t, xin.rs = fx->rs + t;
+            QNN_TRY(tc_lstm_gates_x(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, xin, st));
+        } else {
+            QNN_TRY(tc_lstm_gates(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, st));
+        }
         if (P > 0) {
             QNN_TRY(launch_quantize_rows_f16(mbuf, H, B, H, kpj, m16, prm_m, rs_m, status, gates.pdl, st));
             if (split_proj) {

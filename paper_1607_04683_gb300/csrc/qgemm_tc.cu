@@ -44,7 +44,7 @@ constexpr unsigned long long TC_WAIT_NS = 2000000000ull;
 // those HBM loads delay the tile's TMA stream.)
 // kEpiPartial: split-K, each work item (tile, K range of at most 1024) stores its exact centered
 // integer sums P as int32 into its own slice of a partial-sum buffer; a consumer adds the slices.
-enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiPartial = 4 };
+enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiPartial = 4, kEpiLstmX = 5 };
 
 struct ColConst {  // per-output-column constants of kEpiRow, staged in shared memory per tile
     int cs, zw;
@@ -64,7 +64,9 @@ template <int BN, int EPI>
 struct Tile {
     static_assert(EPI == kEpiLinear || BN <= 128, "row and LSTM epilogues take tiles of at most 128 columns");
     // a 96-column LSTM tile has six 4-cell slices per lane quarter: 24 epilogue warps, one slice each
-    static constexpr bool LSTM96 = EPI == kEpiLstm && BN == 96;
+    // kEpiLstmX: the LSTM step with the input product fused in (a second operand pair and accumulator)
+    static constexpr bool IS_LSTM = EPI == kEpiLstm || EPI == kEpiLstmX;
+    static constexpr bool LSTM96 = IS_LSTM && BN == 96;
     static constexpr int EPI_WARPS = EPI == kEpiLinear ? 8 : (LSTM96 ? 24 : 16);
     // LSTM: cells per epilogue slice (a 32-column tile has 8 cells: 2-cell slices keep 4 warps busy)
     static constexpr int CPS = BN == 32 ? 2 : 4;
@@ -75,7 +77,7 @@ struct Tile {
     // reductions (K <= 1024) take several k-blocks a stage: four for narrow LSTM tiles (two stages in
     // flight), two for row tiles and split-K items; the long-K linear tiles and the 96-column LSTM
     // tiles keep more, smaller stages in flight (each choice measured on GB300)
-    static constexpr int KPS = EPI == kEpiLstm ? (BN <= 32 ? 4 : (BN == 64 ? 2 : 1))
+    static constexpr int KPS = IS_LSTM ? (BN <= 32 ? 4 : (BN == 64 ? 2 : 1))
                                                : ((EPI == kEpiPartial || EPI == kEpiRow) ? 2 : 1);
     static constexpr int SUB_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGE_BYTES = KPS * SUB_BYTES;
@@ -85,8 +87,8 @@ struct Tile {
     // LSTM: the tile's input products px (4 gates x 128 rows x BN/4 cells) and cell state c (128 x
     // BN/4), fp32, double-buffered in shared memory after the stages
     static constexpr int PX_BOX = TBM * (BN / 4) * 4;  // one gate's px box, bytes
-    static constexpr int LSTM_BUF = 5 * PX_BOX;        // 4 px boxes + the c box
-    static constexpr int EPI_BYTES = EPI == kEpiLstm      ? 2 * LSTM_BUF
+    static constexpr int LSTM_BUF = (EPI == kEpiLstmX ? 1 : 5) * PX_BOX;  // [4 px boxes +] the c box
+    static constexpr int EPI_BYTES = IS_LSTM              ? 2 * LSTM_BUF
                                      : EPI == kEpiPartial ? 0
                                                           : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
     static constexpr int SMEM_CAP = 227 * 1024 - 1024 - 256;  // dynamic shared memory left for stages + EPI_BYTES
@@ -94,7 +96,10 @@ struct Tile {
     static constexpr int WANT_STAGES = BASE_STAGES / KPS < 2 ? 2 : BASE_STAGES / KPS;
     static constexpr int STAGES = WANT_STAGES < FIT_STAGES ? WANT_STAGES : FIT_STAGES;
     static_assert(STAGES >= 2, "at least two pipeline stages must fit");
-    static constexpr int TMEM_COLS = 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
+    static constexpr int ACC_COLS = (EPI == kEpiLstmX ? 2 : 1) * BN;  // one tile buffer's accumulator columns
+    static constexpr int TMEM_COLS =
+        2 * ACC_COLS <= 32 ? 32
+                           : (2 * ACC_COLS <= 64 ? 64 : (2 * ACC_COLS <= 128 ? 128 : (2 * ACC_COLS <= 256 ? 256 : 512)));
     // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : (LSTM96 ? 72 : 96);
@@ -125,6 +130,17 @@ struct TcArgs {
     int64_t ldpart;
     int w_static;    // W was written before the previous kernel of the stream started (model weights):
                      // its first tiles may load before the programmatic-launch wait
+    // kEpiLstmX: the input product x_t Wx of the step (k-blocks 0 .. KB_x - 1 of the K loop, into a
+    // second accumulator; A from the x map, W from the Wx map). Row b of x_t has its unit at
+    // pa_x[b * x_stride] and its code sum at rsA_x[b * x_stride]; pw_x, csW_x (gate-major [4][H]) and
+    // bias_x ([4H]) as for the recurrent product; K_x the true input width.
+    const qnn_qparams *pa_x;
+    int64_t x_stride;
+    const int32_t *rsA_x;
+    const qnn_qparams *pw_x;
+    const int32_t *csW_x;
+    const float *bias_x;
+    int K_x, KB_x;
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
@@ -272,6 +288,7 @@ template <int BN, int EPI>
 __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN, EPI>::MAX_REGS))
     qgemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapW,
                     const __grid_constant__ CUtensorMap mapPX, const __grid_constant__ CUtensorMap mapC,
+                    const __grid_constant__ CUtensorMap mapAX, const __grid_constant__ CUtensorMap mapWX,
                     const TcArgs args) {
     using TL = Tile<BN, EPI>;
     constexpr int STAGES = TL::STAGES;
@@ -285,8 +302,10 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     // LSTM only: px/c buffer i loaded (pxfull0 + 8 i) and released by every epilogue warp (pxempty0 + 8 i)
     const uint32_t pxfull0 = su32(bars + 2 * STAGES + 4), pxempty0 = su32(bars + 2 * STAGES + 6);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int KB = args.KB;
-    const int kpc = KCHUNK / TBK;  // k-blocks per chunk (16)
+    constexpr bool LX = EPI == kEpiLstmX;
+    const int KB = args.KB + (LX ? args.KB_x : 0);  // k-blocks of the K loop (kEpiLstmX: x's, then h's)
+    const int kpc = LX ? 64 : KCHUNK / TBK;        // k-blocks per chunk (16; kEpiLstmX: the whole loop, each
+                                                   // accumulator summing at most 1024)
     const int nchunks = (KB + kpc - 1) / kpc;
     const int tiles_n = (int)((args.N + BN - 1) / BN);
     const int64_t tiles_m = (args.M + TBM - 1) / TBM;
@@ -294,6 +313,19 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     // work items: (tile, K range); one K range per tile except for split-K
     const int splits = args.splits;
     const int64_t items = tiles * splits;
+    // the A and W tiles of k-block kb (kEpiLstmX: x_t and Wx for kb < KB_x, then h_{t-1} and Wh)
+    auto load_a = [&](uint32_t dst, uint32_t bar, int kb, int m0) {
+        if (LX && kb < args.KB_x)
+            tma_load_2d(dst, &mapAX, bar, kb * TBK, m0);
+        else
+            tma_load_2d(dst, &mapA, bar, (kb - (LX ? args.KB_x : 0)) * TBK, m0);
+    };
+    auto load_w = [&](uint32_t dst, uint32_t bar, int kb, int n0) {
+        if (LX && kb < args.KB_x)
+            tma_load_2d(dst, &mapWX, bar, kb * TBK, n0);
+        else
+            tma_load_2d(dst, &mapW, bar, (kb - (LX ? args.KB_x : 0)) * TBK, n0);
+    };
     __shared__ int s_abort;
 
     if (threadIdx.x == 0) {
@@ -336,7 +368,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 for (int j = 0; j < w_early; ++j) {
                     const uint32_t sb = su32(smem + j * TL::STAGE_BYTES) + A_BYTES;
                     mb_expect(full0 + 8 * j, TL::STAGE_BYTES);
-                    tma_load_2d(sb, &mapW, full0 + 8 * j, (kb0 + j) * TBK, n0);
+                    load_w(sb, full0 + 8 * j, kb0 + j, (int)n0);
                 }
             } else {
                 w_early = min(STAGES, (kb1 - kb0 + TL::KPS - 1) / TL::KPS);
@@ -345,7 +377,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     const uint32_t sb = su32(smem + j * TL::STAGE_BYTES) + TL::KPS * A_BYTES;
                     mb_expect(full0 + 8 * j, (uint32_t)(nv * TL::SUB_BYTES));
                     for (int v = 0; v < nv; ++v)
-                        tma_load_2d(sb + v * TL::B_BYTES, &mapW, full0 + 8 * j, (kbj + v) * TBK, n0);
+                        load_w(sb + v * TL::B_BYTES, full0 + 8 * j, kbj + v, (int)n0);
                 }
             }
         }
@@ -375,12 +407,12 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         }
                         const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
                         if (g < w_early) {  // W already on its way (expect set with it)
-                            tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
+                            load_a(sa, full0 + 8 * s, kb, (int)m0);
                             continue;
                         }
                         mb_expect(full0 + 8 * s, TL::STAGE_BYTES);
-                        tma_load_2d(sa, &mapA, full0 + 8 * s, kb * TBK, m0);
-                        tma_load_2d(sb, &mapW, full0 + 8 * s, kb * TBK, n0);
+                        load_a(sa, full0 + 8 * s, kb, (int)m0);
+                        load_w(sb, full0 + 8 * s, kb, (int)n0);
                     }
                 }
             }
@@ -410,8 +442,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     #pragma unroll
                         for (int v = 0; v < TL::KPS; ++v) {
                             if (v >= nv) break;
-                            tma_load_2d(st_addr + v * A_BYTES, &mapA, bar_full, (kb + v) * TBK, m0);
-                            if (!w_sent) tma_load_2d(sb + v * TL::B_BYTES, &mapW, bar_full, (kb + v) * TBK, n0);
+                            load_a(st_addr + v * A_BYTES, bar_full, kb + v, m0);
+                            if (!w_sent) load_w(sb + v * TL::B_BYTES, bar_full, kb + v, n0);
                         }
                         if (issued < STAGES) ++issued;
                         if (++slot == STAGES) {
@@ -447,12 +479,15 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         }
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                         const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
-                        const uint32_t tmem_d = tmem_base + (uint32_t)(buf * BN);
+                        // kEpiLstmX: x's k-blocks into the buffer's first accumulator, h's into the second
+                        const bool hpart = LX && kb >= args.KB_x;
+                        const uint32_t tmem_d = tmem_base + (uint32_t)(buf * TL::ACC_COLS + (hpart ? BN : 0));
+                        const bool fresh = kc == 0 || (LX && kb == args.KB_x);
     #pragma unroll
                         for (int k = 0; k < TBK / 16; ++k) {
                             // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
                             mma_f16<TL::IDESC>(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k),
-                                               (kc == 0 && k == 0) ? 0u : 1u);
+                                               (fresh && k == 0) ? 0u : 1u);
                         }
                         mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
                         if (kc == kpc - 1 || kb == kb1 - 1) {
@@ -490,16 +525,19 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         }
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                         const uint64_t da = smem_desc(st_addr), db = smem_desc(st_addr + TL::KPS * A_BYTES);
-                        const uint32_t tmem_d = tmem_base + (uint32_t)(buf * BN);
     #pragma unroll
                         for (int v = 0; v < TL::KPS; ++v) {
                             if (v >= nv) break;
+                            // kEpiLstmX: x's k-blocks into the buffer's first accumulator, h's into the second
+                            const bool hpart = LX && kb + v >= args.KB_x;
+                            const uint32_t tmem_d = tmem_base + (uint32_t)(buf * TL::ACC_COLS + (hpart ? BN : 0));
+                            const bool fresh = (kc == 0 && v == 0) || (LX && kb + v == args.KB_x);
     #pragma unroll
                             for (int k = 0; k < TBK / 16; ++k) {
                                 // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
                                 mma_f16<TL::IDESC>(tmem_d, da + (uint64_t)((v * A_BYTES + 32 * k) >> 4),
                                                    db + (uint64_t)((v * TL::B_BYTES + 32 * k) >> 4),
-                                                   (kc == 0 && v == 0 && k == 0) ? 0u : 1u);
+                                                   (fresh && k == 0) ? 0u : 1u);
                             }
                         }
                         mma_commit(bar_empty);  // frees the stage when these MMAs have read it
@@ -800,6 +838,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         // the block's i-th tile; one thread (warp 2, lane 0) refills a buffer once every epilogue
         // warp has released it, so the loads overlap the arithmetic of the tile in between
         constexpr int CW = BN / 4;  // cells per tile
+        constexpr int C_OFF = LX ? 0 : 4 * TL::PX_BOX;  // the c box within a buffer (after the px boxes)
         float *const pxs0 = reinterpret_cast<float *>(smem + STAGES * TL::STAGE_BYTES);
         const bool issuer = warp == 2 && lane == 0;
         auto issue_px = [&](int64_t t_issue, int pbuf) {
@@ -808,10 +847,12 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             const uint32_t bar = pxfull0 + 8 * pbuf;
             const uint32_t dst = su32(pxs0) + (uint32_t)(pbuf * TL::LSTM_BUF);
             mb_expect(bar, (uint32_t)TL::LSTM_BUF);
+            if constexpr (!LX) {  // kEpiLstmX computes the input products itself: c only
 #pragma unroll
-            for (int g = 0; g < 4; ++g)
-                tma_load_2d(dst + g * TL::PX_BOX, &mapPX, bar, g * H + (int)(n1 / 4), (int)m1);
-            tma_load_2d(dst + 4 * TL::PX_BOX, &mapC, bar, (int)(n1 / 4), (int)m1);
+                for (int g = 0; g < 4; ++g)
+                    tma_load_2d(dst + g * TL::PX_BOX, &mapPX, bar, g * H + (int)(n1 / 4), (int)m1);
+            }
+            tma_load_2d(dst + C_OFF, &mapC, bar, (int)(n1 / 4), (int)m1);
         };
         if (issuer) {
             if (blockIdx.x < tiles) issue_px(blockIdx.x, 0);
@@ -836,6 +877,14 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 rs = args.rsA[b];
             }
             const int za128 = 128 + za;
+            int zx = 0, rsx = 0;  // kEpiLstmX: the unit and code sum of row b of x_t
+            float Qx = 1.0f;
+            if (LX && bv) {
+                const qnn_qparams qa = args.pa_x[b * args.x_stride];
+                zx = qa.z;
+                Qx = qa.Q;
+                rsx = args.rsA_x[b * args.x_stride];
+            }
             const int buf = (int)(gc & 1);
             ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status) &&
                                              mb_wait(pxfull0 + 8 * pbuf, (unsigned)(gc / 2) & 1, args.status));
@@ -845,6 +894,69 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             for (int s = eh; s < SLICES; s += TL::EPI_WARPS / 4) {
                 const int gi = s / SPG, part = s % SPG;
                 const int j0 = (int)(n0 / 4) + gi * 8 + part * CPS;  // H is a multiple of 4: all CPS valid or none
+                if constexpr (LX) {
+                    // pre = (R(x_t Wx) + b) + R(h_{t-1} Wh): both exact sums recovered as in eq. (1)/(3)
+                    // (the input side exactly as the batched product computes px), then the cell
+                    const bool valid = bv && j0 < H;
+                    const int unit = j0 / E.cpu;
+                    const long long ax = max(abs(zx), abs(zx + 255)), ah = max(abs(za), abs(za + 255));
+                    const uint32_t tx = tmem_base + ((uint32_t)(32 * q) << 16) +
+                                        (uint32_t)(buf * TL::ACC_COLS + gi * 32 + part * CPS);
+                    float pre[4][CPS];
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        uint32_t rx[CPS], rh[CPS];
+                        tmem_ld_nowait(tx + 8 * g, rx);
+                        tmem_ld_nowait(tx + BN + 8 * g, rh);
+                        tmem_wait_ld();
+                        if (valid) {
+                            // the gate's row terms (per gate, to keep registers free)
+                            const qnn_qparams qw = args.pw_x[g * E.ups + unit], qh = args.pw[g * E.ups + unit];
+                            const long long rtx = (long long)(128 + qw.z) * rsx +
+                                                  (long long)args.K_x * ((long long)zx * qw.z - 16384);
+                            const long long rth =
+                                (long long)(128 + qh.z) * rs + (long long)K * ((long long)za * qh.z - 16384);
+                            const float denx = __fmul_rn(Qx, qw.Q), denh = __fmul_rn(Qa, qh.Q);
+                            const bool fits =
+                                (long long)args.K_x * ax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31) &&
+                                (long long)K * ah * (long long)max(abs(qh.z), abs(qh.z + 255)) < (1LL << 31);
+                            float bias[CPS];
+                            int csx[CPS], csh[CPS];
+                            ld_vec(args.bias_x + g * H + j0, bias);
+                            ld_vec(args.csW_x + g * H + j0, csx);
+                            ld_vec(args.csW + g * H + j0, csh);
+#pragma unroll
+                            for (int jj = 0; jj < CPS; ++jj) {
+                                const int Px = f32_integer_to_s32(__uint_as_float(rx[jj]));
+                                const int Ph = f32_integer_to_s32(__uint_as_float(rh[jj]));
+                                float vx, vh;
+                                if (fits) {
+                                    vx = __int2float_rn((int)((uint32_t)Px + (uint32_t)rtx +
+                                                              (uint32_t)(128 + zx) * (uint32_t)csx[jj]));
+                                    vh = __int2float_rn((int)((uint32_t)Ph + (uint32_t)rth +
+                                                              (uint32_t)za128 * (uint32_t)csh[jj]));
+                                } else {
+                                    vx = s64_to_f32_rn((long long)Px + rtx + (long long)(128 + zx) * csx[jj]);
+                                    vh = s64_to_f32_rn((long long)Ph + rth + (long long)za128 * csh[jj]);
+                                }
+                                const float yx = __fadd_rn(__fdiv_rn(vx, denx), bias[jj]);
+                                pre[g][jj] = __fadd_rn(yx, __fdiv_rn(vh, denh));
+                            }
+                        }
+                    }
+                    if (valid) {
+                        const int jt = j0 - (int)(n0 / 4);
+                        float *cr = E.c + b * (int64_t)H + j0;
+                        float cv[CPS], mv[CPS];
+                        ld_vec(pxb + C_OFF / 4 + rl * CW + jt, cv);
+#pragma unroll
+                        for (int jj = 0; jj < CPS; ++jj)
+                            lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
+                        st_vec(cr, cv);
+                        st_vec(E.h + b * E.h_ld + j0, mv);
+                    }
+                    continue;
+                }
                 uint32_t r[4][CPS];
                 const uint32_t ta = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN + gi * 32 + part * CPS);
 #pragma unroll
@@ -892,7 +1004,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         }
                     }
                     float cv[CPS], mv[CPS];
-                    ld_vec(pxb + 4 * (TL::PX_BOX / 4) + rl * CW + jt, cv);
+                    ld_vec(pxb + C_OFF / 4 + rl * CW + jt, cv);
 #pragma unroll
                     for (int jj = 0; jj < CPS; ++jj) lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
                     st_vec(cr, cv);
@@ -1008,11 +1120,12 @@ qnn_status make_map_f32(CUtensorMap *map, const float *base, int64_t rows, int64
 }
 
 // 2-D fp16 tensor [rows][ld] (ld a multiple of 64), boxes of 64 x box_rows, 128-byte swizzle.
-qnn_status make_map(CUtensorMap *map, const __half *base, int64_t rows, int64_t ld, int box_rows) {
+qnn_status make_map(CUtensorMap *map, const __half *base, int64_t rows, int64_t ld, int box_rows,
+                    int64_t pitch = 0) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = nullptr;
     QNN_TRY(get_encode(&enc));
     cuuint64_t dims[2] = {(cuuint64_t)ld, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+    cuuint64_t strides[1] = {(cuuint64_t)((pitch > 0 ? pitch : ld) * 2)};  // rows may lie further apart
     cuuint32_t box[2] = {(cuuint32_t)TBK, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half *>(base), dims, strides, box, estr,
@@ -1032,7 +1145,8 @@ namespace {
 
 template <int BN, int EPI>
 qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cudaStream_t st,
-                     const CUtensorMap *map_px = nullptr, const CUtensorMap *map_c = nullptr) {
+                     const CUtensorMap *map_px = nullptr, const CUtensorMap *map_c = nullptr,
+                     const CUtensorMap *map_ax = nullptr, const CUtensorMap *map_wx = nullptr) {
     using TL = Tile<BN, EPI>;
     static int configured = -1;
     int dev = 0;
@@ -1053,7 +1167,7 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
                          "%d blocks per SM\n", BN, EPI, TL::THREADS, fa.numRegs, TL::SMEM, n);
         }
     }
-    const int64_t items = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN) * a.splits;
+    const int64_t items = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN) * a.splits;  // (tile, K range) pairs
     // persistent: one block per SM (a block holding tensor memory has its SM to itself)
     const unsigned grid = (unsigned)std::min<int64_t>(items, (int64_t)sm_count());
     ProfScope prof(name, st);
@@ -1067,9 +1181,9 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = op.pdl ? 1 : 0;
-    // the px and c maps are read by the LSTM epilogue only (the others get A's map, unused)
+    // the px, c, x and Wx maps are read by the LSTM kernels only (the others get A's map, unused)
     QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, qgemm_tc_kernel<BN, EPI>, op.a, op.w, map_px ? *map_px : op.a,
-                                    map_c ? *map_c : op.a, a));
+                                    map_c ? *map_c : op.a, map_ax ? *map_ax : op.a, map_wx ? *map_wx : op.w, a));
     return QNN_OK;
 }
 
@@ -1172,6 +1286,36 @@ qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int3
     TcArgs a{pa, 1, rsA, pw4, 0, cs, nullptr, nullptr, 0, nullptr, op.M, op.N, (int)K, (int)(op.kp / TBK), status, out,
              1, (int)(op.kp / TBK), nullptr, 0, 1};
     return dispatch_lstm(op, a, st);
+}
+
+qnn_status tc_lstm_gates_x(const TcOperands &op, const qnn_qparams *pa, const int32_t *rsA, int64_t K,
+                           const qnn_qparams *pw4, const int32_t *cs, const TcLstmOut &out, const TcLstmInput &in,
+                           cudaStream_t st) {
+    if (K <= 0 || op.kp > KCHUNK || K > op.kp || out.H <= 0 || out.H % 4 != 0) return QNN_ERR_INVALID_ARG;
+    if (out.ups < 1 || out.cpu < 4 || out.cpu % 4 != 0 || out.cpu * out.ups != out.H) return QNN_ERR_INVALID_ARG;
+    if (op.N != 4 * ((out.H + 7) / 8 * 8)) return QNN_ERR_INVALID_ARG;
+    if (in.K_x <= 0 || in.kx % TBK != 0 || in.kx > KCHUNK || in.K_x > in.kx || in.x_pitch < in.kx || in.x_pitch % 8)
+        return QNN_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(in.x16) & 15) || (reinterpret_cast<uintptr_t>(in.wx16) & 15))
+        return QNN_ERR_INVALID_ARG;
+    int *status = nullptr;
+    QNN_TRY(status_word(&status));
+    const int kbh = (int)(op.kp / TBK), kbx = (int)(in.kx / TBK);
+    TcArgs a{pa, 1, rsA, pw4, 0, cs, nullptr, nullptr, 0, nullptr, op.M, op.N, (int)K, kbh, status, out,
+             1, kbh + kbx, nullptr, 0, 1};
+    a.pa_x = in.pa, a.x_stride = in.stride, a.rsA_x = in.rs, a.pw_x = in.pw4, a.csW_x = in.cs, a.bias_x = in.bias;
+    a.K_x = in.K_x, a.KB_x = kbx;
+    CUtensorMap map_c, map_ax, map_wx;
+    QNN_TRY(make_map_f32(&map_c, out.c, op.M, out.H, out.H, op.bn / 4, TBM));
+    QNN_TRY(make_map(&map_ax, in.x16, op.M, in.kx, TBM, in.x_pitch));
+    QNN_TRY(make_map(&map_wx, in.wx16, op.N, in.kx, op.bn));
+    switch (op.bn) {
+        case 32: return launch_tc<32, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
+        case 64: return launch_tc<64, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
+        case 96: return launch_tc<96, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
+        case 128: return launch_tc<128, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
+        default: return QNN_ERR_INVALID_ARG;
+    }
 }
 
 int tc_partial_splits(const TcOperands &op, int max_splits) {

@@ -52,10 +52,34 @@ struct TcLstmOut {
     int cpu = 0;  // cells per unit (H / ups, a multiple of 4)
 };
 
+// The input side of a step when it is fused into the gate kernel (tc_lstm_gates_x): centered fp16
+// codes of x_t (row b at x16 + b * x_pitch, kx columns: K_x true values then zeros, kx a multiple of
+// 64 and at most 1024), row b's unit and code sum at pa[b * stride] and rs[b * stride], the Wx gate
+// matrices interleaved like Wh ([4 round_up(H, 8)][kx]), their units (4 ups, gate-major), row code
+// sums in gate-major order [4][H] and the bias [4H].
+struct TcLstmInput {
+    const __half *x16 = nullptr;
+    int64_t x_pitch = 0, kx = 0;
+    int K_x = 0;
+    const qnn_qparams *pa = nullptr;
+    const int32_t *rs = nullptr;
+    int64_t stride = 1;
+    const __half *wx16 = nullptr;
+    const qnn_qparams *pw4 = nullptr;
+    const int32_t *cs = nullptr;
+    const float *bias = nullptr;
+};
+
 // One recurrent step's gate product and cell update: A = centered codes of h_{t-1} (one unit per
 // row: pa, rsA), W = the four Wh gate matrices interleaved in 8-cell groups [i f g o] x 8 rows
 // (op.N = 4 * round_up(H, 8)), pw4 the gate units (4 ups, gate-major), cs their row code sums in
 // gate-major order [4][H]. K (true) <= 1024.
+// As tc_lstm_gates, with the step's input product computed in the same kernel (a second operand
+// pair and accumulator) instead of read from out.px: pre = (R(x_t Wx) + b) + R(h_{t-1} Wh), the
+// same operations in the same order as the batched product followed by tc_lstm_gates.
+qnn_status tc_lstm_gates_x(const TcOperands &op, const qnn_qparams *pa, const int32_t *rsA, int64_t K,
+                           const qnn_qparams *pw4, const int32_t *cs, const TcLstmOut &out, const TcLstmInput &in,
+                           cudaStream_t st);
 qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int32_t *rsA, int64_t K,
                          const qnn_qparams *pw4, const int32_t *cs, const TcLstmOut &out, cudaStream_t st);
 

@@ -398,6 +398,23 @@ def test_tc_recurrence_bit_exact(qnn, cfg, bn, monkeypatch):
     _compare(got, ref, wl)
 
 
+@pytest.mark.parametrize("fuse", ["1", "0"])
+@pytest.mark.parametrize("cfg", [dict(L=2, I=40, H=100, C=37, B=130, T=4), dict(L=2, I=80, H=1100, P=64, C=20, B=40, T=3,
+                                                                                 w=0.05),
+                                 dict(L=2, I=600, H=64, P=48, B=70, T=3)])
+def test_tc_input_product_fused_and_batched(qnn, cfg, fuse, monkeypatch):
+    # the step's input product computed inside the gate kernel (default) and by the batched product
+    # (QNN_TC_FUSE_X=0) give the oracle's results bit for bit; I = 600 puts the input on two
+    # chunk-sized parts of the fused K loop (10 k-blocks of x, then those of h)
+    wl = _small(**cfg)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x, want_h_all=True)
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    monkeypatch.setenv("QNN_TC_FUSE_X", fuse)
+    got = _gpu_forward(qnn, wl, params, x)
+    _compare(got, ref, wl)
+
+
 @pytest.mark.parametrize("bn", ["32", "96"])
 def test_tc_recurrence_large_weight_offsets(qnn, bn, monkeypatch):
     # every weight shifted by +20: weight ranges far from zero give offsets z of about 32000, so
