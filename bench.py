@@ -123,12 +123,29 @@ def source_sha(sources) -> str:
     return h.hexdigest()[:16]
 
 
+def gates_fused(wl) -> bool:
+    """Whether the gate kernel computes the step's input product itself (the library's default for
+    input widths up to 1024; QNN_TC_FUSE_X=0 turns it off)."""
+    return os.environ.get("QNN_TC_FUSE_X") != "0" and max(wl.input_dim, wl.R) <= 1024
+
+
+def gates_input_width(wl) -> float:
+    """Input width of a layer, averaged over the layers (the first takes the frames, the rest R)."""
+    return (wl.input_dim + (wl.num_layers - 1) * wl.R) / wl.num_layers
+
+
 def gates_bytes_per_launch(wl) -> float:
-    """Algorithmic DRAM bytes of one tensor-core recurrent step: the step's input products px
-    (B x 4H fp32), the cell state read and written (B x H fp32 each way), the cell outputs written
-    (B x H fp32), the recurrent input codes (B x R bytes) and the gate weight codes (4H x R bytes)."""
+    """Algorithmic DRAM bytes of one tensor-core recurrent step: the cell state read and written
+    (B x H fp32 each way), the cell outputs written (B x H fp32), the recurrent input codes (B x R
+    bytes) and the gate weight codes (4H x R bytes); plus, with the input product fused in, the
+    step's input codes (B x I bytes) and the input weight codes (4H x I bytes), else the batched
+    input products px (B x 4H fp32). I is averaged over the layers."""
     B, H, R = wl.batch, wl.hidden, wl.R
-    return float(B * 4 * H * 4 + 2 * B * H * 4 + B * H * 4 + B * R + 4 * H * R)
+    common = 2 * B * H * 4 + B * H * 4 + B * R + 4 * H * R
+    if gates_fused(wl):
+        il = gates_input_width(wl)
+        return float(common + B * il + 4 * H * il)
+    return float(common + B * 4 * H * 4)
 
 
 def traffic_record(kernel: str, workload: str, sources):
@@ -394,17 +411,26 @@ def run_ours(args, wl, rank, world, local):
                                "frac": floor_us / us_frame, "cluster_blocks": cs,
                                "floor_kind": "measured (qnn_measure_exchange_floor)"}
     elif kname == "lstm_gates_tc":
-        # one recurrent step of one layer: the tcgen05 gate product with the LSTM cell in its
-        # epilogue; reported against HBM with the step's algorithmic bytes, plus its tensor rate
+        # one recurrent step of one layer: the tcgen05 gate product (with the input product fused
+        # in, the library's default) and the LSTM cell in its epilogue. Fused, the step moves few
+        # bytes (no px) and its work is the 2 B 4H (R + I) operations of the two products: reported
+        # against the fp16 tensor peak, with its HBM rate beside; unfused against HBM.
         alg = gates_bytes_per_launch(wl)
-        ach = alg / avg_s / 1e9
-        flops = 2.0 * wl.batch * 4 * wl.hidden * wl.R
-        roofline = {"bound": "hbm", "kernel": kname, "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                    "frac": ach / peaks["hbm_gbs"], "peak_kind": peak_kind,
-                    "traffic": traffic_record(kname, wl.name, ["qgemm_tc.cu", "qnn_device.cuh"]),
-                    "alg_bytes_per_launch": alg, "tensor_tflops": flops / avg_s / 1e12,
-                    "tensor_frac": flops / avg_s / 1e12 / peaks["bf16_tflops"],
-                    "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
+        gbs = alg / avg_s / 1e9
+        flops = 2.0 * wl.batch * 4 * wl.hidden * (wl.R + (gates_input_width(wl) if gates_fused(wl) else 0))
+        tfs = flops / avg_s / 1e12
+        traffic = traffic_record(kname, wl.name, ["qgemm_tc.cu", "qnn_device.cuh"])
+        if gates_fused(wl):
+            roofline = {"bound": "tensor", "kernel": kname, "achieved": tfs, "peak": peaks["bf16_tflops"],
+                        "unit": "TFLOP/s", "frac": tfs / peaks["bf16_tflops"], "peak_kind": peak_kind,
+                        "traffic": traffic, "alg_flops_per_launch": flops, "alg_bytes_per_launch": alg,
+                        "hbm_gbs": gbs, "hbm_frac": gbs / peaks["hbm_gbs"], "input_product": "fused",
+                        "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
+        else:
+            roofline = {"bound": "hbm", "kernel": kname, "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "frac": gbs / peaks["hbm_gbs"], "peak_kind": peak_kind, "traffic": traffic,
+                        "alg_bytes_per_launch": alg, "tensor_tflops": tfs, "tensor_frac": tfs / peaks["bf16_tflops"],
+                        "input_product": "batched", "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
     line = {
         "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
