@@ -460,8 +460,11 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     int *status = nullptr;
     QNN_TRY(status_word(&status));
     TcOperands gates, proj;
-    static const int gate_bn[] = {128, 96, 64, 32};
-    QNN_TRY(tc_operands(&gates, a16, B, tl.wh16, 4 * H8, kh, tc_choose_bn(B, 4 * H8, gate_bn, 4)));
+    // tile widths, widest first; the fused kernel's 96-column tile (24 warps at 72 registers) spills
+    // with the second recovery and measured slower than 64 columns, so it is left out there
+    static const int gate_bn[] = {128, 96, 64, 32}, gate_bn_fused[] = {128, 64, 32};
+    QNN_TRY(tc_operands(&gates, a16, B, tl.wh16, 4 * H8, kh,
+                        fx ? tc_choose_bn(B, 4 * H8, gate_bn_fused, 3) : tc_choose_bn(B, 4 * H8, gate_bn, 4)));
     // the projection: split-K partial sums, finished (offsets, recovery, next step's quantization)
     // by one row kernel when P <= 2048; else one tcgen05 product with its own epilogue per step
     const bool split_proj = P > 0 && P <= 2048;
