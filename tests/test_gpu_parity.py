@@ -389,6 +389,8 @@ def test_tc_recurrence_bit_exact(qnn, cfg, bn, monkeypatch):
     ref = _oracle(wl, params, x, want_h_all=True)
     monkeypatch.setenv("QNN_LSTM_PATH", "tc")
     monkeypatch.setenv("QNN_TC_BN", bn)
+    # the fused gate kernel takes 128/64/32-column tiles; the 96-column one serves the px path
+    monkeypatch.setenv("QNN_TC_FUSE_X", "0" if bn == "96" else "1")
     qnn.profile_read()
     qnn.profile_enable(True)
     got = _gpu_forward(qnn, wl, params, x)
