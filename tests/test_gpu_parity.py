@@ -417,8 +417,8 @@ def test_tc_input_product_fused_and_batched(qnn, cfg, fuse, monkeypatch):
     _compare(got, ref, wl)
 
 
-@pytest.mark.parametrize("bn", ["32", "96"])
-def test_tc_recurrence_large_weight_offsets(qnn, bn, monkeypatch):
+@pytest.mark.parametrize("bn,fuse", [("32", "1"), ("64", "1"), ("96", "0")])
+def test_tc_recurrence_large_weight_offsets(qnn, bn, fuse, monkeypatch):
     # every weight shifted by +20: weight ranges far from zero give offsets z of about 32000, so
     # K |a' + za| |w' + zw| exceeds 2^31 and the gate epilogue sums S in 64 bits
     wl = _small(L=1, I=40, H=128, B=70, T=3, w=0.08)
@@ -427,6 +427,7 @@ def test_tc_recurrence_large_weight_offsets(qnn, bn, monkeypatch):
     ref = _oracle(wl, params, x, want_h_all=True)
     monkeypatch.setenv("QNN_LSTM_PATH", "tc")
     monkeypatch.setenv("QNN_TC_BN", bn)
+    monkeypatch.setenv("QNN_TC_FUSE_X", fuse)
     got = _gpu_forward(qnn, wl, params, x)
     _compare(got, ref, wl)
 
