@@ -439,7 +439,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         const uint32_t sb = st_addr + TL::KPS * A_BYTES;
                         const bool w_sent = issued < w_early;   // W already on its way (expect set with it)
                         if (!w_sent) mb_expect(bar_full, (uint32_t)(nv * TL::SUB_BYTES));
-    #pragma unroll
+#pragma unroll
                         for (int v = 0; v < TL::KPS; ++v) {
                             if (v >= nv) break;
                             load_a(st_addr + v * A_BYTES, bar_full, kb + v, m0);
@@ -483,7 +483,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         const bool hpart = LX && kb >= args.KB_x;
                         const uint32_t tmem_d = tmem_base + (uint32_t)(buf * TL::ACC_COLS + (hpart ? BN : 0));
                         const bool fresh = kc == 0 || (LX && kb == args.KB_x);
-    #pragma unroll
+#pragma unroll
                         for (int k = 0; k < TBK / 16; ++k) {
                             // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
                             mma_f16<TL::IDESC>(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k),
@@ -525,14 +525,14 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         }
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                         const uint64_t da = smem_desc(st_addr), db = smem_desc(st_addr + TL::KPS * A_BYTES);
-    #pragma unroll
+#pragma unroll
                         for (int v = 0; v < TL::KPS; ++v) {
                             if (v >= nv) break;
                             // kEpiLstmX: x's k-blocks into the buffer's first accumulator, h's into the second
                             const bool hpart = LX && kb + v >= args.KB_x;
                             const uint32_t tmem_d = tmem_base + (uint32_t)(buf * TL::ACC_COLS + (hpart ? BN : 0));
                             const bool fresh = (kc == 0 && v == 0) || (LX && kb + v == args.KB_x);
-    #pragma unroll
+#pragma unroll
                             for (int k = 0; k < TBK / 16; ++k) {
                                 // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
                                 mma_f16<TL::IDESC>(tmem_d, da + (uint64_t)((v * A_BYTES + 32 * k) >> 4),
