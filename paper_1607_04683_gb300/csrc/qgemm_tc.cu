@@ -356,9 +356,17 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     // Static weights: the producer starts the W tiles of its first stages before the wait below
     // (the A tiles, outputs of the previous kernel, follow after it); their barriers expect both.
     int w_early = 0;
+    // kEpiLstmX: the input side (x_t codes, Wx) was written before the step loop began, not by the
+    // previous kernel, so leading stages that hold only x's k-blocks are issued whole before the
+    // wait (their MMAs then overlap the previous kernel too)
+    int full_early = 0;
     if (warp == 0 && lane == 0) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapW)) : "memory");
+        if (LX) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapAX)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapWX)) : "memory");
+        }
         if (args.w_static && blockIdx.x < items) {
             int64_t m0, n0;
             tile_origin(blockIdx.x / splits, tiles_m, tiles_n, BN, m0, n0);
@@ -369,6 +377,10 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     const uint32_t sb = su32(smem + j * TL::STAGE_BYTES) + A_BYTES;
                     mb_expect(full0 + 8 * j, TL::STAGE_BYTES);
                     load_w(sb, full0 + 8 * j, kb0 + j, (int)n0);
+                    if (LX && full_early == j && kb0 + j < args.KB_x) {
+                        load_a(sb - A_BYTES, full0 + 8 * j, kb0 + j, (int)m0);
+                        ++full_early;
+                    }
                 }
             } else {
                 w_early = min(STAGES, (kb1 - kb0 + TL::KPS - 1) / TL::KPS);
@@ -378,13 +390,20 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     mb_expect(full0 + 8 * j, (uint32_t)(nv * TL::SUB_BYTES));
                     for (int v = 0; v < nv; ++v)
                         load_w(sb + v * TL::B_BYTES, full0 + 8 * j, kbj + v, (int)n0);
+                    if (LX && full_early == j && kbj + nv <= args.KB_x) {
+                        for (int v = 0; v < nv; ++v)
+                            load_a(sb - TL::KPS * A_BYTES + v * A_BYTES, full0 + 8 * j, kbj + v, (int)m0);
+                        ++full_early;
+                    }
                 }
             }
         }
     }
     // With a programmatic dependent launch the setup above overlaps the previous kernel of the
     // stream; its outputs (this kernel's operands) are complete and visible after this wait.
-    grid_dependency_wait();
+    // (kEpiLstmX: the MMA warp reads only shared and tensor memory, so it starts on the early
+    // input-side stages at once.)
+    if (!(LX && warp == 1)) grid_dependency_wait();
     grid_dependents_launch();
 
     // Persistent: block b takes tiles b, b + grid, ... in grouped order (tile_origin). The k-block
@@ -406,6 +425,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                             break;
                         }
                         const uint32_t sa = su32(smem + s * TL::STAGE_BYTES), sb = sa + A_BYTES;
+                        if (g < full_early) continue;  // issued whole before the wait
                         if (g < w_early) {  // W already on its way (expect set with it)
                             load_a(sa, full0 + 8 * s, kb, (int)m0);
                             continue;
@@ -438,12 +458,14 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         const int nv = min(TL::KPS, kb1 - kb);  // k-blocks in this stage (the last may be short)
                         const uint32_t sb = st_addr + TL::KPS * A_BYTES;
                         const bool w_sent = issued < w_early;   // W already on its way (expect set with it)
-                        if (!w_sent) mb_expect(bar_full, (uint32_t)(nv * TL::SUB_BYTES));
+                        if (issued >= full_early) {             // (else issued whole before the wait)
+                            if (!w_sent) mb_expect(bar_full, (uint32_t)(nv * TL::SUB_BYTES));
 #pragma unroll
-                        for (int v = 0; v < TL::KPS; ++v) {
-                            if (v >= nv) break;
-                            load_a(st_addr + v * A_BYTES, bar_full, kb + v, m0);
-                            if (!w_sent) load_w(sb + v * TL::B_BYTES, bar_full, kb + v, n0);
+                            for (int v = 0; v < TL::KPS; ++v) {
+                                if (v >= nv) break;
+                                load_a(st_addr + v * A_BYTES, bar_full, kb + v, m0);
+                                if (!w_sent) load_w(sb + v * TL::B_BYTES, bar_full, kb + v, n0);
+                            }
                         }
                         if (issued < STAGES) ++issued;
                         if (++slot == STAGES) {
