@@ -168,7 +168,10 @@ qnn_status qnn_lstm_model_weights(const qnn_lstm_model *m, uint8_t *codes_host, 
  *   h_all    [L][B][T][R], nullable: every layer's output at every frame (diagnostics).
  * x, y, h_state, c_state and h_all may each be host or device memory: host buffers are copied
  * to or from device memory on `stream` inside the call (pinned host memory keeps the copies
- * asynchronous). Activations are quantized per row (one frame of one sequence), weights per
+ * asynchronous). Posteriors (num_classes > 0) for a y in pinned host memory are written there
+ * by the softmax kernel itself, without a device copy and a second transfer. With any host
+ * buffer the results are complete once `stream` has been synchronized. Activations are
+ * quantized per row (one frame of one sequence), weights per
  * gate matrix. The model keeps a device workspace sized for the largest B*T seen; calls on one
  * model must not overlap in time.
  */

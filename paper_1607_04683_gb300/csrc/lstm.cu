@@ -434,11 +434,7 @@ __global__ void __launch_bounds__(256) softmax_rows_kernel(const float *__restri
     __syncthreads();
     mx = s_bcast;
     float s = 0.0f;
-    for (int c = threadIdx.x; c < C; c += 256) {
-        float e = pexp(__fsub_rn(l[c], mx));
-        yr[c] = e;
-        s = __fadd_rn(s, e);
-    }
+    for (int c = threadIdx.x; c < C; c += 256) s = __fadd_rn(s, pexp(__fsub_rn(l[c], mx)));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) s = __fadd_rn(s, __shfl_xor_sync(0xffffffffu, s, o));
     __syncthreads();
@@ -451,7 +447,20 @@ __global__ void __launch_bounds__(256) softmax_rows_kernel(const float *__restri
     }
     __syncthreads();
     s = s_bcast;
-    for (int c = threadIdx.x; c < C; c += 256) yr[c] = __fdiv_rn(yr[c], s);
+    // y is written once (it may be host memory): E(l - max) is recomputed, the same value as above;
+    // 16-byte stores where the rows allow them (each posterior is computed on its own, so the
+    // grouping does not change a value)
+    if ((C & 3) == 0 && ((reinterpret_cast<uintptr_t>(l) | reinterpret_cast<uintptr_t>(yr)) & 15) == 0) {
+        const float4 *l4 = reinterpret_cast<const float4 *>(l);
+        float4 *y4 = reinterpret_cast<float4 *>(yr);
+        for (int v = threadIdx.x; v < C / 4; v += 256) {
+            const float4 lv = l4[v];
+            y4[v] = make_float4(__fdiv_rn(pexp(__fsub_rn(lv.x, mx)), s), __fdiv_rn(pexp(__fsub_rn(lv.y, mx)), s),
+                                __fdiv_rn(pexp(__fsub_rn(lv.z, mx)), s), __fdiv_rn(pexp(__fsub_rn(lv.w, mx)), s));
+        }
+    } else {
+        for (int c = threadIdx.x; c < C; c += 256) yr[c] = __fdiv_rn(pexp(__fsub_rn(l[c], mx)), s);
+    }
 }
 
 // fp32 output layer for the "quant" variant: logits[m][c] = sum_k r[m][k] Wo[c][k] + bo[c].
@@ -809,6 +818,8 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const bool x_dev = is_device_ptr(x), y_dev = is_device_ptr(y);
     const bool hs_dev = h_state && is_device_ptr(h_state), cs_dev = c_state && is_device_ptr(c_state);
     const bool ha_dev = h_all && is_device_ptr(h_all);
+    // posteriors into pinned host memory: the softmax writes them there directly (no staging copy)
+    float *const y_map = (!y_dev && C > 0) ? static_cast<float *>(host_mapped_ptr(y)) : nullptr;
     const PathChoice choice = path_choice();
     if (choice == PathChoice::kAuto || choice == PathChoice::kSmall) {
         bool used = false;
@@ -849,7 +860,7 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const size_t o_qp = acct(B * sizeof(qnn_qparams));
     const size_t o_qs = acct(B * 4);
     const size_t o_lg = acct(C > 0 ? rows * C * 4 : 0);
-    const size_t o_y = y_dev ? 0 : acct(rows * ycols * 4);
+    const size_t o_y = (y_dev || y_map) ? 0 : acct(rows * ycols * 4);
     const size_t o_tc = use_tc ? acct(tc_work_bytes(m, B)) : 0;
     if (need > m->ws_bytes) {
         if (m->ws) {
@@ -878,7 +889,7 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     float *cbuf = reinterpret_cast<float *>(ws + o_c);
     float *mbuf = P > 0 ? reinterpret_cast<float *>(ws + o_m) : nullptr;
     float *lg = C > 0 ? reinterpret_cast<float *>(ws + o_lg) : nullptr;
-    float *yd = y_dev ? y : reinterpret_cast<float *>(ws + o_y);
+    float *yd = y_dev ? y : y_map ? y_map : reinterpret_cast<float *>(ws + o_y);
 
     if (h_state)
         QNN_CUDA_TRY(cudaMemcpyAsync(h0, h_state, L * B * R * 4, cudaMemcpyDefault, st));
@@ -968,7 +979,7 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     } else {
         QNN_CUDA_TRY(cudaMemcpyAsync(yd, in, rows * R * 4, cudaMemcpyDeviceToDevice, st));
     }
-    if (!y_dev) QNN_CUDA_TRY(cudaMemcpyAsync(y, yd, rows * ycols * 4, cudaMemcpyDeviceToHost, st));
+    if (!y_dev && !y_map) QNN_CUDA_TRY(cudaMemcpyAsync(y, yd, rows * ycols * 4, cudaMemcpyDeviceToHost, st));
     (void)hs_dev;
     (void)cs_dev;
     return QNN_OK;

@@ -995,6 +995,8 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
     const bool x_dev = is_device_ptr(x), y_dev = is_device_ptr(y);
     const bool hs_dev = h_state && is_device_ptr(h_state), cs_dev = c_state && is_device_ptr(c_state);
     const bool ha_dev = h_all && is_device_ptr(h_all);
+    // posteriors into pinned host memory: the softmax writes them there directly (no staging copy)
+    float *const y_map = (!y_dev && C > 0) ? static_cast<float *>(host_mapped_ptr(y)) : nullptr;
     const int64_t rows = B * T, ycols = C > 0 ? C : R;
     size_t need = 0;
     auto acct = [&](size_t n) {
@@ -1006,7 +1008,7 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
     const size_t o_hx = acct(sizeof(unsigned long long) * L * rows * R);
     const size_t o_lg = acct(C > 0 ? sizeof(float) * rows * C : 0);
     const size_t o_x = x_dev ? 0 : acct(sizeof(float) * rows * I);
-    const size_t o_y = y_dev ? 0 : acct(sizeof(float) * rows * ycols);
+    const size_t o_y = (y_dev || y_map) ? 0 : acct(sizeof(float) * rows * ycols);
     const size_t o_h = acct(sizeof(float) * L * B * R);
     const size_t o_c = acct(sizeof(float) * L * B * H);
     const size_t o_ha = (h_all && !ha_dev) ? acct(sizeof(float) * L * rows * R) : 0;
@@ -1034,7 +1036,7 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
         QNN_CUDA_TRY(cudaMemcpyAsync(ws + o_x, x, sizeof(float) * rows * I, cudaMemcpyHostToDevice, st));
         xd = reinterpret_cast<const float *>(ws + o_x);
     }
-    float *yd = y_dev ? y : reinterpret_cast<float *>(ws + o_y);
+    float *yd = y_dev ? y : y_map ? y_map : reinterpret_cast<float *>(ws + o_y);
     float *h0 = reinterpret_cast<float *>(ws + o_h), *c0 = reinterpret_cast<float *>(ws + o_c);
     if (h_state)
         QNN_CUDA_TRY(cudaMemcpyAsync(h0, h_state, sizeof(float) * L * B * R, cudaMemcpyDefault, st));
@@ -1063,7 +1065,8 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
         QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, lstm_small_kernel, a));
     }
     if (C > 0) QNN_TRY(launch_softmax_rows(a.logits, rows, C, yd, st));
-    if (!y_dev) QNN_CUDA_TRY(cudaMemcpyAsync(y, yd, sizeof(float) * rows * ycols, cudaMemcpyDeviceToHost, st));
+    if (!y_dev && !y_map)
+        QNN_CUDA_TRY(cudaMemcpyAsync(y, yd, sizeof(float) * rows * ycols, cudaMemcpyDeviceToHost, st));
     if (h_all && !ha_dev)
         QNN_CUDA_TRY(cudaMemcpyAsync(h_all, a.h_all, sizeof(float) * L * rows * R, cudaMemcpyDeviceToHost, st));
     if (h_state && !hs_dev)

@@ -32,6 +32,11 @@ inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s
 // allocations). Pinned or pageable host memory is rejected by the compute calls.
 bool is_device_ptr(const void *p);
 
+// The address under which kernels of the current device reach p when p is pinned (page-locked)
+// host memory mapped into the device's address space; null for any other memory. Kernels that
+// write a host output through it send each byte over the host link once, with no staging copy.
+void *host_mapped_ptr(void *p);
+
 // Library-owned, grow-only device scratch of the current device (one slot per purpose).
 enum ScratchSlot { kScratchReduce = 0, kScratchTc = 1, kScratchCount = 2 };
 qnn_status scratch(ScratchSlot slot, size_t bytes, void **out);

@@ -296,6 +296,32 @@ def test_lstm_streaming_state_and_host_buffers(qnn):
     assert np.array_equal(y_host, full["y"])
 
 
+@pytest.mark.parametrize("path,B,mode", [("small", 2, 1), ("small", 4, 1), ("tc", 64, 1), ("layerwise", 5, 1),
+                                         ("layerwise", 5, 2)])
+def test_lstm_posteriors_into_pinned_host_memory(qnn, path, B, mode, monkeypatch):
+    # a y in pinned host memory is written by the softmax kernel itself (no staging copy): the
+    # same posteriors as a device y, bit for bit, with pinned or pageable inputs; a pageable y
+    # takes the copy
+    monkeypatch.setenv("QNN_LSTM_PATH", path)
+    wl = _small(L=2, I=8, H=32, C=300, B=B, T=5, mode=mode)
+    params, x = wl.make()
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, gpu(params))
+    y_dev = model.forward(gpu(x))
+    torch.cuda.synchronize()
+    y_dev = y_dev.cpu().numpy()
+    assert np.max(np.abs(y_dev - _oracle(wl, params, x)["y"])) <= SOFTMAX_TOL
+    for xin in (torch.from_numpy(x).pin_memory(), x):
+        y_pin = torch.full((B, wl.frames, wl.num_classes), float("nan")).pin_memory()
+        model.forward(xin, y=y_pin)
+        torch.cuda.synchronize()
+        assert np.array_equal(y_pin.numpy(), y_dev)
+    y_np = model.forward(x)
+    torch.cuda.synchronize()
+    assert np.array_equal(y_np, y_dev)
+    assert qnn.device_status() == qnn.QNN_OK
+
+
 def test_lstm_nonfinite_input_reported(qnn):
     wl = _small(L=1, H=8, B=1, T=3)
     params, x = wl.make()
