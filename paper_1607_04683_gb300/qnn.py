@@ -272,7 +272,9 @@ class LstmModel:
 
     def forward(self, x, y=None, h_state=None, c_state=None, h_all=None, stream=None):
         """x [B, T, I] fp32 (CUDA tensor, or numpy/pinned CPU tensor: copied inside the call).
-        Returns y ([B, T, C] or [B, T, R])."""
+        Returns y ([B, T, C] or [B, T, R]). A y given in pinned CPU memory receives the posteriors
+        from the softmax kernel directly; with any CPU buffer, synchronize the stream before
+        reading it."""
         import torch
         B, T, I = x.shape
         d = self.desc
