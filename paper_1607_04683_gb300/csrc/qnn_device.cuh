@@ -125,18 +125,22 @@ __device__ __forceinline__ float pexp(float x) {
     return __fmul_rn(p, __int_as_float((n + 127) << 23));
 }
 
-__device__ __forceinline__ float psigmoid(float x) { return __fdiv_rn(1.0f, __fadd_rn(1.0f, pexp(-x))); }
+// sigma(x) = 1/(E(-x) + 1) and tanh(x) = 1 - 2/(E(2x) + 1), each quotient correctly rounded.
+// The quotients are taken from the correctly rounded reciprocal r of d = E + 1 (d >= 1): 1/d is r
+// itself, and 2/d is 2 r exactly whenever r is a normal number; where it is not (d > 2^126) the
+// quotient is below 2^-125 and 1 - 2/d rounds to 1 from either.
+__device__ __forceinline__ float psigmoid(float x) { return __frcp_rn(__fadd_rn(1.0f, pexp(-x))); }
 
 __device__ __forceinline__ float ptanh(float x) {
-    return __fsub_rn(1.0f, __fdiv_rn(2.0f, __fadd_rn(pexp(__fmul_rn(2.0f, x)), 1.0f)));
+    return __fsub_rn(1.0f, __fmul_rn(2.0f, __frcp_rn(__fadd_rn(pexp(__fmul_rn(2.0f, x)), 1.0f))));
 }
 
 // psigmoid(x) or ptanh(x) without a branch (lanes of one warp may need different ones): the same
-// operations in the same order, 1/(E(-x) + 1) or 1 - 2/(E(2x) + 1).
+// operations in the same order.
 __device__ __forceinline__ float gate_activation(float x, bool is_tanh) {
     const float e = pexp(is_tanh ? __fmul_rn(2.0f, x) : -x);
-    const float q = __fdiv_rn(is_tanh ? 2.0f : 1.0f, __fadd_rn(e, 1.0f));
-    return is_tanh ? __fsub_rn(1.0f, q) : q;
+    const float r = __frcp_rn(__fadd_rn(e, 1.0f));
+    return is_tanh ? __fsub_rn(1.0f, __fmul_rn(2.0f, r)) : r;
 }
 
 // LSTM cell update from the gate activations (no peepholes): c' = f c + i g; returns m = o tanh(c').
