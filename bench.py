@@ -3,8 +3,11 @@
 
 A step is one qnn_lstm_forward over one batch of synthetic frames: per-frame activation
 quantization, the integer products of every layer, recovery fused with the gates and the cell
-update, the 8-bit output layer and its softmax. Default workload: 5 LSTM layers of 500 cells,
-40-dimensional input frames, 2000-class 8-bit softmax layer, batch 1, T = 300 frames.
+update, the 8-bit output layer and its softmax. Default workload: the largest single-GPU one, a
+projected LSTM (LSTMP) of 5 layers of 2048 cells with 512-unit projections, 80-dimensional input
+frames, an 8192-class 8-bit softmax layer, batch 1024, T = 1000 frames. The same line also
+carries the standalone quantized product at 16384 x 8192 x 8192 (`int8_gemm`) and the batch-1
+5 x 500-cell workload (`batch1`).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl reference]
 
@@ -30,7 +33,8 @@ sys.path.insert(0, ROOT)
 from paper_1607_04683_gb300 import inputs  # noqa: E402
 
 METRIC = "quantized LSTM frames/sec at batch B; int8 GEMM TOPS as % of GB300 int8 peak"
-DEFAULT_WORKLOAD = inputs.LSTM_5x500_B1.name
+DEFAULT_WORKLOAD = inputs.LSTMP_5x2048P512_B1024.name
+GEMM_SHAPE = inputs.QmatmulShape(16384, 8192, 8192)  # the largest product of the standalone sweep
 L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
 
 
@@ -42,6 +46,7 @@ def parse():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(inputs.LSTM_WORKLOADS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true", help="skip the int8_gemm and batch1 keys")
     ap.add_argument("--sweep", action="store_true", help="standalone quantized matmul sweep instead")
     ap.add_argument("--shape", default="", help="with --sweep: one shape M,N,K only")
     ap.add_argument("--stream", action="store_true",
@@ -236,30 +241,52 @@ def oracle_frames_per_s(wl, params, x, min_seconds=8.0, max_frames=None, reps_ma
     return frames / dt, frames, dt
 
 
-def run_reference(args, wl, rank, world):
-    if rank != 0:
-        return 0
-    params, x = wl.make(batch=1)
-    per_frame_ops = ops_per_frame(wl)
-    # a step: the oracle on the first sequence's first frames, bounded to ~1-3 s
-    sample_frames = max(1, min(wl.frames, int(2.0e9 / max(per_frame_ops, 1))))
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def oracle_frames_per_s_threads(wl, params, x, frames, threads):
+    """The oracle on `threads` sequences at once, one host thread each (its C calls release the
+    interpreter lock, so they run in parallel; the oracle itself stays single-threaded per call)."""
+    from concurrent.futures import ThreadPoolExecutor
+
     import oracle
     d = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
-    xs = x[:1, :sample_frames]
-    for _ in range(args.warmup):
-        oracle.lstm_forward(d, params, xs)
+    seqs = [x[b % x.shape[0]: b % x.shape[0] + 1, :frames] for b in range(threads)]
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        oracle.lstm_forward(d, params, xs)
+    with ThreadPoolExecutor(max_workers=threads) as ex:
+        list(ex.map(lambda xs: oracle.lstm_forward(d, params, xs), seqs))
     dt = time.perf_counter() - t0
-    fps = args.steps * sample_frames / dt
-    sample = f"sequence 0, first {sample_frames} frames of {wl.frames}, per step"
+    return threads * frames / dt, dt
+
+
+def run_reference(args, wl, rank, world):
+    """The CPU oracle as it stands, on the host's cores: each step runs the oracle on one sequence
+    per core (one host thread each), every sequence cut to its first frames so that a step takes
+    about a second or two."""
+    if rank != 0:
+        return 0
+    cores = host_cores()
+    params, x = wl.make(batch=min(wl.batch, cores))
+    per_frame_ops = ops_per_frame(wl)
+    sample_frames = max(1, min(wl.frames, int(2.0e9 / max(per_frame_ops, 1))))
+    for _ in range(args.warmup):
+        oracle_frames_per_s_threads(wl, params, x, sample_frames, cores)
+    dt = 0.0
+    for _ in range(args.steps):
+        dt += oracle_frames_per_s_threads(wl, params, x, sample_frames, cores)[1]
+    fps = args.steps * cores * sample_frames / dt
+    sample = (f"per step: sequences 0..{cores - 1} (repeating past the batch), first {sample_frames} frames of "
+              f"{wl.frames} each, one host thread per sequence")
     line = {
         "impl": "reference", "metric": METRIC, "value": fps, "unit": "frames/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u8", "data": "synthetic",
         "config": workload_config(wl),
-        "cpu_baseline": {"value": fps, "unit": "frames/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": fps, "unit": "frames/s", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": fps, "unit": "frames/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -421,8 +448,11 @@ def run_ours(args, wl, rank, world, local):
         tfs = flops / avg_s / 1e12
         traffic = traffic_record(kname, wl.name, ["qgemm_tc.cu", "qnn_device.cuh"])
         if gates_fused(wl):
-            roofline = {"bound": "tensor", "kernel": kname, "achieved": tfs, "peak": peaks["bf16_tflops"],
-                        "unit": "TFLOP/s", "frac": tfs / peaks["bf16_tflops"], "peak_kind": peak_kind,
+            # the kernel runs inside a long step (thousands of launches per pass): the sustained peak
+            tpk = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+            roofline = {"bound": "tensor", "kernel": kname, "achieved": tfs, "peak": tpk,
+                        "unit": "TFLOP/s", "frac": tfs / tpk,
+                        "peak_kind": f"{peak_kind} (fp16/bf16 dense, sustained)",
                         "traffic": traffic, "alg_flops_per_launch": flops, "alg_bytes_per_launch": alg,
                         "hbm_gbs": gbs, "hbm_frac": gbs / peaks["hbm_gbs"], "input_product": "fused",
                         "avg_launch_ms": avg_s * 1e3, "share_of_step": share}
@@ -443,14 +473,117 @@ def run_ours(args, wl, rank, world, local):
                 "d2h_bytes_per_step": int(wl.batch * wl.frames * ycols * 4)},
         "clocks": clk.summary(),
     }
+    if world == 1 and not args.no_extras:
+        line["int8_gemm"] = gemm_metric(qnn, torch, peaks, peak_kind, flush, max(5, args.steps))
+        line["batch1"] = batch1_metric(qnn, torch, dev, flush, args.steps, args.warmup)
     if world == 1 and not args.no_cpu_baseline:
-        fps, frames, dt = oracle_frames_per_s(wl, params, x, min_seconds=8.0,
-                                              max_frames=max(1, min(wl.frames, int(3.0e9 / ops_per_frame(wl)))))
+        sample_frames = min(wl.frames, max(1, int(3.0e9 / ops_per_frame(wl))))
+        fps, frames, dt = oracle_frames_per_s(wl, params, x, min_seconds=8.0, max_frames=sample_frames)
         line["cpu_baseline"] = {"value": fps, "unit": "frames/s", "cores": 1, "kind": "oracle",
-                                "sample": f"sequence 0 frames 0..{min(wl.frames, max(1, int(3.0e9 / ops_per_frame(wl))))}"
+                                "sample": f"sequence 0 frames 0..{sample_frames}"
                                           f", repeated: {frames} frames in {dt:.1f} s, single thread"}
+        cores = host_cores()
+        fps_mt, dt_mt = oracle_frames_per_s_threads(wl, params, x, sample_frames, cores)
+        line["cpu_baseline_mt"] = {"value": fps_mt, "unit": "frames/s", "cores": cores, "kind": "oracle",
+                                   "sample": f"sequences 0..{cores - 1}, frames 0..{sample_frames} each, one host "
+                                             f"thread per sequence on {cores} cores (os.sched_getaffinity): "
+                                             f"{cores * sample_frames} frames in {dt_mt:.1f} s"}
     print(json.dumps(line), flush=True)
     return 0
+
+
+def gemm_metric(qnn, torch, peaks, peak_kind, flush, reps):
+    """The standalone quantized product at its largest sweep shape, 16384 x 8192 x 8192, codes in
+    and fp32 out (eq. 1 offsets and eq. 3 recovery in the epilogue): tera-operations per second of
+    the tensor-core product kernel alone and of the whole qnn_qmatmul call (which also converts both
+    operands' codes to centered fp16 on every call), against the measured fp16 tensor peak (the
+    datapath the exact product runs on) and the measured peak of the warp-level u8 integer MMA."""
+    shape = GEMM_SHAPE
+    W, A = inputs.make_qmatmul_operands(shape)
+    Ag, Wg = torch.from_numpy(A).cuda(), torch.from_numpy(W).cuda()
+    del W, A
+    cw, pw, cs = qnn.qnn_quantize(Wg, qnn.PER_MATRIX)
+    ca, pa, ra = qnn.qnn_quantize(Ag, qnn.PER_MATRIX)
+    del Ag, Wg
+    Y = torch.empty((shape.M, shape.N), dtype=torch.float32, device="cuda")
+    for _ in range(2):
+        qnn.qnn_qmatmul(ca, pa, 0, ra, cw, pw, cs, out=Y)
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(reps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        qnn.qnn_qmatmul(ca, pa, 0, ra, cw, pw, cs, out=Y)
+        b.record()
+        b.synchronize()
+        ts.append(a.elapsed_time(b) / 1e3)
+    qnn.profile_read()
+    qnn.profile_enable(True)
+    for _ in range(reps):
+        flush.zero_()
+        qnn.qnn_qmatmul(ca, pa, 0, ra, cw, pw, cs, out=Y)
+    torch.cuda.synchronize()
+    qnn.profile_enable(False)
+    prof = qnn.profile_read()
+    assert qnn.device_status() == qnn.QNN_OK
+    n, kms = prof["qgemm_tc"]
+    t_kernel = kms / n / 1e3
+    t_call = statistics.median(ts)
+    ops = 2.0 * shape.M * shape.N * shape.K
+    imma = qnn.measure_peak(0)
+    pk = peaks["bf16_tflops"]  # a kernel timed alone: the burst peak
+    del ca, cw, Y
+    torch.cuda.empty_cache()
+    return {"M": shape.M, "N": shape.N, "K": shape.K, "unit": "TOP/s",
+            "datapath": "tcgen05 kind::f16 on centered codes (exact integer sums; sm_103a has no kind::i8)",
+            "kernel_tops": ops / t_kernel / 1e12, "kernel_ms": t_kernel * 1e3,
+            "call_tops": ops / t_call / 1e12, "call_ms": t_call * 1e3,
+            "centering_ms": (prof["center_fp16"][1] / prof["center_fp16"][0]) if "center_fp16" in prof else None,
+            "peak": pk, "peak_kind": f"{peak_kind} (fp16/bf16 dense, burst)",
+            "frac_kernel": ops / t_kernel / 1e12 / pk, "frac_call": ops / t_call / 1e12 / pk,
+            "mma_u8_peak_tops": imma, "vs_mma_u8_peak_kernel": ops / t_kernel / 1e12 / imma,
+            "l2": "flushed before every timed call"}
+
+
+def batch1_metric(qnn, torch, dev, flush, steps, warmup):
+    """The batch-1 workload (5 x 500 cells, 2000 classes, T = 300): frames per second of whole
+    forward passes, and the per-frame time of the batch-of-few kernel against the measured floor of
+    its per-frame synchronisation."""
+    wl = inputs.LSTM_5x500_B1
+    params, x = wl.make()
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, torch.from_numpy(params).to(dev))
+    xd = torch.from_numpy(x).to(dev)
+    yd = torch.empty((1, wl.frames, wl.num_classes), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    for _ in range(max(3, warmup)):
+        model.forward(xd, y=yd)
+    torch.cuda.synchronize()
+    ms = []
+    for _ in range(steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        model.forward(xd, y=yd)
+        b.record(stream)
+        b.synchronize()
+        ms.append(a.elapsed_time(b))
+    qnn.profile_read()
+    qnn.profile_enable(True)
+    for _ in range(steps):
+        model.forward(xd, y=yd)
+    torch.cuda.synchronize()
+    qnn.profile_enable(False)
+    prof = qnn.profile_read()
+    assert qnn.device_status() == qnn.QNN_OK
+    n, kms = prof["lstm_small"]
+    us_frame = kms / n * 1e3 / wl.frames
+    floor = qnn.measure_exchange_floor((wl.hidden + 31) // 32, 20000)
+    model.close()
+    return {"workload": wl.name, "value": wl.frames * steps / (sum(ms) / 1e3), "unit": "frames/s",
+            "ms_per_step": sum(ms) / steps, "steps": steps, "kernel": "lstm_small",
+            "us_per_frame": us_frame, "floor_us_per_frame": floor, "latency_frac": floor / us_frame}
 
 
 def run_sweep(args):

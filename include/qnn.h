@@ -179,6 +179,21 @@ qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_
                             float *c_state, float *h_all, void *stream);
 
 /*
+ * qnn_lstm_forward_logits — qnn_lstm_forward that also returns the output layer's values before
+ * the softmax (Sec. 5: "quant-all" takes the softmax layer's product in 8 bits, "quant" in float).
+ *   logits   [B][T][C] fp32, host or device memory, caller-owned, nullable (NULL: the call is
+ *            qnn_lstm_forward). logits[b][t][c] is exactly the value the softmax receives: with
+ *            QNN_OUT_QUANT the recovered product of the top layer's quantized outputs with the
+ *            output weights, eq. (1) and eq. (3), plus the output bias (Fig. 1); with QNN_OUT_FLOAT
+ *            the fp32 product plus the bias. With frame stacking T is the stacked length T'.
+ * Other arguments and behaviour as for qnn_lstm_forward. QNN_ERR_INVALID_ARG if logits is given
+ * for a model without an output layer (num_classes == 0). The copy is made on `stream` after the
+ * output product; a host buffer is complete once the stream has been synchronized.
+ */
+qnn_status qnn_lstm_forward_logits(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *logits,
+                                   float *h_state, float *c_state, float *h_all, void *stream);
+
+/*
  * Streaming server mode — frame-at-a-time inference with a resident kernel (the embedded,
  * frame-by-frame setting of Sec. 1 and Sec. 3.1, where inputs are quantized on the fly as they
  * arrive). One launch of the batch-of-few dataflow kernel stays resident for `chunk` frames and
@@ -243,6 +258,8 @@ qnn_status qnn_stack_frames(const float *x, int64_t B, int64_t T, int64_t I, int
  *     one entry.
  *   status   device int, nullable, caller-owned: QNN_ERR_NONFINITE is written into it (if it is
  *     still 0) when the matrix holds NaN or +-Inf; the codes are then unspecified.
+ *   A pointer that is not device memory of the current device (x, codes, params, and code_sums or
+ *   status when given) returns QNN_ERR_INVALID_ARG before anything runs.
  * Limits: rows <= 524288 (its scratch holds one partial range per 32 rows); larger inputs return
  * QNN_ERR_INVALID_ARG before anything runs.
  * Scratch: a 128 KiB + 256 B static device array inside the library, held on every GPU that loads

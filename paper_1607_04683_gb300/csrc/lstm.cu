@@ -804,9 +804,13 @@ qnn_status stack_input(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, 
 
 }  // namespace
 
-extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y,
-                                       float *h_state, float *c_state, float *h_all, void *stream) {
+namespace {
+
+// qnn_lstm_forward with an optional copy of the output layer's logits ([B][T'][C], host or device).
+qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *logits,
+                        float *h_state, float *c_state, float *h_all, void *stream) {
     if (!m || B < 0 || T < 0) return QNN_ERR_INVALID_ARG;
+    if (logits && m->C == 0) return QNN_ERR_INVALID_ARG;
     if (B == 0 || T == 0) return QNN_OK;
     if (!x || !y) return QNN_ERR_INVALID_ARG;
     cudaStream_t st = as_stream(stream);
@@ -823,7 +827,7 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     const PathChoice choice = path_choice();
     if (choice == PathChoice::kAuto || choice == PathChoice::kSmall) {
         bool used = false;
-        QNN_TRY(small_path_forward(m, x, B, T, y, h_state, c_state, h_all, st, &used));
+        QNN_TRY(small_path_forward(m, x, B, T, y, logits, h_state, c_state, h_all, st, &used));
         if (used) return QNN_OK;
         if (choice == PathChoice::kSmall) return QNN_ERR_INVALID_ARG;
     }
@@ -975,6 +979,7 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
             float_linear_kernel<<<grid, 256, 0, st>>>(in, rows, (int)R, m->wo_f, (int)C, m->bo, lg);
             QNN_CUDA_TRY(cudaGetLastError());
         }
+        if (logits) QNN_CUDA_TRY(cudaMemcpyAsync(logits, lg, rows * C * 4, cudaMemcpyDefault, st));
         QNN_TRY(launch_softmax_rows(lg, rows, C, yd, st));
     } else {
         QNN_CUDA_TRY(cudaMemcpyAsync(yd, in, rows * R * 4, cudaMemcpyDeviceToDevice, st));
@@ -983,4 +988,17 @@ extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_
     (void)hs_dev;
     (void)cs_dev;
     return QNN_OK;
+}
+
+}  // namespace
+
+extern "C" qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y,
+                                       float *h_state, float *c_state, float *h_all, void *stream) {
+    return forward_impl(m, x, B, T, y, nullptr, h_state, c_state, h_all, stream);
+}
+
+extern "C" qnn_status qnn_lstm_forward_logits(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y,
+                                              float *logits, float *h_state, float *c_state, float *h_all,
+                                              void *stream) {
+    return forward_impl(m, x, B, T, y, logits, h_state, c_state, h_all, stream);
 }

@@ -74,9 +74,9 @@ struct qnn_lstm_model {
 namespace qnn {
 // Runs qnn_lstm_forward on the batch-of-few persistent path (lstm_small.cu) if the model and
 // batch qualify; *used tells whether it ran (false: the caller takes the layer-by-layer path).
-// Arguments as for qnn_lstm_forward.
-qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
-                              float *c_state, float *h_all, cudaStream_t st, bool *used);
+// Arguments as for qnn_lstm_forward_logits (logits nullable).
+qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *logits,
+                              float *h_state, float *c_state, float *h_all, cudaStream_t st, bool *used);
 // Streaming with the batch-of-few kernel (stream.cu): one launch serves T frames that the host
 // supplies while it runs. Buffers: xs [B][T][I] tagged input rows (host-mapped), out [B][T][C]
 // posteriors (or [B][T][R] top-layer outputs without an output layer; host-mapped), done

@@ -979,8 +979,8 @@ PathChoice path_choice() {
     return PathChoice::kAuto;
 }
 
-qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
-                              float *c_state, float *h_all, cudaStream_t st, bool *used) {
+qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *logits,
+                              float *h_state, float *c_state, float *h_all, cudaStream_t st, bool *used) {
     *used = false;
     const int64_t L = m->L, I = m->I, H = m->H, C = m->C, R = m->R;
     SmallGeom geo;
@@ -1064,6 +1064,7 @@ qnn_status small_path_forward(qnn_lstm_model *m, const float *x, int64_t B, int6
         ProfScope prof("lstm_small", st);
         QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, lstm_small_kernel, a));
     }
+    if (logits) QNN_CUDA_TRY(cudaMemcpyAsync(logits, a.logits, sizeof(float) * rows * C, cudaMemcpyDefault, st));
     if (C > 0) QNN_TRY(launch_softmax_rows(a.logits, rows, C, yd, st));
     if (!y_dev && !y_map)
         QNN_CUDA_TRY(cudaMemcpyAsync(y, yd, sizeof(float) * rows * ycols, cudaMemcpyDeviceToHost, st));

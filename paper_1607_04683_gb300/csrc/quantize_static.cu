@@ -152,6 +152,11 @@ extern "C" qnn_status qnn_quantize_matrix_static(const float *x, int64_t rows, i
     if (rows <= 0 || cols <= 0 || ldx < cols || ldc < cols || cols > INT32_MAX) return QNN_ERR_INVALID_ARG;
     if (rows > kStaticMaxRows) return QNN_ERR_INVALID_ARG;  // the static scratch holds 16384 block partials
     if (!x || !codes || !params) return QNN_ERR_INVALID_ARG;
+    // every pointer must be device memory of the current device: a host pointer is rejected here
+    // rather than faulting in a kernel
+    if (!is_device_ptr(x) || !is_device_ptr(codes) || !is_device_ptr(params) ||
+        (code_sums && !is_device_ptr(code_sums)) || (status && !is_device_ptr(status)))
+        return QNN_ERR_INVALID_ARG;
     void *scratch = nullptr;
     QNN_TRY(static_scratch_address(&scratch));
     cudaStream_t st = as_stream(stream);

@@ -35,6 +35,7 @@ class LstmWorkload:
     forget_bias: float = 0.0
     seq_mean_range: float = 0.0  # per-sequence mean offset ~ U(-r, r) added to x
     output_mode: int = 1  # 0 none, 1 quantized output layer ("quant-all"), 2 float output layer ("quant")
+    out_w_range: float = 0.0  # output weights ~ U(-r, r) if r > 0 (spreads the logits), else w_range
 
     @property
     def R(self) -> int:
@@ -75,13 +76,19 @@ class LstmWorkload:
                 out[off:off + wp.size] = wp.ravel()
                 off += wp.size
         if self.num_classes > 0:
-            wo = rng.uniform(-a, a, (self.num_classes, R)).astype(np.float32)
+            ao = self.out_w_range if self.out_w_range > 0 else a
+            wo = rng.uniform(-ao, ao, (self.num_classes, R)).astype(np.float32)
             out[off:off + wo.size] = wo.ravel()
             off += wo.size
             out[off:off + self.num_classes] = 0.0
             off += self.num_classes
         assert off == out.size
         return out
+
+    def out_weights(self, params: np.ndarray) -> np.ndarray:
+        """The output layer's weights Wo [C, R] inside a packed parameter buffer."""
+        C, R = self.num_classes, self.R
+        return params[params.size - C * R - C: params.size - C].reshape(C, R)
 
     def make_frames(self, rng: np.random.Generator, batch: int | None = None, frames: int | None = None) -> np.ndarray:
         B = self.batch if batch is None else batch

@@ -32,6 +32,7 @@ QPARAMS_DTYPE = np.dtype([("vmin", "<f4"), ("vmax", "<f4"), ("Q", "<f4"), ("z", 
 # Every symbol the header declares (checked by the CPU test that loads the library).
 EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmul", "qnn_lstm_param_count",
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
+           "qnn_lstm_forward_logits",
            "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static",
            "qnn_selftest_s64_to_f32", "qnn_stack_frames", "qnn_selftest_wait_timeout", "qnn_lstm_stream_open",
            "qnn_lstm_stream_push", "qnn_lstm_stream_pull", "qnn_lstm_stream_close", "qnn_measure_exchange_floor")
@@ -79,6 +80,8 @@ def lib():
         L.qnn_lstm_model_weights.restype = i32
         L.qnn_lstm_forward.argtypes = [P, P, i64, i64, P, P, P, P, P]
         L.qnn_lstm_forward.restype = i32
+        L.qnn_lstm_forward_logits.argtypes = [P, P, i64, i64, P, P, P, P, P, P]
+        L.qnn_lstm_forward_logits.restype = i32
         L.qnn_profile_enable.argtypes = [i32]
         L.qnn_profile_enable.restype = i32
         L.qnn_profile_read.argtypes = [i32, P, P, P, C.POINTER(i32)]
@@ -270,11 +273,12 @@ class LstmModel:
         _check(lib().qnn_lstm_model_weights(self._h, _p(codes), _p(prm), C.byref(nu)), "qnn_lstm_model_weights")
         return codes, prm
 
-    def forward(self, x, y=None, h_state=None, c_state=None, h_all=None, stream=None):
+    def forward(self, x, y=None, h_state=None, c_state=None, h_all=None, stream=None, logits=None):
         """x [B, T, I] fp32 (CUDA tensor, or numpy/pinned CPU tensor: copied inside the call).
         Returns y ([B, T, C] or [B, T, R]). A y given in pinned CPU memory receives the posteriors
         from the softmax kernel directly; with any CPU buffer, synchronize the stream before
-        reading it."""
+        reading it. logits: optional [B, T, C] buffer (host or device) that receives the output
+        layer's values before the softmax (qnn_lstm_forward_logits)."""
         import torch
         B, T, I = x.shape
         d = self.desc
@@ -286,8 +290,12 @@ class LstmModel:
                 y = np.empty((B, T, ycols), np.float32)
             else:
                 y = torch.empty((B, T, ycols), dtype=torch.float32, device=x.device)
-        _check(lib().qnn_lstm_forward(self._h, _p(x), B, x.shape[1], _p(y), _p(h_state), _p(c_state), _p(h_all),
-                                      _stream(stream)), "qnn_lstm_forward")
+        if logits is None:
+            _check(lib().qnn_lstm_forward(self._h, _p(x), B, x.shape[1], _p(y), _p(h_state), _p(c_state),
+                                          _p(h_all), _stream(stream)), "qnn_lstm_forward")
+        else:
+            _check(lib().qnn_lstm_forward_logits(self._h, _p(x), B, x.shape[1], _p(y), _p(logits), _p(h_state),
+                                                 _p(c_state), _p(h_all), _stream(stream)), "qnn_lstm_forward_logits")
         return y
 
 

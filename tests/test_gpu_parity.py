@@ -2,21 +2,22 @@
 
 Bar: codes, parameters, code sums and int32 accumulators bit-exact; every LSTM layer output
 bit-exact (the whole recurrence is the same sequence of fp32 operations on both sides, so any
-difference would be a bug); softmax outputs within 1e-4 absolute (their sums run in a different
-order on the GPU).
+difference would be a bug); the 8-bit output layer's logits bit-exact; posteriors within 1e-4
+absolute and 1e-5 relative (their sums run in a different order on the GPU). The rules are in
+tests/parity.py.
 """
 import ctypes
+from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
 import pytest
 
 import oracle
+import parity
 from paper_1607_04683_gb300 import inputs
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
-
-SOFTMAX_TOL = 1e-4
 
 
 @pytest.fixture(scope="module")
@@ -218,40 +219,40 @@ def test_qmatmul_sweep_full_size_sampled(qnn, KN):
 # qnn_lstm_forward
 # ------------------------------------------------------------------------------------------
 
-def _small(name="t", L=2, I=7, H=9, P=0, C=0, B=2, T=6, seed=5, mode=None, fb=1.0, w=0.5, mu=0.0):
+def _small(name="t", L=2, I=7, H=9, P=0, C=0, B=2, T=6, seed=5, mode=None, fb=1.0, w=0.5, mu=0.0, wo=0.0):
     return inputs.LstmWorkload(name, seed=seed, num_layers=L, input_dim=I, hidden=H, proj=P, num_classes=C,
                                batch=B, frames=T, w_range=w, forget_bias=fb, seq_mean_range=mu,
-                               output_mode=(mode if mode is not None else (1 if C > 0 else 0)))
+                               output_mode=(mode if mode is not None else (1 if C > 0 else 0)), out_w_range=wo)
 
 
-def _gpu_forward(qnn, wl, params, x, h_all=True, h0=None, c0=None):
+def _gpu_forward(qnn, wl, params, x, h_all=True, h0=None, c0=None, logits=True):
     d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
     model = qnn.LstmModel(d, gpu(params))
     B, T, _ = x.shape
     ha = torch.empty((wl.num_layers, B, T, wl.R), dtype=torch.float32, device="cuda") if h_all else None
     hs = gpu(h0) if h0 is not None else torch.zeros((wl.num_layers, B, wl.R), dtype=torch.float32, device="cuda")
     cs = gpu(c0) if c0 is not None else torch.zeros((wl.num_layers, B, wl.hidden), dtype=torch.float32, device="cuda")
-    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha)
+    lg = None
+    if logits and wl.num_classes > 0:
+        lg = torch.full((B, T, wl.num_classes), float("nan"), dtype=torch.float32, device="cuda")
+    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha, logits=lg)
     assert qnn.device_status() == qnn.QNN_OK
     out = {"y": y.cpu().numpy(), "h": hs.cpu().numpy(), "c": cs.cpu().numpy(), "model": model}
     if h_all:
         out["h_all"] = ha.cpu().numpy()
+    if lg is not None:
+        out["logits"] = lg.cpu().numpy()
     return out
 
 
-def _compare(got, ref, wl):
-    if "h_all" in got and "h_all" in ref:
-        for l in range(wl.num_layers):
-            assert np.array_equal(got["h_all"][l], ref["h_all"][l]), f"layer {l} outputs differ"
-    assert np.array_equal(got["h"], ref["h"]) and np.array_equal(got["c"], ref["c"])
-    if wl.num_classes > 0:
-        assert np.max(np.abs(got["y"] - ref["y"])) <= SOFTMAX_TOL
-    else:
-        assert np.array_equal(got["y"], ref["y"])
+def _compare(got, ref, wl, params=None):
+    w_out = wl.out_weights(params) if (params is not None and wl.num_classes > 0) else None
+    parity.compare(got, ref, wl.num_layers, wl.num_classes, wl.output_mode, w_out)
 
 
 def _oracle(wl, params, x, **kw):
     d = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    kw.setdefault("want_logits", wl.num_classes > 0)
     return oracle.lstm_forward(d, params, x, **kw)
 
 
@@ -259,7 +260,13 @@ SMALL_CASES = [dict(), dict(L=1, I=3, H=4, B=1, T=9), dict(L=3, H=16, C=11, B=3)
                dict(L=2, I=6, H=10, P=4, C=7, B=2, T=5), dict(L=2, I=80, H=130, P=48, C=70, B=20, T=6),
                dict(L=2, H=12, C=5, mode=2), dict(L=1, I=40, H=500, B=70, T=3, C=2000, w=0.08),
                dict(L=2, I=40, H=64, C=9, B=6, T=5), dict(L=2, I=40, H=50, P=16, C=9, B=6, T=4),
-               dict(L=3, I=5, H=8, B=65, T=3, mu=0.5)]
+               dict(L=3, I=5, H=8, B=65, T=3, mu=0.5),
+               # output weights wide enough that the posteriors are far from uniform (logits over
+               # several units), on the batch-of-few, integer-MMA and tensor-core paths
+               dict(L=2, I=40, H=64, C=2000, B=2, T=7, w=0.1, wo=2.0),
+               dict(L=2, I=40, H=64, C=2000, B=9, T=4, w=0.1, wo=2.0),
+               dict(L=2, I=40, H=64, P=32, C=2000, B=70, T=3, w=0.1, wo=2.0),
+               dict(L=2, I=40, H=64, C=300, B=9, T=4, w=0.1, wo=2.0, mode=2)]
 
 
 @pytest.mark.parametrize("cfg", SMALL_CASES)
@@ -268,7 +275,9 @@ def test_lstm_small_bit_exact(qnn, cfg):
     params, x = wl.make()
     got = _gpu_forward(qnn, wl, params, x)
     ref = _oracle(wl, params, x, want_h_all=True)
-    _compare(got, ref, wl)
+    _compare(got, ref, wl, params)
+    if wl.out_w_range > 0:  # the case is meant to spread the posteriors: check that it does
+        assert ref["y"].max() > 10.0 / wl.num_classes
 
 
 def test_lstm_weight_codes_bit_exact(qnn):
@@ -310,7 +319,7 @@ def test_lstm_posteriors_into_pinned_host_memory(qnn, path, B, mode, monkeypatch
     y_dev = model.forward(gpu(x))
     torch.cuda.synchronize()
     y_dev = y_dev.cpu().numpy()
-    assert np.max(np.abs(y_dev - _oracle(wl, params, x)["y"])) <= SOFTMAX_TOL
+    parity.check_posteriors(y_dev, _oracle(wl, params, x)["y"])
     for xin in (torch.from_numpy(x).pin_memory(), x):
         y_pin = torch.full((B, wl.frames, wl.num_classes), float("nan")).pin_memory()
         model.forward(xin, y=y_pin)
@@ -320,6 +329,36 @@ def test_lstm_posteriors_into_pinned_host_memory(qnn, path, B, mode, monkeypatch
     torch.cuda.synchronize()
     assert np.array_equal(y_np, y_dev)
     assert qnn.device_status() == qnn.QNN_OK
+
+
+@pytest.mark.parametrize("path,B", [("small", 2), ("layerwise", 5), ("tc", 64)])
+def test_lstm_logits_into_host_memory(qnn, path, B, monkeypatch):
+    # qnn_lstm_forward_logits with the logits in pinned and in pageable host memory: the same bits
+    # as into device memory and as the oracle's
+    monkeypatch.setenv("QNN_LSTM_PATH", path)
+    wl = _small(L=2, I=8, H=32, C=300, B=B, T=5, wo=1.0)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x)
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, gpu(params))
+    for lg in (torch.full((B, wl.frames, wl.num_classes), float("nan")).pin_memory(),
+               np.full((B, wl.frames, wl.num_classes), np.nan, np.float32)):
+        y = model.forward(gpu(x), logits=lg)
+        torch.cuda.synchronize()
+        lgn = lg.numpy() if hasattr(lg, "numpy") else lg
+        parity.check_logits(lgn, ref["logits"], 1)
+        parity.check_posteriors(y.cpu().numpy(), ref["y"])
+    assert qnn.device_status() == qnn.QNN_OK
+
+
+def test_lstm_logits_need_an_output_layer(qnn):
+    wl = _small(L=1, H=8, B=1, T=3)
+    params, x = wl.make()
+    model = qnn.LstmModel(qnn.lstm_desc(1, wl.input_dim, wl.hidden), gpu(params))
+    lg = torch.empty((1, 3, 4), dtype=torch.float32, device="cuda")
+    with pytest.raises(qnn.QnnError) as e:
+        model.forward(gpu(x), logits=lg)
+    assert e.value.status == qnn.QNN_ERR_INVALID_ARG
 
 
 def test_lstm_nonfinite_input_reported(qnn):
@@ -337,40 +376,70 @@ def test_config_small_1x128_full(qnn):
     params, x = wl.make()
     got = _gpu_forward(qnn, wl, params, x)
     ref = _oracle(wl, params, x, want_h_all=True)
-    _compare(got, ref, wl)
+    _compare(got, ref, wl, params)
 
 
 def test_config_5x500_b1_full(qnn):
-    # the benchmarked workload, whole: 5 x 500 cells, 2000 classes, T = 300, batch 1
+    # the batch-1 workload, whole: 5 x 500 cells, 2000 classes, T = 300
     wl = inputs.LSTM_5x500_B1
     params, x = wl.make()
     got = _gpu_forward(qnn, wl, params, x)
     ref = _oracle(wl, params, x, want_h_all=True)
-    _compare(got, ref, wl)
+    _compare(got, ref, wl, params)
+
+
+def _sequences_by_oracle(wl, params, x, seqs):
+    """The oracle on single sequences, in threads (its C calls release the interpreter lock);
+    per-row quantization makes every sequence independent of its batch-mates."""
+    with ThreadPoolExecutor(max_workers=len(seqs)) as ex:
+        return list(ex.map(lambda b: _oracle(wl, params, x[b:b + 1]), seqs))
+
+
+def _check_sequence(got, ref, b, frames=slice(None)):
+    assert np.array_equal(got["h"][:, b], ref["h"][:, 0]) and np.array_equal(got["c"][:, b], ref["c"][:, 0])
+    parity.check_logits(got["logits"][b, frames], ref["logits"][0, frames], 1)
+    parity.check_posteriors(got["y"][b, frames], ref["y"][0, frames])
 
 
 def test_config_5x500_b256_sampled(qnn):
-    # batch 256 x 500 frames on the GPU; the oracle recomputes two whole sequences (per-row
-    # quantization makes every sequence independent of the others).
+    # batch 256 x 500 frames on the GPU; the oracle recomputes two whole sequences: final state,
+    # logits (bit-exact) and posteriors of every frame
     wl = inputs.LSTM_5x500_B256
     params, x = wl.make()
     got = _gpu_forward(qnn, wl, params, x, h_all=False)
-    for b in (0, 173):
-        ref = _oracle(wl, params, x[b:b + 1])
-        assert np.array_equal(got["h"][:, b], ref["h"][:, 0]) and np.array_equal(got["c"][:, b], ref["c"][:, 0])
-        assert np.max(np.abs(got["y"][b] - ref["y"][0])) <= SOFTMAX_TOL
+    seqs = (0, 173)
+    for b, ref in zip(seqs, _sequences_by_oracle(wl, params, x, seqs)):
+        _check_sequence(got, ref, b)
 
 
-def test_config_lstmp_2048_b1024_sampled(qnn):
-    # the large projected model at full batch, a 24-frame prefix (outputs are causal in time);
-    # the oracle recomputes one sequence.
+def test_config_lstmp_2048_b1024_full_length(qnn):
+    # the large projected model at its full size (batch 1024, T = 1000: the recurrence through all
+    # 1000 steps of the tensor-core path); the oracle recomputes two whole sequences, about a
+    # minute each: final (h, c) of every layer bit-exact, logits bit-exact and posteriors on every
+    # 7th frame
     wl = inputs.LSTMP_5x2048P512_B1024
-    params, x = wl.make(frames=24)
-    got = _gpu_forward(qnn, wl, params, x, h_all=False)
-    b = 611
-    ref = _oracle(wl, params, x[b:b + 1])
-    assert np.array_equal(got["h"][:, b], ref["h"][:, 0]) and np.array_equal(got["c"][:, b], ref["c"][:, 0])
-    assert np.max(np.abs(got["y"][b] - ref["y"][0])) <= SOFTMAX_TOL
+    params, x = wl.make()
+    B, T = wl.batch, wl.frames
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, gpu(params))
+    hs = torch.zeros((wl.num_layers, B, wl.R), dtype=torch.float32, device="cuda")
+    cs = torch.zeros((wl.num_layers, B, wl.hidden), dtype=torch.float32, device="cuda")
+    lg = torch.empty((B, T, wl.num_classes), dtype=torch.float32, device="cuda")
+    y = model.forward(gpu(x), h_state=hs, c_state=cs, logits=lg)
+    torch.cuda.synchronize()
+    assert qnn.device_status() == qnn.QNN_OK
+    seqs = (611, 5)
+    frames = slice(0, T, 7)
+    got = {"h": hs.cpu().numpy(), "c": cs.cpu().numpy()}
+    got["logits"] = {b: lg[b, frames].cpu().numpy() for b in seqs}
+    got["y"] = {b: y[b, frames].cpu().numpy() for b in seqs}
+    del y, lg
+    model.close()
+    torch.cuda.empty_cache()
+    for b, ref in zip(seqs, _sequences_by_oracle(wl, params, x, seqs)):
+        assert np.array_equal(got["h"][:, b], ref["h"][:, 0]) and np.array_equal(got["c"][:, b], ref["c"][:, 0])
+        parity.check_logits(got["logits"][b], ref["logits"][0, frames], 1)
+        parity.check_posteriors(got["y"][b], ref["y"][0, frames])
 
 
 # ------------------------------------------------------------------------------------------
@@ -395,7 +464,7 @@ def test_small_and_layerwise_paths_agree(qnn, cfg, monkeypatch):
         qnn.profile_enable(False)
         kernels = qnn.profile_read()
         assert ("lstm_small" in kernels) == (path == "small"), kernels
-        _compare(got, ref, wl)
+        _compare(got, ref, wl, params)
         outs[path] = got
     assert np.array_equal(outs["small"]["y"], outs["layerwise"]["y"])
 
@@ -423,7 +492,7 @@ def test_tc_recurrence_bit_exact(qnn, cfg, bn, monkeypatch):
     qnn.profile_enable(False)
     kernels = qnn.profile_read()
     assert "lstm_gates_tc" in kernels and "lstm_recurrent" not in kernels, kernels
-    _compare(got, ref, wl)
+    _compare(got, ref, wl, params)
 
 
 @pytest.mark.parametrize("fuse", ["1", "0"])
@@ -440,7 +509,7 @@ def test_tc_input_product_fused_and_batched(qnn, cfg, fuse, monkeypatch):
     monkeypatch.setenv("QNN_LSTM_PATH", "tc")
     monkeypatch.setenv("QNN_TC_FUSE_X", fuse)
     got = _gpu_forward(qnn, wl, params, x)
-    _compare(got, ref, wl)
+    _compare(got, ref, wl, params)
 
 
 @pytest.mark.parametrize("bn,fuse", [("32", "1"), ("64", "1"), ("96", "0")])
@@ -455,7 +524,7 @@ def test_tc_recurrence_large_weight_offsets(qnn, bn, fuse, monkeypatch):
     monkeypatch.setenv("QNN_TC_BN", bn)
     monkeypatch.setenv("QNN_TC_FUSE_X", fuse)
     got = _gpu_forward(qnn, wl, params, x)
-    _compare(got, ref, wl)
+    _compare(got, ref, wl, params)
 
 
 def test_tc_recurrence_state_round_trip(qnn, monkeypatch):
@@ -525,11 +594,13 @@ def test_lstm_with_stacked_frames(qnn, path, B, monkeypatch):
     ha = torch.empty((L, B, Tp, H), dtype=torch.float32, device="cuda")
     hs = torch.zeros((L, B, H), dtype=torch.float32, device="cuda")
     cs = torch.zeros((L, B, H), dtype=torch.float32, device="cuda")
-    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha)
+    lg = torch.empty((B, Tp, C), dtype=torch.float32, device="cuda")
+    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha, logits=lg)
     assert qnn.device_status() == qnn.QNN_OK
     assert y.shape == (B, Tp, C)
-    got = {"y": y.cpu().numpy(), "h": hs.cpu().numpy(), "c": cs.cpu().numpy(), "h_all": ha.cpu().numpy()}
-    _compare(got, ref, wl)
+    got = {"y": y.cpu().numpy(), "h": hs.cpu().numpy(), "c": cs.cpu().numpy(), "h_all": ha.cpu().numpy(),
+           "logits": lg.cpu().numpy()}
+    _compare(got, ref, wl, params)
     y_host = model.forward(x)  # host frames: staged inside the call
     assert np.array_equal(y_host, got["y"])
 
@@ -577,7 +648,7 @@ def test_lstm_sub_matrix_units_bit_exact(qnn, path, cfg, nb, monkeypatch):
     params, x = wl.make()
     params = _block_scaled(params, wl, nb, seed=nb)
     od = oracle.desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode, nb)
-    ref = oracle.lstm_forward(od, params, x, want_h_all=True)
+    ref = oracle.lstm_forward(od, params, x, want_h_all=True, want_logits=wl.num_classes > 0)
     d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode,
                       weight_blocks=nb)
     model = qnn.LstmModel(d, gpu(params))
@@ -585,16 +656,19 @@ def test_lstm_sub_matrix_units_bit_exact(qnn, path, cfg, nb, monkeypatch):
     ha = torch.empty((wl.num_layers, B, T, wl.R), dtype=torch.float32, device="cuda")
     hs = torch.zeros((wl.num_layers, B, wl.R), dtype=torch.float32, device="cuda")
     cs = torch.zeros((wl.num_layers, B, wl.hidden), dtype=torch.float32, device="cuda")
+    lg = torch.empty((B, T, wl.num_classes), dtype=torch.float32, device="cuda") if wl.num_classes else None
     qnn.profile_read()
     qnn.profile_enable(True)
-    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha)
+    y = model.forward(gpu(x), h_state=hs, c_state=cs, h_all=ha, logits=lg)
     qnn.profile_enable(False)
     kernels = qnn.profile_read()
     want = {"small": "lstm_small", "tc": "lstm_gates_tc", "layerwise": "lstm_recurrent"}[path]
     assert want in kernels, kernels
     assert qnn.device_status() == qnn.QNN_OK
     got = {"y": y.cpu().numpy(), "h": hs.cpu().numpy(), "c": cs.cpu().numpy(), "h_all": ha.cpu().numpy()}
-    _compare(got, ref, wl)
+    if lg is not None:
+        got["logits"] = lg.cpu().numpy()
+    _compare(got, ref, wl, params)
     codes, prm = model.weights()
     c_ref, p_ref = oracle.lstm_quantize_weights(od, params)
     assert np.array_equal(codes, c_ref) and np.array_equal(prm.view(np.int32), p_ref.view(np.int32))

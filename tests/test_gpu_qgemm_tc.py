@@ -79,6 +79,67 @@ def test_tc_extreme_codes_at_the_exactness_limit(qnn, K, a_code, w_code, monkeyp
     assert np.all(acc.cpu().numpy() == a_code * w_code * K)
 
 
+def _adversarial_rows(g, n, K):
+    """Centered code rows (s = c - 128) that drive partial sums of s_a s_w towards +-2^24 and then
+    add small odd terms: runs of -128 or 127 (products +-16384, +-16256, 16129) followed by +-1 and
+    +-3, sign patterns alternating in blocks of 16 (one MMA's K step) and of 64 (one k-block),
+    random extremes, and random extremes that end in small odd values."""
+    rows = []
+    for i in range(n):
+        kind = i % 6
+        s = np.empty(K, np.int64)
+        if kind == 0:    # a long run of -128, then a tail of +-1 / +-3
+            s[:] = -128
+            tail = min(K, 16 + (i % 48))
+            s[K - tail:] = g.choice([-3, -1, 1, 3], tail)
+        elif kind == 1:  # a run of 127 (products of 16129 or -16256 against -128), odd tail
+            s[:] = 127
+            tail = min(K, 1 + (i % 31))
+            s[K - tail:] = g.choice([-1, 1], tail)
+        elif kind == 2:  # sign alternating in blocks of 16
+            s[:] = np.where((np.arange(K) // 16) % 2 == 0, -128, 127)
+            s[-1] = 1
+        elif kind == 3:  # sign alternating in blocks of 64, an odd term in each block
+            s[:] = np.where((np.arange(K) // 64) % 2 == 0, 127, -128)
+            s[63::64] = 3
+        elif kind == 4:  # random extremes
+            s[:] = g.choice([-128, 127], K)
+        else:            # random extremes, then random small odd values
+            s[:] = g.choice([-128, 127], K)
+            tail = min(K, 8 + (i % 100))
+            s[K - tail:] = g.choice([-3, -1, 1, 3], tail)
+        rows.append(s + 128)
+    return np.array(rows, np.uint8)
+
+
+@pytest.mark.parametrize("K", [256, 512, 1000, 1024, 1025, 2048])
+def test_tc_adversarial_partial_sums_bit_exact(qnn, K, monkeypatch):
+    # the fp16 datapath is exact only if the tensor-memory accumulator keeps every integer up to
+    # 2^24: large partial sums followed by small odd terms, with mixed signs, must come out exact
+    # at K-chunk lengths 256, 512, 1024 and across chunk boundaries
+    monkeypatch.delenv("QNN_TC_BN", raising=False)
+    g = np.random.Generator(np.random.PCG64(K + 17))
+    M, N = 192, 144
+    ca = _adversarial_rows(g, M, K)
+    cw = _adversarial_rows(g, N, K)
+    cw = np.concatenate([cw[:N // 2], 255 - cw[N // 2:]])  # sign-flipped half: sums towards -2^24 too
+    p = np.zeros(1, qnn.QPARAMS_DTYPE)
+    p[0] = (0.0, 1.0, 255.0, 0)
+    ra = ca.astype(np.int64).sum(1).astype(np.int32)
+    cs = cw.astype(np.int64).sum(1).astype(np.int32)
+    ref = oracle.qmatmul(ca, p, 0, cw, p)
+    cent = (ca.astype(np.int64) - 128) @ (cw.astype(np.int64) - 128).T
+    # the centered sums come close to the largest a chunk of min(K, 1024) terms can reach (2^24)
+    assert np.abs(cent).max() > 0.9 * min(K, 1024) * (1 << 14)
+    assert np.count_nonzero(cent % 2) > 0           # and end odd
+    for path in ("tc", "imma"):
+        monkeypatch.setenv("QNN_QGEMM", path)
+        Y, acc = _run(qnn, ca, p, 0, ra, cw, p, cs)
+        assert qnn.device_status() == qnn.QNN_OK
+        assert np.array_equal(acc.cpu().numpy(), ref["acc"]), path
+        assert np.array_equal(Y.cpu().numpy(), ref["y"]), path
+
+
 @pytest.mark.parametrize("K", [64, 1000, 3000])
 def test_tc_large_offsets_bit_exact(qnn, K, monkeypatch):
     """Rows with a narrow range far from zero have large offsets z (eq. 2), so the offset-applied
