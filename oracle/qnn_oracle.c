@@ -32,6 +32,9 @@
  *      of one sequence) inside the LSTM.
  *   R7 output layer: logits = R(Q(r) Wo) + bo then softmax ("quant-all", Sec. 5); the float
  *      variant ("quant") computes the logits in fp64 and rounds them once to fp32.
+ *   R11 softmax normalisation: the paper does not fix its precision; the terms E(l - max) are
+ *      fp32 (R5), their sum and each quotient fp64, rounded once. (A sequential fp32 sum of 8192
+ *      nearly equal terms drifts by a few 1e-5 relative, beyond the 1e-5 bar on the posteriors.)
  *   R9 frame stacking (Sec. 4 frontend): network input t' is the n frames starting at frame
  *      stride*t' (the frame and n-1 frames of right context), concatenated; T' = ceil(T/stride)
  *      inputs; frames past the end of the sequence repeat its last frame.
@@ -345,18 +348,19 @@ static int quantize_row(const float *v, int64_t n, uint8_t *codes, orc_qparams *
     return orc_quantize(v, 1, n, n, ORC_PER_ROW, codes, n, p, NULL);
 }
 
-/* Softmax with the pinned E: exp(l - max) / sum, summed in index order. */
+/* Softmax (R11): y_c = E(l_c - max) / sum_j E(l_j - max) with the pinned E (R5) on fp32
+ * differences; the normalising sum and each quotient are taken in fp64 and rounded once. */
 static void softmax_row(const float *logits, int64_t C, float *y)
 {
     float mx = logits[0];
     for (int64_t c = 1; c < C; ++c)
         if (logits[c] > mx) mx = logits[c];
-    float s = 0.0f;
+    double s = 0.0;
     for (int64_t c = 0; c < C; ++c) {
         y[c] = orc_exp(logits[c] - mx);
-        s = s + y[c];
+        s = s + (double)y[c];
     }
-    for (int64_t c = 0; c < C; ++c) y[c] = y[c] / s;
+    for (int64_t c = 0; c < C; ++c) y[c] = (float)((double)y[c] / s);
 }
 
 /*

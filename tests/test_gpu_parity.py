@@ -263,10 +263,10 @@ SMALL_CASES = [dict(), dict(L=1, I=3, H=4, B=1, T=9), dict(L=3, H=16, C=11, B=3)
                dict(L=3, I=5, H=8, B=65, T=3, mu=0.5),
                # output weights wide enough that the posteriors are far from uniform (logits over
                # several units), on the batch-of-few, integer-MMA and tensor-core paths
-               dict(L=2, I=40, H=64, C=2000, B=2, T=7, w=0.1, wo=2.0),
-               dict(L=2, I=40, H=64, C=2000, B=9, T=4, w=0.1, wo=2.0),
-               dict(L=2, I=40, H=64, P=32, C=2000, B=70, T=3, w=0.1, wo=2.0),
-               dict(L=2, I=40, H=64, C=300, B=9, T=4, w=0.1, wo=2.0, mode=2)]
+               dict(L=2, I=40, H=64, C=2000, B=2, T=7, w=0.3, wo=1.0),
+               dict(L=2, I=40, H=64, C=2000, B=9, T=4, w=0.3, wo=1.0),
+               dict(L=2, I=40, H=64, P=32, C=2000, B=70, T=3, w=0.3, wo=2.0),
+               dict(L=2, I=40, H=64, C=300, B=9, T=4, w=0.3, wo=1.0, mode=2)]
 
 
 @pytest.mark.parametrize("cfg", SMALL_CASES)
@@ -277,7 +277,7 @@ def test_lstm_small_bit_exact(qnn, cfg):
     ref = _oracle(wl, params, x, want_h_all=True)
     _compare(got, ref, wl, params)
     if wl.out_w_range > 0:  # the case is meant to spread the posteriors: check that it does
-        assert ref["y"].max() > 10.0 / wl.num_classes
+        assert ref["y"].max() > 5.0 / wl.num_classes and ref["y"].min() < 0.1 / wl.num_classes
 
 
 def test_lstm_weight_codes_bit_exact(qnn):

@@ -66,7 +66,7 @@ STREAM_CASES = [
     dict(L=2, I=5, H=16, C=0, B=2, T=19),               # no output layer: the top layer's outputs
     dict(L=1, I=40, H=500, C=2000, B=1, T=14, w=0.08),  # one full cluster of 16 output blocks
     dict(L=2, I=40, H=100, C=4500, B=4, T=9, w=0.1),    # 36 output blocks: two gathering rounds
-    dict(L=2, I=40, H=64, C=2000, B=2, T=11, w=0.1, wo=2.0),  # logits spread over several units
+    dict(L=2, I=40, H=64, C=2000, B=2, T=11, w=0.3, wo=1.0),  # logits spread over several units
 ]
 
 

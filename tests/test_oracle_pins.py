@@ -468,6 +468,27 @@ def test_softmax_rows():
     assert np.max(np.abs(res["y"] - e / e.sum(-1, keepdims=True))) <= 1e-6
 
 
+def test_softmax_of_many_nearly_equal_logits():
+    # 8192 classes whose logits lie within +-5e-4 (a wide output layer with small weights): every
+    # posterior equals the fp64 softmax of the same logits to within the pinned E's error (a few
+    # fp32 ulp), which a running fp32 sum of the 8192 nearly equal terms misses by far
+    wl = inputs.LstmWorkload("flat", seed=3, num_layers=1, input_dim=5, hidden=8, proj=0, num_classes=8192,
+                             batch=1, frames=3, w_range=0.5, out_w_range=2e-4)
+    params, x = wl.make()
+    res = _run(wl, params, x)
+    lg = res["logits"].astype(np.float64)
+    assert np.abs(lg).max() < 1e-3
+    e = np.exp(lg - lg.max(-1, keepdims=True))
+    want = e / e.sum(-1, keepdims=True)
+    assert np.max(np.abs(res["y"] / want - 1.0)) <= 5e-7
+    # the same terms summed in a running fp32 sum drift by more than 1e-5 of the posterior
+    ef = np.array([oracle.exp_(float(v)) for v in (res["logits"][0, 0] - res["logits"][0, 0].max())], np.float32)
+    s = np.float32(0.0)
+    for v in ef:
+        s = np.float32(s + v)
+    assert abs(float(s) / ef.astype(np.float64).sum() - 1.0) > 1e-5
+
+
 def test_float_output_layer_variant():
     # 'quant' (Sec. 5): every layer quantized except the softmax layer, which stays float.
     wl = _small(L=2, H=8, C=9, B=1, T=5, mode=2)
