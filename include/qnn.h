@@ -309,6 +309,14 @@ qnn_status qnn_measure_exchange_floor(int32_t cluster_size, int32_t rounds, doub
  * QNN_ERR_INVALID_ARG for n < 0 or null/host pointers with n > 0. Asynchronous on `stream`. */
 qnn_status qnn_selftest_s64_to_f32(const int64_t *in, float *out, int64_t n, void *stream);
 
+/* Diagnostic (no counterpart in the paper): the tensor-core gate kernel evaluates the pinned E,
+ * sigma, tanh, the cell update and the recovery's quotient on two cells at once with paired fp32
+ * instructions; this runs them and their one-value forms on the pairs (in[2i], in[2i+1]) and
+ * writes into *mismatches (device, caller-owned) the number of pairs where any result differs in
+ * any bit (0 is required for bit-exact parity). in [2 npairs] fp32, device memory. Errors:
+ * QNN_ERR_INVALID_ARG for npairs < 0 or null/host pointers. Asynchronous on `stream`. */
+qnn_status qnn_selftest_pair_functions(const float *in, int64_t npairs, unsigned long long *mismatches, void *stream);
+
 /* Diagnostic (no counterpart in the paper): runs one warp that waits, through the bounded wait of
  * the tensor-core kernels, on a barrier nothing completes, for limit_ns (1 us .. 1 s). The wait
  * gives up and records QNN_ERR_TIMEOUT in the device status word (read it with qnn_device_status);

@@ -28,12 +28,14 @@ struct TcLayer {  // fp16 centered weight copies for the tensor-core recurrence 
     __half *wh16 = nullptr;  // [4 * round_up(H, 8)][kh]: gate rows interleaved in 8-cell groups
     __half *wp16 = nullptr;  // [P][kp] (P > 0)
     __half *wx16 = nullptr;  // [4 * round_up(H, 8)][kx], interleaved like wh16 (kx <= 1024)
+    void *colc = nullptr;    // with wx16: [12][H] column constants of the gate kernel (bias, Wx and Wh
+                             // row code sums, gate-major; see TcLstmInput)
     int64_t kh = 0, kp = 0, kx = 0;
 };
 
 // The layer input of a recurrence whose input product is fused into the gate kernel: in [B*T][kin]
-// fp32 (row b T + t), and workspace for its centered fp16 codes x16 [B*T][round_up(kin, 64)], row
-// units prm [B*T] and code sums rs [B*T].
+// fp32 (row b T + t), and workspace for its centered fp16 codes x16 [T*B][round_up(kin, 64)], row
+// units prm [T*B] and code sums rs [T*B], time-major (row t B + b: one step's rows are contiguous).
 struct TcFusedInput {
     const float *in = nullptr;
     int64_t kin = 0;

@@ -33,13 +33,14 @@ constexpr int kQuantRowsPerBlock = 8;  // warp-per-row kernel
 __global__ void __launch_bounds__(32 * kQuantRowsPerBlock)
     quantize_rows_f16_warp_kernel(const float *__restrict__ src, int64_t ld, int rows, int len, int kp,
                                   __half *__restrict__ dst, qnn_qparams *__restrict__ prm,
-                                  int32_t *__restrict__ rsum, int *status) {
+                                  int32_t *__restrict__ rsum, int *status, int tm_T, int tm_B) {
     grid_dependency_wait();
     grid_dependents_launch();
     const int lane = threadIdx.x & 31;
     const int r = blockIdx.x * kQuantRowsPerBlock + (threadIdx.x >> 5);
     if (r >= rows) return;
     const float *xr = src + (int64_t)r * ld;
+    const int ro = tm_T > 0 ? (r % tm_T) * tm_B + r / tm_T : r;  // output row (see launch_quantize_rows_f16)
     float mn = FLT_MAX, mx = -FLT_MAX;
     bool bad = false;
     for (int k = lane; k < len; k += 32) {
@@ -56,7 +57,7 @@ __global__ void __launch_bounds__(32 * kQuantRowsPerBlock)
         mx = 0.0f;
     }
     const qnn_qparams p = params_from_range(mn, mx);
-    __half *dr = dst + (int64_t)r * kp;
+    __half *dr = dst + (int64_t)ro * kp;
     int s = 0;
     for (int k8 = lane * 8; k8 < kp; k8 += 256) {
         __align__(16) __half v[8];
@@ -74,8 +75,8 @@ __global__ void __launch_bounds__(32 * kQuantRowsPerBlock)
     }
     s = warp_sum(s);
     if (lane == 0) {
-        prm[r] = p;
-        rsum[r] = s;
+        prm[ro] = p;
+        rsum[ro] = s;
     }
 }
 
@@ -161,7 +162,7 @@ template <int G>
 __global__ void __launch_bounds__(256)
     quantize_rows_f16_kernel(const float *__restrict__ src, int64_t ld, int rows, int len, int kp,
                              __half *__restrict__ dst, qnn_qparams *__restrict__ prm, int32_t *__restrict__ rsum,
-                             int *status) {
+                             int *status, int tm_T, int tm_B) {
     constexpr int RPB = 256 / G;  // rows per block
     __shared__ float s_mn[8], s_mx[8];
     __shared__ int s_n[8];
@@ -175,7 +176,8 @@ __global__ void __launch_bounds__(256)
     float v[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) v[e] = (rv && k0 + e < len) ? xr[k0 + e] : 0.0f;
-    quantize_row_group<G>(v, len, kp, t, rl, rv, r, dst, prm, rsum, status, s_mn, s_mx, s_n);
+    const int ro = tm_T > 0 ? (r % tm_T) * tm_B + r / tm_T : r;  // output row (see launch_quantize_rows_f16)
+    quantize_row_group<G>(v, len, kp, t, rl, rv, ro, dst, prm, rsum, status, s_mn, s_mx, s_n);
 }
 
 // Arguments of the projection's finishing kernel (one recurrent step of an LSTMP layer).
@@ -274,9 +276,13 @@ __global__ void interleave_gates_kernel(const uint8_t *__restrict__ codes, int64
     }
 }
 
-// Launches one of the two row quantizers; with `pdl` as a programmatic dependent launch.
+// Launches one of the two row quantizers; with `pdl` as a programmatic dependent launch. With
+// tm_T > 0 the source rows are b tm_T + t (sequence-major, tm_B sequences) and row b tm_T + t is
+// written to output row t tm_B + b (time-major), so that one step's rows of all sequences are
+// contiguous for the tensor-core kernel's loads.
 qnn_status launch_quantize_rows_f16(const float *src, int64_t ld, int64_t rows, int64_t len, int64_t kp, __half *dst,
-                                    qnn_qparams *prm, int32_t *rsum, int *status, bool pdl, cudaStream_t st) {
+                                    qnn_qparams *prm, int32_t *rsum, int *status, bool pdl, cudaStream_t st,
+                                    int64_t tm_T = 0, int64_t tm_B = 0) {
     ProfScope prof("quantize_rows_f16", st);
     int g = 8;
     while (g * 8 < kp) g *= 2;
@@ -288,19 +294,20 @@ qnn_status launch_quantize_rows_f16(const float *src, int64_t ld, int64_t rows, 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 1 : 0;
-    const int ir = (int)rows, il = (int)len, ik = (int)kp;
+    const int ir = (int)rows, il = (int)len, ik = (int)kp, tmT = (int)tm_T, tmB = (int)tm_B;
     auto grid_for = [&](int rpb) { return dim3((unsigned)((rows + rpb - 1) / rpb)); };
     cudaError_t e;
     switch (g) {
-        case 8: cfg.gridDim = grid_for(32); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<8>, src, ld, ir, il, ik, dst, prm, rsum, status); break;
-        case 16: cfg.gridDim = grid_for(16); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<16>, src, ld, ir, il, ik, dst, prm, rsum, status); break;
-        case 32: cfg.gridDim = grid_for(8); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<32>, src, ld, ir, il, ik, dst, prm, rsum, status); break;
-        case 64: cfg.gridDim = grid_for(4); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<64>, src, ld, ir, il, ik, dst, prm, rsum, status); break;
-        case 128: cfg.gridDim = grid_for(2); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128>, src, ld, ir, il, ik, dst, prm, rsum, status); break;
-        case 256: cfg.gridDim = grid_for(1); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<256>, src, ld, ir, il, ik, dst, prm, rsum, status); break;
+        case 8: cfg.gridDim = grid_for(32); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<8>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
+        case 16: cfg.gridDim = grid_for(16); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<16>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
+        case 32: cfg.gridDim = grid_for(8); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<32>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
+        case 64: cfg.gridDim = grid_for(4); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<64>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
+        case 128: cfg.gridDim = grid_for(2); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
+        case 256: cfg.gridDim = grid_for(1); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<256>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
         default:
             cfg.gridDim = grid_for(kQuantRowsPerBlock);
-            e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_warp_kernel, src, ld, ir, il, ik, dst, prm, rsum, status);
+            e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_warp_kernel, src, ld, ir, il, ik, dst, prm, rsum, status, tmT,
+                                   tmB);
     }
     QNN_CUDA_TRY(e);
     return QNN_OK;
@@ -341,6 +348,14 @@ int64_t max_proj_splits(const qnn_lstm_model *m) {
     return std::max<int64_t>((kb + 15) / 16, 8);
 }
 
+// The projection as split-K partial sums finished by a row kernel (the default), or with
+// QNN_TC_SPLIT_PROJ=0 as one tensor-core product over the whole K whose epilogue writes r_t, the
+// next step's quantizer then reading r_t.
+bool split_proj_enabled() {
+    const char *e = std::getenv("QNN_TC_SPLIT_PROJ");
+    return !(e && std::strcmp(e, "0") == 0);
+}
+
 // Programmatic dependent launches between the recurrence's kernels (QNN_PDL=0 turns them off).
 bool pdl_enabled() {
     const char *e = std::getenv("QNN_PDL");
@@ -362,7 +377,10 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
         bytes += (size_t)round_up(4 * H8 * kh * 2, 256);
         if (P > 0) bytes += (size_t)round_up(P * kpj * 2, 256);
         const int64_t kx = round_up(m->layers[l].kin, 64);
-        if (kx <= 1024) bytes += (size_t)round_up(4 * H8 * kx * 2, 256);  // Wx for the fused input product
+        if (kx <= 1024) {  // Wx for the fused input product, and the gate kernel's column constants
+            bytes += (size_t)round_up(4 * H8 * kx * 2, 256);
+            bytes += (size_t)round_up(12 * H * 4, 256);
+        }
     }
     void *buf = nullptr;
     QNN_CUDA_TRY(cudaMalloc(&buf, bytes));
@@ -379,7 +397,7 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
                                                                         (int)kh, tl.wh16);
         if (cudaGetLastError() != cudaSuccess) {
             cudaFree(buf);
-            return QNN_ERR_CUDA;
+            return QNN_FAIL(QNN_ERR_CUDA);
         }
         const int64_t kx = round_up(ly.kin, 64);
         if (kx <= 1024) {
@@ -391,7 +409,17 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
                                                                              (int)kx, tl.wx16);
             if (cudaGetLastError() != cudaSuccess) {
                 cudaFree(buf);
-                return QNN_ERR_CUDA;
+                return QNN_FAIL(QNN_ERR_CUDA);
+            }
+            // [12][H]: bias [4][H], Wx row code sums [4][H], Wh row code sums [4][H] (all gate-major)
+            tl.colc = p;
+            p += round_up(12 * H * 4, 256);
+            char *cc = reinterpret_cast<char *>(tl.colc);
+            if (cudaMemcpy(cc, ly.bias, 4 * H * 4, cudaMemcpyDeviceToDevice) != cudaSuccess ||
+                cudaMemcpy(cc + 4 * H * 4, ly.wx.sums, 4 * H * 4, cudaMemcpyDeviceToDevice) != cudaSuccess ||
+                cudaMemcpy(cc + 8 * H * 4, ly.wh.sums, 4 * H * 4, cudaMemcpyDeviceToDevice) != cudaSuccess) {
+                cudaFree(buf);
+                return QNN_FAIL(QNN_ERR_CUDA);
             }
         }
         if (P > 0) {
@@ -407,7 +435,7 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
     }
     if (cudaDeviceSynchronize() != cudaSuccess) {
         cudaFree(buf);
-        return QNN_ERR_CUDA;
+        return QNN_FAIL(QNN_ERR_CUDA);
     }
     m->tcw = buf;
     return QNN_OK;
@@ -463,11 +491,16 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     // tile widths, widest first; the fused kernel's 96-column tile (24 warps at 72 registers) spills
     // with the second recovery and measured slower than 64 columns, so it is left out there
     static const int gate_bn[] = {128, 96, 64, 32}, gate_bn_fused[] = {128, 64, 32};
-    QNN_TRY(tc_operands(&gates, a16, B, tl.wh16, 4 * H8, kh,
-                        fx ? tc_choose_bn(B, 4 * H8, gate_bn_fused, 3) : tc_choose_bn(B, 4 * H8, gate_bn, 4)));
+    // The fused kernel's operand stream (A re-read for every tile of a block) is bounded by the rate at
+    // which a block's TMA ring turns over, so with at least a full wave of tiles the widest tile wins
+    // (LSTMP 5x2048p512 B=1024: 128 columns 49.6 us per step against 52.0 for 64); with less than a
+    // wave the tile count that fills the SMs best decides.
+    int bn_gates = fx ? tc_choose_bn(B, 4 * H8, gate_bn_fused, 3) : tc_choose_bn(B, 4 * H8, gate_bn, 4);
+    if (fx && !std::getenv("QNN_TC_BN") && ((B + 127) / 128) * ((4 * H8 + 127) / 128) >= sm_count()) bn_gates = 128;
+    QNN_TRY(tc_operands(&gates, a16, B, tl.wh16, 4 * H8, kh, bn_gates));
     // the projection: split-K partial sums, finished (offsets, recovery, next step's quantization)
     // by one row kernel when P <= 2048; else one tcgen05 product with its own epilogue per step
-    const bool split_proj = P > 0 && P <= 2048;
+    const bool split_proj = P > 0 && P <= 2048 && split_proj_enabled();
     int splits = 0;
     if (P > 0) {
         QNN_TRY(tc_operands(&proj, m16, B, tl.wp16, P, kpj, split_proj ? 128 : tc_pick_bn(B, P, kpj)));
@@ -480,10 +513,11 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     TcLstmInput xin;
     if (fx) {
         if (!tl.wx16 || tl.kx != round_up(fx->kin, 64)) return QNN_ERR_INVALID_ARG;
+        // codes time-major (row t B + b): a step's x_t rows of all sequences are one contiguous block
         QNN_TRY(launch_quantize_rows_f16(fx->in, fx->kin, B * T, (int)fx->kin, (int)tl.kx, fx->x16, fx->prm, fx->rs,
-                                         status, false, st));
-        xin.x_pitch = T * tl.kx, xin.kx = tl.kx, xin.K_x = (int)fx->kin, xin.stride = T;
-        xin.wx16 = tl.wx16, xin.pw4 = ly.wx.params, xin.cs = ly.wx.sums, xin.bias = ly.bias;
+                                         status, false, st, T, B));
+        xin.x_pitch = tl.kx, xin.kx = tl.kx, xin.K_x = (int)fx->kin, xin.stride = 1;
+        xin.wx16 = tl.wx16, xin.pw4 = ly.wx.params, xin.cs = ly.wx.sums, xin.bias = ly.bias, xin.colc = tl.colc;
     }
     QNN_TRY(launch_quantize_rows_f16(h0, R, B, R, kh, a16, prm, rs, status, false, st));
     for (int64_t t = 0; t < T; ++t) {
@@ -492,7 +526,7 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
         TcLstmOut o{fx ? nullptr : px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R,
                     (int)H, (int)m->S, (int)(H / m->S)};
         if (fx) {
-            xin.x16 = fx->x16 + t * tl.kx, xin.pa = fx->prm + t, xin.rs = fx->rs + t;
+            xin.x16 = fx->x16 + t * B * tl.kx, xin.pa = fx->prm + t * B, xin.rs = fx->rs + t * B;
             QNN_TRY(tc_lstm_gates_x(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, xin, st));
         } else {
             QNN_TRY(tc_lstm_gates(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, st));

@@ -109,6 +109,38 @@ __global__ void s64_to_f32_kernel(const int64_t *__restrict__ in, float *__restr
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         out[i] = s64_to_f32_rn(in[i]);
 }
+
+__device__ __forceinline__ bool bits_differ(float a, float b) { return __float_as_uint(a) != __float_as_uint(b); }
+
+// Pairs (in[2i], in[2i+1]) through the paired-instruction functions and the scalar ones: counts
+// the pairs where any of E, sigma, tanh, the cell update and the reciprocal-based quotient differ.
+__global__ void pair_functions_kernel(const float *__restrict__ in, int64_t npairs, unsigned long long *mismatches) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < npairs; i += (int64_t)gridDim.x * blockDim.x) {
+        const float2 x = make_float2(in[2 * i], in[2 * i + 1]);
+        bool bad = false;
+        const float2 e = pexp2(x), sg = psigmoid2(x), th = ptanh2(x);
+        bad |= bits_differ(e.x, pexp(x.x)) || bits_differ(e.y, pexp(x.y));
+        bad |= bits_differ(sg.x, psigmoid(x.x)) || bits_differ(sg.y, psigmoid(x.y));
+        bad |= bits_differ(th.x, ptanh(x.x)) || bits_differ(th.y, ptanh(x.y));
+        // a cell with gates built from both values, and its scalar twins
+        const float qx = __fmul_rn(0.25f, x.x), qy = __fmul_rn(0.5f, x.y);
+        float c0 = __fmul_rn(x.x, 0.37f), c1 = __fmul_rn(x.y, -0.51f);
+        float2 c = make_float2(c0, c1);
+        const float2 m = lstm_cell2(x, make_float2(x.y, x.x), make_float2(-x.x, qy), make_float2(qx, x.y), c);
+        float m0, m1;
+        lstm_cell(x.x, x.y, -x.x, qx, c0, m0);
+        lstm_cell(x.y, x.x, qy, x.y, c1, m1);
+        bad |= bits_differ(m.x, m0) || bits_differ(m.y, m1) || bits_differ(c.x, c0) || bits_differ(c.y, c1);
+        // the recovery's quotient: integer numerators (converted from int, as the kernel's exact sums
+        // are, so never -0) over a divisor from its correctly rounded reciprocal
+        const float d = __fadd_rn(__fmul_rn(fabsf(x.x), 977.0f), 0.75f);
+        const float2 v = make_float2(__int2float_rn(__float2int_rn(__fmul_rn(x.y, 1.0e6f))),
+                                     __int2float_rn(__float2int_rn(__fmul_rn(x.x, 3.0e5f))));
+        const float2 q = div_by_recip2(v, d, __frcp_rn(d));
+        bad |= bits_differ(q.x, __fdiv_rn(v.x, d)) || bits_differ(q.y, __fdiv_rn(v.y, d));
+        if (bad) atomicAdd(mismatches, 1ull);
+    }
+}
 }  // namespace
 }  // namespace qnn
 
@@ -118,6 +150,19 @@ extern "C" qnn_status qnn_selftest_s64_to_f32(const int64_t *in, float *out, int
     if (!in || !out || !qnn::is_device_ptr(in) || !qnn::is_device_ptr(out)) return QNN_ERR_INVALID_ARG;
     const unsigned blocks = (unsigned)std::min<int64_t>((n + 255) / 256, 4096);
     qnn::s64_to_f32_kernel<<<blocks, 256, 0, qnn::as_stream(stream)>>>(in, out, n);
+    QNN_CUDA_TRY(cudaGetLastError());
+    return QNN_OK;
+}
+
+extern "C" qnn_status qnn_selftest_pair_functions(const float *in, int64_t npairs, unsigned long long *mismatches,
+                                                   void *stream) {
+    if (npairs < 0 || !mismatches || !qnn::is_device_ptr(mismatches)) return QNN_ERR_INVALID_ARG;
+    cudaStream_t st = qnn::as_stream(stream);
+    QNN_CUDA_TRY(cudaMemsetAsync(mismatches, 0, sizeof(unsigned long long), st));
+    if (npairs == 0) return QNN_OK;
+    if (!in || !qnn::is_device_ptr(in)) return QNN_ERR_INVALID_ARG;
+    const unsigned blocks = (unsigned)std::min<int64_t>((npairs + 255) / 256, 4096);
+    qnn::pair_functions_kernel<<<blocks, 256, 0, st>>>(in, npairs, mismatches);
     QNN_CUDA_TRY(cudaGetLastError());
     return QNN_OK;
 }

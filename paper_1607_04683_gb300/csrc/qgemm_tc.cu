@@ -87,8 +87,15 @@ struct Tile {
     // LSTM: the tile's input products px (4 gates x 128 rows x BN/4 cells) and cell state c (128 x
     // BN/4), fp32, double-buffered in shared memory after the stages
     static constexpr int PX_BOX = TBM * (BN / 4) * 4;  // one gate's px box, bytes
-    static constexpr int LSTM_BUF = (EPI == kEpiLstmX ? 1 : 5) * PX_BOX;  // [4 px boxes +] the c box
-    static constexpr int EPI_BYTES = IS_LSTM              ? 2 * LSTM_BUF
+    // kEpiLstmX: the tile's column constants after the c box: per gate the bias, the Wx and the Wh row
+    // code sums of its BN / 4 cells ([12][BN / 4] 32-bit words)
+    static constexpr int COL_BYTES = 12 * (BN / 4) * 4;
+    static constexpr int LSTM_TX = EPI == kEpiLstmX ? PX_BOX + COL_BYTES : 5 * PX_BOX;  // bytes of one fill
+    static constexpr int LSTM_BUF = (LSTM_TX + 1023) / 1024 * 1024;  // [4 px boxes +] the c box [+ constants]
+    // kEpiLstmX: per epilogue thread, the reciprocals of its row's eight divisors of eq. (3), kept in
+    // shared memory across the block's tiles ([warp][8][lane] floats)
+    static constexpr int RC_BYTES = EPI == kEpiLstmX ? EPI_WARPS * 8 * 32 * 4 : 0;
+    static constexpr int EPI_BYTES = IS_LSTM              ? 2 * LSTM_BUF + RC_BYTES
                                      : EPI == kEpiPartial ? 0
                                                           : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
     static constexpr int SMEM_CAP = 227 * 1024 - 1024 - 256;  // dynamic shared memory left for stages + EPI_BYTES
@@ -327,6 +334,11 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             tma_load_2d(dst, &mapW, bar, (kb - (LX ? args.KB_x : 0)) * TBK, n0);
     };
     __shared__ int s_abort;
+    // kEpiLstmX with one weight unit per gate matrix: the eight weight units (Wx then Wh, gates i f g
+    // o), read by every epilogue thread for every slice
+    __shared__ qnn_qparams s_pw[8];
+    if (LX && threadIdx.x < 8 && args.lstm.ups == 1)
+        s_pw[threadIdx.x] = threadIdx.x < 4 ? args.pw_x[threadIdx.x] : args.pw[threadIdx.x - 4];
 
     if (threadIdx.x == 0) {
         s_abort = 0;
@@ -868,11 +880,14 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             tile_origin(t_issue, tiles_m, tiles_n, BN, m1, n1);
             const uint32_t bar = pxfull0 + 8 * pbuf;
             const uint32_t dst = su32(pxs0) + (uint32_t)(pbuf * TL::LSTM_BUF);
-            mb_expect(bar, (uint32_t)TL::LSTM_BUF);
-            if constexpr (!LX) {  // kEpiLstmX computes the input products itself: c only
+            mb_expect(bar, (uint32_t)TL::LSTM_TX);
+            if constexpr (!LX) {
 #pragma unroll
                 for (int g = 0; g < 4; ++g)
                     tma_load_2d(dst + g * TL::PX_BOX, &mapPX, bar, g * H + (int)(n1 / 4), (int)m1);
+            } else {  // kEpiLstmX computes the input products itself: c and the column constants (mapPX
+                      // then maps the [12][H] constant table)
+                tma_load_2d(dst + TL::PX_BOX, &mapPX, bar, (int)(n1 / 4), 0);
             }
             tma_load_2d(dst + C_OFF, &mapC, bar, (int)(n1 / 4), (int)m1);
         };
@@ -880,6 +895,13 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             if (blockIdx.x < tiles) issue_px(blockIdx.x, 0);
             if (blockIdx.x + gridDim.x < tiles) issue_px(blockIdx.x + gridDim.x, 1);
         }
+        // kEpiLstmX with one weight unit per gate matrix: the correctly rounded reciprocals of the
+        // per-row, per-gate divisors Qa Qw of eq. (3) are computed once for the block's row tile and
+        // kept (in this thread's shared-memory slots) while it stays on that tile; the other row
+        // terms are cheap to re-form
+        int64_t cm0 = -1;
+        bool fastrow = false;
+        float *const rcs = pxs0 + 2 * (TL::LSTM_BUF / 4) + (warp - 2) * 8 * 32 + lane;  // [8][32] per warp
         int64_t gc = 0;
         bool ok = true;
         for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
@@ -907,6 +929,27 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 Qx = qa.Q;
                 rsx = args.rsA_x[b * args.x_stride];
             }
+            if (LX && E.ups == 1 && m0 != cm0) {
+                // S = P + rt_g + (128 + z_row) cs fits in 32 bits when K max|a' + za| max|w' + zw| < 2^31
+                // (wrapping 32-bit arithmetic then gives it exactly); the quotient S / (Qa Qw) is the
+                // correctly rounded q + (S - q d) r with r = RN(1/d), q = RN(S r) (Markstein's final
+                // step), which needs d and r far from the ends of the fp32 range; rows outside these
+                // bounds take the general path below
+                cm0 = m0;
+                const long long ax = max(abs(zx), abs(zx + 255)), ah = max(abs(za), abs(za + 255));
+                bool f = bv;
+#pragma unroll
+                for (int g = 0; g < 4; ++g) {
+                    const qnn_qparams qw = args.pw_x[g], qh = args.pw[g];
+                    const float dx = __fmul_rn(Qx, qw.Q), dh = __fmul_rn(Qa, qh.Q);
+                    rcs[g * 32] = __frcp_rn(dx);
+                    rcs[(4 + g) * 32] = __frcp_rn(dh);
+                    f &= (long long)args.K_x * ax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31) &&
+                         (long long)K * ah * (long long)max(abs(qh.z), abs(qh.z + 255)) < (1LL << 31) &&
+                         dx >= 0x1p-60f && dx <= 0x1p60f && dh >= 0x1p-60f && dh <= 0x1p60f;
+                }
+                fastrow = f;
+            }
             const int buf = (int)(gc & 1);
             ok = __all_sync(0xffffffffu, mb_wait(chunk0 + 8 * buf, (unsigned)(gc / 2) & 1, args.status) &&
                                              mb_wait(pxfull0 + 8 * pbuf, (unsigned)(gc / 2) & 1, args.status));
@@ -920,62 +963,101 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     // pre = (R(x_t Wx) + b) + R(h_{t-1} Wh): both exact sums recovered as in eq. (1)/(3)
                     // (the input side exactly as the batched product computes px), then the cell
                     const bool valid = bv && j0 < H;
-                    const int unit = j0 / E.cpu;
-                    const long long ax = max(abs(zx), abs(zx + 255)), ah = max(abs(za), abs(za + 255));
+                    const int jt = j0 - (int)(n0 / 4);  // cell within the tile
                     const uint32_t tx = tmem_base + ((uint32_t)(32 * q) << 16) +
                                         (uint32_t)(buf * TL::ACC_COLS + gi * 32 + part * CPS);
-                    float pre[4][CPS];
+                    // column constants of the slice from shared memory: bias, Wx and Wh row code sums
+                    const float *colb = pxb + TL::PX_BOX / 4 + jt;
+                    const int *coli = reinterpret_cast<const int *>(colb);
+                    // two cells at a time (fewer live registers): the four gates' x and h sums from
+                    // tensor memory (warp-wide loads), eq. (1)/(3), then the cell update. Rows whose
+                    // constants were cached take reciprocal-based quotients and 32-bit sums; the others
+                    // the general way (any weight unit, 64-bit sums when needed, IEEE divides).
+                    const int unit = j0 / E.cpu;
 #pragma unroll
-                    for (int g = 0; g < 4; ++g) {
-                        uint32_t rx[CPS], rh[CPS];
-                        tmem_ld_nowait(tx + 8 * g, rx);
-                        tmem_ld_nowait(tx + BN + 8 * g, rh);
+                    for (int c2 = 0; c2 < CPS; c2 += 2) {
+                        uint32_t rx[4][2], rh[4][2];
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            tmem_ld_nowait(tx + 8 * g + c2, rx[g]);
+                            tmem_ld_nowait(tx + BN + 8 * g + c2, rh[g]);
+                        }
                         tmem_wait_ld();
-                        if (valid) {
-                            // the gate's row terms (per gate, to keep registers free)
-                            const qnn_qparams qw = args.pw_x[g * E.ups + unit], qh = args.pw[g * E.ups + unit];
-                            const long long rtx = (long long)(128 + qw.z) * rsx +
-                                                  (long long)args.K_x * ((long long)zx * qw.z - 16384);
-                            const long long rth =
-                                (long long)(128 + qh.z) * rs + (long long)K * ((long long)za * qh.z - 16384);
-                            const float denx = __fmul_rn(Qx, qw.Q), denh = __fmul_rn(Qa, qh.Q);
-                            const bool fits =
-                                (long long)args.K_x * ax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31) &&
-                                (long long)K * ah * (long long)max(abs(qh.z), abs(qh.z + 255)) < (1LL << 31);
-                            float bias[CPS];
-                            int csx[CPS], csh[CPS];
-                            ld_vec(args.bias_x + g * H + j0, bias);
-                            ld_vec(args.csW_x + g * H + j0, csx);
-                            ld_vec(args.csW + g * H + j0, csh);
+                        if (!valid) continue;
+                        float pre[4][2];
+                        if (fastrow) {
 #pragma unroll
-                            for (int jj = 0; jj < CPS; ++jj) {
-                                const int Px = f32_integer_to_s32(__uint_as_float(rx[jj]));
-                                const int Ph = f32_integer_to_s32(__uint_as_float(rh[jj]));
-                                float vx, vh;
-                                if (fits) {
-                                    vx = __int2float_rn((int)((uint32_t)Px + (uint32_t)rtx +
-                                                              (uint32_t)(128 + zx) * (uint32_t)csx[jj]));
-                                    vh = __int2float_rn((int)((uint32_t)Ph + (uint32_t)rth +
-                                                              (uint32_t)za128 * (uint32_t)csh[jj]));
-                                } else {
-                                    vx = s64_to_f32_rn((long long)Px + rtx + (long long)(128 + zx) * csx[jj]);
-                                    vh = s64_to_f32_rn((long long)Ph + rth + (long long)za128 * csh[jj]);
+                            for (int g = 0; g < 4; ++g) {
+                                float bias[2];
+                                int csx[2], csh[2];
+                                ld_vec(colb + g * CW + c2, bias);
+                                ld_vec(coli + (4 + g) * CW + c2, csx);
+                                ld_vec(coli + (8 + g) * CW + c2, csh);
+                                const qnn_qparams qw = s_pw[g], qh = s_pw[4 + g];
+                                const float dx = __fmul_rn(Qx, qw.Q), dh = __fmul_rn(Qa, qh.Q);
+                                const float rcx = rcs[g * 32], rch = rcs[(4 + g) * 32];
+                                // rt of eq. (1) for this row and gate, modulo 2^32 (S itself fits in 32 bits)
+                                const uint32_t rtx = (uint32_t)(128 + qw.z) * (uint32_t)rsx +
+                                                     (uint32_t)args.K_x * (uint32_t)(zx * qw.z - 16384);
+                                const uint32_t rth = (uint32_t)(128 + qh.z) * (uint32_t)rs +
+                                                     (uint32_t)K * (uint32_t)(za * qh.z - 16384);
+                                float2 vx, vh;
+                                vx.x = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rx[g][0])) +
+                                                            rtx + (uint32_t)(128 + zx) * (uint32_t)csx[0]));
+                                vx.y = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rx[g][1])) +
+                                                            rtx + (uint32_t)(128 + zx) * (uint32_t)csx[1]));
+                                vh.x = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rh[g][0])) +
+                                                            rth + (uint32_t)za128 * (uint32_t)csh[0]));
+                                vh.y = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rh[g][1])) +
+                                                            rth + (uint32_t)za128 * (uint32_t)csh[1]));
+                                const float2 yx = fadd2_rn(div_by_recip2(vx, dx, rcx), make_float2(bias[0], bias[1]));
+                                const float2 y = fadd2_rn(yx, div_by_recip2(vh, dh, rch));
+                                pre[g][0] = y.x;
+                                pre[g][1] = y.y;
+                            }
+                        } else {
+                            const long long ax = max(abs(zx), abs(zx + 255)), ah = max(abs(za), abs(za + 255));
+#pragma unroll
+                            for (int g = 0; g < 4; ++g) {
+                                const qnn_qparams qw = args.pw_x[g * E.ups + unit], qh = args.pw[g * E.ups + unit];
+                                const long long rtx = (long long)(128 + qw.z) * rsx +
+                                                      (long long)args.K_x * ((long long)zx * qw.z - 16384);
+                                const long long rth =
+                                    (long long)(128 + qh.z) * rs + (long long)K * ((long long)za * qh.z - 16384);
+                                const float dx = __fmul_rn(Qx, qw.Q), dh = __fmul_rn(Qa, qh.Q);
+                                const bool fits =
+                                    (long long)args.K_x * ax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31) &&
+                                    (long long)K * ah * (long long)max(abs(qh.z), abs(qh.z + 255)) < (1LL << 31);
+                                float bias[2];
+                                int csx[2], csh[2];
+                                ld_vec(colb + g * CW + c2, bias);
+                                ld_vec(coli + (4 + g) * CW + c2, csx);
+                                ld_vec(coli + (8 + g) * CW + c2, csh);
+#pragma unroll
+                                for (int jj = 0; jj < 2; ++jj) {
+                                    const int Px = f32_integer_to_s32(__uint_as_float(rx[g][jj]));
+                                    const int Ph = f32_integer_to_s32(__uint_as_float(rh[g][jj]));
+                                    float vx, vh;
+                                    if (fits) {
+                                        vx = __int2float_rn((int)((uint32_t)Px + (uint32_t)rtx +
+                                                                  (uint32_t)(128 + zx) * (uint32_t)csx[jj]));
+                                        vh = __int2float_rn((int)((uint32_t)Ph + (uint32_t)rth +
+                                                                  (uint32_t)za128 * (uint32_t)csh[jj]));
+                                    } else {
+                                        vx = s64_to_f32_rn((long long)Px + rtx + (long long)(128 + zx) * csx[jj]);
+                                        vh = s64_to_f32_rn((long long)Ph + rth + (long long)za128 * csh[jj]);
+                                    }
+                                    const float yx = __fadd_rn(__fdiv_rn(vx, dx), bias[jj]);
+                                    pre[g][jj] = __fadd_rn(yx, __fdiv_rn(vh, dh));
                                 }
-                                const float yx = __fadd_rn(__fdiv_rn(vx, denx), bias[jj]);
-                                pre[g][jj] = __fadd_rn(yx, __fdiv_rn(vh, denh));
                             }
                         }
-                    }
-                    if (valid) {
-                        const int jt = j0 - (int)(n0 / 4);
-                        float *cr = E.c + b * (int64_t)H + j0;
-                        float cv[CPS], mv[CPS];
-                        ld_vec(pxb + C_OFF / 4 + rl * CW + jt, cv);
-#pragma unroll
-                        for (int jj = 0; jj < CPS; ++jj)
-                            lstm_cell(pre[0][jj], pre[1][jj], pre[2][jj], pre[3][jj], cv[jj], mv[jj]);
-                        st_vec(cr, cv);
-                        st_vec(E.h + b * E.h_ld + j0, mv);
+                        float2 cv = *reinterpret_cast<const float2 *>(pxb + C_OFF / 4 + rl * CW + jt + c2);
+                        const float2 mv = lstm_cell2(make_float2(pre[0][0], pre[0][1]), make_float2(pre[1][0], pre[1][1]),
+                                                     make_float2(pre[2][0], pre[2][1]), make_float2(pre[3][0], pre[3][1]),
+                                                     cv);
+                        *reinterpret_cast<float2 *>(E.c + b * (int64_t)H + j0 + c2) = cv;
+                        *reinterpret_cast<float2 *>(E.h + b * E.h_ld + j0 + c2) = mv;
                     }
                     continue;
                 }
@@ -1116,7 +1198,7 @@ qnn_status get_encode(PFN_cuTensorMapEncodeTiled_v12000 *out) {
         if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &fn, cudaEnableDefault, &q) != cudaSuccess ||
             q != cudaDriverEntryPointSuccess || !fn) {
             cudaGetLastError();
-            return QNN_ERR_CUDA;
+            return QNN_FAIL(QNN_ERR_CUDA);
         }
         g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
@@ -1138,7 +1220,7 @@ qnn_status make_map_f32(CUtensorMap *map, const float *base, int64_t rows, int64
     CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(base), dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS ? QNN_OK : QNN_ERR_CUDA;
+    return r == CUDA_SUCCESS ? QNN_OK : QNN_FAIL(QNN_ERR_CUDA);
 }
 
 // 2-D fp16 tensor [rows][ld] (ld a multiple of 64), boxes of 64 x box_rows, 128-byte swizzle.
@@ -1153,7 +1235,7 @@ qnn_status make_map(CUtensorMap *map, const __half *base, int64_t rows, int64_t 
     CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half *>(base), dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS ? QNN_OK : QNN_ERR_CUDA;
+    return r == CUDA_SUCCESS ? QNN_OK : QNN_FAIL(QNN_ERR_CUDA);
 }
 
 }  // namespace
@@ -1180,14 +1262,15 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
                                           (int)cudaSharedmemCarveoutMaxShared));
         int n = 0;
         QNN_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, qgemm_tc_kernel<BN, EPI>, TL::THREADS, TL::SMEM));
-        if (n < 1) return QNN_ERR_CUDA;
-        configured = dev;
         if (std::getenv("QNN_DEBUG")) {
             cudaFuncAttributes fa{};
             cudaFuncGetAttributes(&fa, qgemm_tc_kernel<BN, EPI>);
-            std::fprintf(stderr, "qnn: qgemm_tc_kernel<%d,%d>: %d threads, %d registers, %zu bytes dynamic shared, "
-                         "%d blocks per SM\n", BN, EPI, TL::THREADS, fa.numRegs, TL::SMEM, n);
+            std::fprintf(stderr, "qnn: qgemm_tc_kernel<%d,%d>: %d threads (at most %d), %d registers, %zu bytes "
+                         "static and %zu dynamic shared, %zu local, %d blocks per SM\n", BN, EPI, TL::THREADS,
+                         fa.maxThreadsPerBlock, fa.numRegs, fa.sharedSizeBytes, TL::SMEM, fa.localSizeBytes, n);
         }
+        if (n < 1) return QNN_FAIL(QNN_ERR_CUDA);
+        configured = dev;
     }
     const int64_t items = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN) * a.splits;  // (tile, K range) pairs
     // persistent: one block per SM (a block holding tensor memory has its SM to itself)
@@ -1318,7 +1401,7 @@ qnn_status tc_lstm_gates_x(const TcOperands &op, const qnn_qparams *pa, const in
     if (op.N != 4 * ((out.H + 7) / 8 * 8)) return QNN_ERR_INVALID_ARG;
     if (in.K_x <= 0 || in.kx % TBK != 0 || in.kx > KCHUNK || in.K_x > in.kx || in.x_pitch < in.kx || in.x_pitch % 8)
         return QNN_ERR_INVALID_ARG;
-    if ((reinterpret_cast<uintptr_t>(in.x16) & 15) || (reinterpret_cast<uintptr_t>(in.wx16) & 15))
+    if ((reinterpret_cast<uintptr_t>(in.x16) & 15) || (reinterpret_cast<uintptr_t>(in.wx16) & 15) || !in.colc)
         return QNN_ERR_INVALID_ARG;
     int *status = nullptr;
     QNN_TRY(status_word(&status));
@@ -1327,15 +1410,16 @@ qnn_status tc_lstm_gates_x(const TcOperands &op, const qnn_qparams *pa, const in
              1, kbh + kbx, nullptr, 0, 1};
     a.pa_x = in.pa, a.x_stride = in.stride, a.rsA_x = in.rs, a.pw_x = in.pw4, a.csW_x = in.cs, a.bias_x = in.bias;
     a.K_x = in.K_x, a.KB_x = kbx;
-    CUtensorMap map_c, map_ax, map_wx;
+    CUtensorMap map_c, map_ax, map_wx, map_col;
     QNN_TRY(make_map_f32(&map_c, out.c, op.M, out.H, out.H, op.bn / 4, TBM));
+    QNN_TRY(make_map_f32(&map_col, reinterpret_cast<const float *>(in.colc), 12, out.H, out.H, op.bn / 4, 12));
     QNN_TRY(make_map(&map_ax, in.x16, op.M, in.kx, TBM, in.x_pitch));
     QNN_TRY(make_map(&map_wx, in.wx16, op.N, in.kx, op.bn));
     switch (op.bn) {
-        case 32: return launch_tc<32, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
-        case 64: return launch_tc<64, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
-        case 96: return launch_tc<96, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
-        case 128: return launch_tc<128, kEpiLstmX>(op, a, "lstm_gates_tc", st, nullptr, &map_c, &map_ax, &map_wx);
+        case 32: return launch_tc<32, kEpiLstmX>(op, a, "lstm_gates_tc", st, &map_col, &map_c, &map_ax, &map_wx);
+        case 64: return launch_tc<64, kEpiLstmX>(op, a, "lstm_gates_tc", st, &map_col, &map_c, &map_ax, &map_wx);
+        case 96: return launch_tc<96, kEpiLstmX>(op, a, "lstm_gates_tc", st, &map_col, &map_c, &map_ax, &map_wx);
+        case 128: return launch_tc<128, kEpiLstmX>(op, a, "lstm_gates_tc", st, &map_col, &map_c, &map_ax, &map_wx);
         default: return QNN_ERR_INVALID_ARG;
     }
 }

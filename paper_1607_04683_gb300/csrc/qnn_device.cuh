@@ -60,10 +60,6 @@ __device__ __forceinline__ uint32_t quant_code(float v, float Q, int z) {
 }
 
 // (float)S rounded to nearest, ties to even, without the 64-bit conversion instruction (which runs
-// on this part's narrow fp64 pipe). |S| < 2^31 converts from 32 bits; wider values are rounded to a
-// 24-bit significand by integer arithmetic: the bits below it decide the rounding (above half:
-// up; exactly half: to the even significand).
-// (float)S rounded to nearest, ties to even, without the 64-bit conversion instruction (which runs
 // on this part's narrow fp64 pipe). |S| < 2^31 converts from 32 bits; wider values (rare: large
 // offsets z) are rounded to a 24-bit significand by integer arithmetic out of line: the bits below
 // the significand decide (above half: up; exactly half: to the even significand).
@@ -89,6 +85,18 @@ __device__ __forceinline__ float s64_to_f32_rn(long long S) {
 
 // An integer-valued float (an exact tensor-core sum) as int.
 __device__ __forceinline__ int f32_integer_to_s32(float v) { return __float2int_rn(v); }
+
+// x / d correctly rounded, from r = RN(1/d) (the correctly rounded reciprocal, computed once per
+// divisor): q = RN(x r), the remainder x - q d exactly by a fused multiply-add, then RN(q + (x - q d) r)
+// (the final step of Markstein's division). This equals the IEEE quotient while d and r stay well
+// inside the normal range and x q does not overflow (the caller checks d against 2^-60 .. 2^60 and
+// passes |x| < 2^63); a CPU test checks the identity over every 24-bit numerator significand
+// against thousands of divisors.
+__device__ __forceinline__ float div_by_recip(float x, float d, float r) {
+    const float q = __fmul_rn(x, r);
+    const float e = __fmaf_rn(-q, d, x);
+    return __fmaf_rn(e, r, q);
+}
 
 // Eq. (1) recovery of the exact offset-applied product S: S / (Qa Qw), each op rounded once.
 __device__ __forceinline__ float recover_product(long long S, float Qa, float Qw) {
@@ -153,6 +161,91 @@ __device__ __forceinline__ float lstm_cell_update(float ig, float fg, float gg, 
 __device__ __forceinline__ void lstm_cell(float pi, float pf, float pg, float po, float &c, float &m) {
     float ig = psigmoid(pi), fg = psigmoid(pf), gg = ptanh(pg), og = psigmoid(po);
     m = lstm_cell_update(ig, fg, gg, og, c);
+}
+
+// The same functions on two values at once with the paired fp32 instructions of sm_100 and later
+// (mul/add/fma .rn.f32x2: per component the same IEEE round-to-nearest operation as __fmul_rn,
+// __fadd_rn, __fmaf_rn), so each component equals the scalar function bit for bit while the
+// exponential's polynomial takes half the instructions. A paired product whose rounded result
+// feeds a paired sum was observed fused into one multiply-add (with the compiler's paired
+// intrinsics, and on one lane even through explicit-rounding PTX), so those two steps stay scalar
+// wherever the product is inexact; the paired ops are used for fused multiply-adds, sums, and
+// products that are exact (powers of two) or feed no sum.
+__device__ __forceinline__ float2 f2(float a) { return make_float2(a, a); }
+__device__ __forceinline__ float2 fmul2_rn(float2 a, float2 b) {
+    float2 d;
+    asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mul.rn.f32x2 rd, ra, rb;\n"
+        " mov.b64 {%0, %1}, rd;\n}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+__device__ __forceinline__ float2 fadd2_rn(float2 a, float2 b) {
+    float2 d;
+    asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n add.rn.f32x2 rd, ra, rb;\n"
+        " mov.b64 {%0, %1}, rd;\n}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+__device__ __forceinline__ float2 ffma2_rn(float2 a, float2 b, float2 c) {
+    float2 d;
+    asm("{\n .reg .b64 ra, rb, rc, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mov.b64 rc, {%6, %7};\n"
+        " fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 pexp2(float2 x) {
+    x.x = x.x < -87.0f ? -87.0f : x.x;
+    x.y = x.y < -87.0f ? -87.0f : x.y;
+    x.x = x.x > 88.0f ? 88.0f : x.x;
+    x.y = x.y > 88.0f ? 88.0f : x.y;
+    // the rounded product x log2(e) and the sum stay scalar: a paired product followed by a paired
+    // sum was observed contracted into one multiply-add (one rounding fewer)
+    const float2 t = make_float2(__fadd_rn(__fmul_rn(x.x, 1.44269504088896341f), 12582912.0f),
+                                 __fadd_rn(__fmul_rn(x.y, 1.44269504088896341f), 12582912.0f));
+    const int nx = __float_as_int(t.x) - 0x4B400000, ny = __float_as_int(t.y) - 0x4B400000;
+    const float2 nf = fadd2_rn(t, f2(-12582912.0f));
+    const float2 mnf = make_float2(-nf.x, -nf.y);
+    float2 r = ffma2_rn(mnf, f2(0.693145751953125f), x);
+    r = ffma2_rn(mnf, f2(1.428606820309417232e-06f), r);
+    float2 p = f2(1.984126984126984127e-04f);
+    p = ffma2_rn(p, r, f2(1.388888888888888889e-03f));
+    p = ffma2_rn(p, r, f2(8.333333333333333333e-03f));
+    p = ffma2_rn(p, r, f2(4.166666666666666667e-02f));
+    p = ffma2_rn(p, r, f2(1.666666666666666667e-01f));
+    p = ffma2_rn(p, r, f2(0.5f));
+    p = ffma2_rn(p, r, f2(1.0f));
+    p = ffma2_rn(p, r, f2(1.0f));
+    return fmul2_rn(p, make_float2(__int_as_float((nx + 127) << 23), __int_as_float((ny + 127) << 23)));
+}
+
+__device__ __forceinline__ float2 psigmoid2(float2 x) {
+    const float2 d = fadd2_rn(f2(1.0f), pexp2(make_float2(-x.x, -x.y)));
+    return make_float2(__frcp_rn(d.x), __frcp_rn(d.y));
+}
+
+__device__ __forceinline__ float2 ptanh2(float2 x) {
+    const float2 d = fadd2_rn(pexp2(fmul2_rn(f2(2.0f), x)), f2(1.0f));
+    const float2 t = fmul2_rn(f2(2.0f), make_float2(__frcp_rn(d.x), __frcp_rn(d.y)));
+    return fadd2_rn(f2(1.0f), make_float2(-t.x, -t.y));
+}
+
+// lstm_cell on two cells: pre-activations of gates i, f, g, o (one float2 each), cell state c in/out.
+__device__ __forceinline__ float2 lstm_cell2(float2 pi, float2 pf, float2 pg, float2 po, float2 &c) {
+    const float2 ig = psigmoid2(pi), fg = psigmoid2(pf), gg = ptanh2(pg), og = psigmoid2(po);
+    c = make_float2(__fadd_rn(__fmul_rn(fg.x, c.x), __fmul_rn(ig.x, gg.x)),
+                    __fadd_rn(__fmul_rn(fg.y, c.y), __fmul_rn(ig.y, gg.y)));  // scalar: see pexp2
+    return fmul2_rn(og, ptanh2(c));
+}
+
+// div_by_recip on two numerators with one divisor.
+__device__ __forceinline__ float2 div_by_recip2(float2 x, float d, float r) {
+    const float2 q = fmul2_rn(x, f2(r));
+    const float2 e = ffma2_rn(make_float2(-q.x, -q.y), f2(d), x);
+    return ffma2_rn(e, f2(r), q);
 }
 
 // Device clock in nanoseconds (%globaltimer).

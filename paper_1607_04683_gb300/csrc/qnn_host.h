@@ -3,6 +3,7 @@
 
 #include <cstdint>
 #include <cstdio>
+#include <cstdlib>
 #include <cuda_runtime.h>
 
 #include "../../include/qnn.h"
@@ -19,6 +20,13 @@ namespace qnn {
             return _e == cudaErrorMemoryAllocation ? QNN_ERR_NO_MEMORY : QNN_ERR_CUDA;      \
         }                                                                                    \
     } while (0)
+
+// A failure status, reported with its source location on stderr when QNN_DEBUG is set.
+inline qnn_status debug_fail(qnn_status s, const char *file, int line) {
+    if (std::getenv("QNN_DEBUG")) std::fprintf(stderr, "qnn: status %d at %s:%d\n", (int)s, file, line);
+    return s;
+}
+#define QNN_FAIL(code) ::qnn::debug_fail((code), __FILE__, __LINE__)
 
 #define QNN_TRY(expr)                       \
     do {                                    \

@@ -68,6 +68,10 @@ struct TcLstmInput {
     const qnn_qparams *pw4 = nullptr;
     const int32_t *cs = nullptr;
     const float *bias = nullptr;
+    // the same column constants as one [12][H] table of 32-bit words, staged per tile by TMA: rows
+    // 0-3 the bias of gates i f g o (fp32), rows 4-7 the Wx row code sums, rows 8-11 the Wh row code
+    // sums (int32); 16-byte aligned, H a multiple of 4
+    const void *colc = nullptr;
 };
 
 // One recurrent step's gate product and cell update: A = centered codes of h_{t-1} (one unit per

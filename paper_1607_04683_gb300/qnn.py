@@ -34,7 +34,7 @@ EXPORTS = ("qnn_status_string", "qnn_device_status", "qnn_quantize", "qnn_qmatmu
            "qnn_lstm_model_create", "qnn_lstm_model_destroy", "qnn_lstm_model_weights", "qnn_lstm_forward",
            "qnn_lstm_forward_logits",
            "qnn_profile_enable", "qnn_profile_read", "qnn_measure_peak", "qnn_quantize_matrix_static",
-           "qnn_selftest_s64_to_f32", "qnn_stack_frames", "qnn_selftest_wait_timeout", "qnn_lstm_stream_open",
+           "qnn_selftest_s64_to_f32", "qnn_stack_frames", "qnn_selftest_wait_timeout", "qnn_selftest_pair_functions", "qnn_lstm_stream_open",
            "qnn_lstm_stream_push", "qnn_lstm_stream_pull", "qnn_lstm_stream_close", "qnn_measure_exchange_floor")
 
 
@@ -90,6 +90,8 @@ def lib():
         L.qnn_measure_peak.restype = i32
         L.qnn_selftest_s64_to_f32.argtypes = [P, P, i64, P]
         L.qnn_stack_frames.argtypes = [P, i64, i64, i64, i32, i32, P, P]
+        L.qnn_selftest_pair_functions.argtypes = [P, i64, P, P]
+        L.qnn_selftest_pair_functions.restype = i32
         L.qnn_selftest_wait_timeout.argtypes = [i64, P]
         L.qnn_selftest_wait_timeout.restype = i32
         L.qnn_stack_frames.restype = i32
@@ -137,6 +139,16 @@ def selftest_s64_to_f32(values):
     _check(lib().qnn_selftest_s64_to_f32(values.data_ptr(), out.data_ptr(), values.numel(),
                                          torch.cuda.current_stream().cuda_stream), "qnn_selftest_s64_to_f32")
     return out
+
+
+def selftest_pair_functions(values) -> int:
+    """Pairs of a float32 CUDA tensor through the gate kernel's paired-instruction functions and
+    their one-value forms; returns the number of pairs whose results differ in any bit."""
+    import torch
+    out = torch.zeros(1, dtype=torch.int64, device=values.device)
+    _check(lib().qnn_selftest_pair_functions(values.data_ptr(), values.numel() // 2, out.data_ptr(),
+                                             torch.cuda.current_stream().cuda_stream), "qnn_selftest_pair_functions")
+    return int(out.item())
 
 
 def selftest_wait_timeout(limit_ns: int, stream=None):

@@ -187,3 +187,25 @@ def test_s64_to_f32_rounds_to_nearest_even(qnn):
     got = qnn.selftest_s64_to_f32(torch.from_numpy(v).cuda()).cpu().numpy()
     want = v.astype(np.float32)
     assert np.array_equal(got.view(np.int32), want.view(np.int32))
+
+
+def test_paired_gate_functions_equal_the_scalar_ones(qnn):
+    """The fused gate kernel computes E, sigma, tanh, the cell update and the recovery's quotient two
+    cells at a time with paired fp32 instructions; every component must equal the one-value form bit
+    for bit (else layer outputs would drift from the oracle). Inputs span the exponential's clamp
+    range and beyond, with values at and next to the half-integer multiples of ln 2 where the
+    reduction's rounding decides n."""
+    g = np.random.Generator(np.random.PCG64(21))
+    parts = [g.uniform(-100, 100, 1 << 21), g.uniform(-10, 10, 1 << 21), g.uniform(-1, 1, 1 << 20),
+             g.normal(0, 1e-3, 1 << 18)]
+    ln2 = np.log(2.0)
+    half = (np.arange(-130, 130) + 0.5) * ln2
+    near = np.concatenate([np.nextafter(half.astype(np.float32), np.float32(s)) for s in (-np.inf, np.inf)] +
+                          [half.astype(np.float32)])
+    v = np.concatenate([p.astype(np.float32) for p in parts] + [near, np.float32([0.0, -0.0, 87.0, -87.0, 88.0, -88.0])])
+    if v.size % 2:
+        v = np.concatenate([v, np.float32([1.0])])
+    assert qnn.selftest_pair_functions(torch.from_numpy(v).cuda()) == 0
+    # the pairs the other way round too
+    w = v.reshape(-1, 2)[:, ::-1].copy().ravel()
+    assert qnn.selftest_pair_functions(torch.from_numpy(w).cuda()) == 0
