@@ -415,7 +415,10 @@ int orc_lstm_forward(const orc_lstm_desc *d, const float *params, const float *x
         bo = q;
     }
 
+    /* the widest row any step quantizes: the network input, the cell outputs m_t or the recurrent
+       input r_t (R = P can exceed H) */
     int64_t maxK = I > H ? I : H;
+    if (R > maxK) maxK = R;
     float *hprev = (float *)calloc((size_t)(L * R), sizeof(float));
     float *cprev = (float *)calloc((size_t)(L * H), sizeof(float));
     float *layer_in = (float *)calloc((size_t)maxK, sizeof(float));

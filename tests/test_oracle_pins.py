@@ -384,8 +384,11 @@ def test_lstm_reduces_to_textbook_lstm_on_recovered_operands(cfg):
     _textbook_check(wl, params, x, res, tol_h=2e-6)
 
 
-def test_lstmp_reduces_to_textbook_on_recovered_operands():
-    wl = _small(L=2, I=6, H=10, P=4, C=7, B=2, T=5)
+# a projection narrower than the cells, and one wider than both the cells and the input (the
+# recurrent input is then the widest row a step quantizes)
+@pytest.mark.parametrize("cfg", [dict(L=2, I=6, H=10, P=4, C=7, B=2, T=5), dict(L=2, I=5, H=6, P=20, C=7, B=2, T=5)])
+def test_lstmp_reduces_to_textbook_on_recovered_operands(cfg):
+    wl = _small(**cfg)
     params, x = wl.make()
     res = _run(wl, params, x)
     # the projection re-quantizes m, computed here in fp64: a code may flip on an fp32 tie
