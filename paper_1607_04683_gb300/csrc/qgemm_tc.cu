@@ -28,6 +28,7 @@
 #include "qnn_device.cuh"
 #include "qnn_host.h"
 #include "tc_gemm.h"
+#include "tc_ptx.cuh"
 
 namespace qnn {
 namespace {
@@ -92,9 +93,9 @@ struct Tile {
     static constexpr int COL_BYTES = 12 * (BN / 4) * 4;
     static constexpr int LSTM_TX = EPI == kEpiLstmX ? PX_BOX + COL_BYTES : 5 * PX_BOX;  // bytes of one fill
     static constexpr int LSTM_BUF = (LSTM_TX + 1023) / 1024 * 1024;  // [4 px boxes +] the c box [+ constants]
-    // kEpiLstmX: per epilogue thread, the reciprocals of its row's eight divisors of eq. (3), kept in
-    // shared memory across the block's tiles ([warp][8][lane] floats)
-    static constexpr int RC_BYTES = EPI == kEpiLstmX ? EPI_WARPS * 8 * 32 * 4 : 0;
+    // kEpiLstmX: per epilogue thread, the reciprocals of its row's eight divisors of eq. (3) and its
+    // eight row terms rt of eq. (1), kept in shared memory across the block's tiles ([warp][16][lane] floats)
+    static constexpr int RC_BYTES = EPI == kEpiLstmX ? EPI_WARPS * 16 * 32 * 4 : 0;
     static constexpr int EPI_BYTES = IS_LSTM              ? 2 * LSTM_BUF + RC_BYTES
                                      : EPI == kEpiPartial ? 0
                                                           : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
@@ -150,77 +151,10 @@ struct TcArgs {
     int K_x, KB_x;
 };
 
-__device__ __forceinline__ uint32_t su32(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
 __device__ __forceinline__ unsigned long long gtime() { return global_timer_ns(); }
-__device__ __forceinline__ void mb_init(uint32_t b, unsigned n) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(b), "r"(n) : "memory");
-}
-__device__ __forceinline__ void mb_expect(uint32_t b, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(b), "r"(bytes) : "memory");
-}
 // Bounded wait; false (and QNN_ERR_TIMEOUT recorded) if the phase did not complete in time.
 __device__ __forceinline__ bool mb_wait(uint32_t b, unsigned parity, int *status) {
     return mbar_wait_bounded(b, parity, status, TC_WAIT_NS);
-}
-
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
-            dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
-        : "memory");
-}
-
-// Shared-memory matrix descriptor of a K-major tile with 128-byte swizzle: rows of 128 bytes,
-// 8-row groups 1024 bytes apart (stride byte offset), tcgen05 descriptor version 1.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
-    uint64_t d = 0;
-    d |= (uint64_t)((addr & 0x3FFFF) >> 4);        // start address
-    d |= (uint64_t)1 << 16;                          // leading byte offset (unused with this swizzle)
-    d |= (uint64_t)(1024 >> 4) << 32;                // stride byte offset
-    d |= (uint64_t)1 << 46;                          // version
-    d |= (uint64_t)2 << 61;                          // 128-byte swizzle
-    return d;
-}
-
-template <uint32_t IDESC>
-__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate)
-        : "memory");
-}
-__device__ __forceinline__ void mma_commit(uint32_t bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-
-// 32 consecutive fp32 columns of this warp's 32 tensor-memory lanes (one row per lane).
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
-        "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
-          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
-          "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-    tmem_wait_ld();
-}
-// 16 consecutive fp32 columns.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
-          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-    tmem_wait_ld();
-}
-// 2 consecutive fp32 columns, without the wait.
-__device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[2]) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(taddr));
 }
 // Vector loads and stores of 2 or 4 consecutive (8- or 16-byte aligned) values.
 __device__ __forceinline__ void ld_vec(const float *p, float (&v)[4]) {
@@ -244,13 +178,6 @@ __device__ __forceinline__ void st_vec(float *p, const float (&v)[4]) {
 }
 __device__ __forceinline__ void st_vec(float *p, const float (&v)[2]) {
     *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
-}
-
-// 4 consecutive fp32 columns, without the wait (the caller waits once for several loads).
-__device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[4]) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-                 : "r"(taddr));
 }
 
 // Tile order: groups of kGroupM row tiles, columns outer within a group, so that the tiles one
@@ -901,7 +828,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         // terms are cheap to re-form
         int64_t cm0 = -1;
         bool fastrow = false;
-        float *const rcs = pxs0 + 2 * (TL::LSTM_BUF / 4) + (warp - 2) * 8 * 32 + lane;  // [8][32] per warp
+        float *const rcs = pxs0 + 2 * (TL::LSTM_BUF / 4) + (warp - 2) * 16 * 32 + lane;  // [16][32] per warp
         int64_t gc = 0;
         bool ok = true;
         for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
@@ -921,6 +848,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 rs = args.rsA[b];
             }
             const int za128 = 128 + za;
+            const float za128f = (float)za128;
             int zx = 0, rsx = 0;  // kEpiLstmX: the unit and code sum of row b of x_t
             float Qx = 1.0f;
             if (LX && bv) {
@@ -929,12 +857,16 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 Qx = qa.Q;
                 rsx = args.rsA_x[b * args.x_stride];
             }
+            const float zx128f = (float)(128 + zx);
             if (LX && E.ups == 1 && m0 != cm0) {
-                // S = P + rt_g + (128 + z_row) cs fits in 32 bits when K max|a' + za| max|w' + zw| < 2^31
-                // (wrapping 32-bit arithmetic then gives it exactly); the quotient S / (Qa Qw) is the
-                // correctly rounded q + (S - q d) r with r = RN(1/d), q = RN(S r) (Markstein's final
-                // step), which needs d and r far from the ends of the fp32 range; rows outside these
-                // bounds take the general path below
+                // The fast path forms S = P + rt_g + (128 + z_row) cs of eq. (1) in fp32: the tensor-core
+                // sum P is an exact integer, and when |rt_g| + |128 + z_row| 255 K < 2^24 the offset term
+                // rt_g + (128 + z_row) cs is an exact integer too (cs <= 255 K) and one fused multiply-add
+                // forms it without rounding, so the single rounded addition P + (offset term) equals the
+                // correctly rounded S (S itself stays below 2^31 when K max|a' + za| max|w' + zw| < 2^31).
+                // The quotient S / (Qa Qw) is the correctly rounded q + (S - q d) r with r = RN(1/d),
+                // q = RN(S r) (Markstein's final step), which needs d and r far from the ends of the fp32
+                // range. Rows outside these bounds take the general path below.
                 cm0 = m0;
                 const long long ax = max(abs(zx), abs(zx + 255)), ah = max(abs(za), abs(za + 255));
                 bool f = bv;
@@ -942,10 +874,16 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 for (int g = 0; g < 4; ++g) {
                     const qnn_qparams qw = args.pw_x[g], qh = args.pw[g];
                     const float dx = __fmul_rn(Qx, qw.Q), dh = __fmul_rn(Qa, qh.Q);
+                    const long long rtx = (long long)(128 + qw.z) * rsx + (long long)args.K_x * ((long long)zx * qw.z - 16384);
+                    const long long rth = (long long)(128 + qh.z) * rs + (long long)K * ((long long)za * qh.z - 16384);
                     rcs[g * 32] = __frcp_rn(dx);
                     rcs[(4 + g) * 32] = __frcp_rn(dh);
+                    rcs[(8 + g) * 32] = (float)rtx;  // exact when the bound below holds
+                    rcs[(12 + g) * 32] = (float)rth;
                     f &= (long long)args.K_x * ax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31) &&
                          (long long)K * ah * (long long)max(abs(qh.z), abs(qh.z + 255)) < (1LL << 31) &&
+                         llabs(rtx) + (long long)abs(128 + zx) * 255 * args.K_x < (1LL << 24) &&
+                         llabs(rth) + (long long)abs(za128) * 255 * K < (1LL << 24) &&
                          dx >= 0x1p-60f && dx <= 0x1p60f && dh >= 0x1p-60f && dh <= 0x1p60f;
                 }
                 fastrow = f;
@@ -966,9 +904,9 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     const int jt = j0 - (int)(n0 / 4);  // cell within the tile
                     const uint32_t tx = tmem_base + ((uint32_t)(32 * q) << 16) +
                                         (uint32_t)(buf * TL::ACC_COLS + gi * 32 + part * CPS);
-                    // column constants of the slice from shared memory: bias, Wx and Wh row code sums
+                    // column constants of the slice from shared memory: bias, Wx and Wh row code sums (the
+                    // sums as exact fp32 integers)
                     const float *colb = pxb + TL::PX_BOX / 4 + jt;
-                    const int *coli = reinterpret_cast<const int *>(colb);
                     // two cells at a time (fewer live registers): the four gates' x and h sums from
                     // tensor memory (warp-wide loads), eq. (1)/(3), then the cell update. Rows whose
                     // constants were cached take reciprocal-based quotients and 32-bit sums; the others
@@ -988,28 +926,18 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                         if (fastrow) {
 #pragma unroll
                             for (int g = 0; g < 4; ++g) {
-                                float bias[2];
-                                int csx[2], csh[2];
+                                float bias[2], csx[2], csh[2];
                                 ld_vec(colb + g * CW + c2, bias);
-                                ld_vec(coli + (4 + g) * CW + c2, csx);
-                                ld_vec(coli + (8 + g) * CW + c2, csh);
+                                ld_vec(colb + (4 + g) * CW + c2, csx);
+                                ld_vec(colb + (8 + g) * CW + c2, csh);
                                 const qnn_qparams qw = s_pw[g], qh = s_pw[4 + g];
                                 const float dx = __fmul_rn(Qx, qw.Q), dh = __fmul_rn(Qa, qh.Q);
                                 const float rcx = rcs[g * 32], rch = rcs[(4 + g) * 32];
-                                // rt of eq. (1) for this row and gate, modulo 2^32 (S itself fits in 32 bits)
-                                const uint32_t rtx = (uint32_t)(128 + qw.z) * (uint32_t)rsx +
-                                                     (uint32_t)args.K_x * (uint32_t)(zx * qw.z - 16384);
-                                const uint32_t rth = (uint32_t)(128 + qh.z) * (uint32_t)rs +
-                                                     (uint32_t)K * (uint32_t)(za * qh.z - 16384);
-                                float2 vx, vh;
-                                vx.x = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rx[g][0])) +
-                                                            rtx + (uint32_t)(128 + zx) * (uint32_t)csx[0]));
-                                vx.y = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rx[g][1])) +
-                                                            rtx + (uint32_t)(128 + zx) * (uint32_t)csx[1]));
-                                vh.x = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rh[g][0])) +
-                                                            rth + (uint32_t)za128 * (uint32_t)csh[0]));
-                                vh.y = __int2float_rn((int)((uint32_t)f32_integer_to_s32(__uint_as_float(rh[g][1])) +
-                                                            rth + (uint32_t)za128 * (uint32_t)csh[1]));
+                                // S = P + (rt + (128 + z) cs): the offset term exact, then one rounding
+                                const float2 ox = ffma2_rn(f2(zx128f), make_float2(csx[0], csx[1]), f2(rcs[(8 + g) * 32]));
+                                const float2 oh = ffma2_rn(f2(za128f), make_float2(csh[0], csh[1]), f2(rcs[(12 + g) * 32]));
+                                const float2 vx = fadd2_rn(make_float2(__uint_as_float(rx[g][0]), __uint_as_float(rx[g][1])), ox);
+                                const float2 vh = fadd2_rn(make_float2(__uint_as_float(rh[g][0]), __uint_as_float(rh[g][1])), oh);
                                 const float2 yx = fadd2_rn(div_by_recip2(vx, dx, rcx), make_float2(bias[0], bias[1]));
                                 const float2 y = fadd2_rn(yx, div_by_recip2(vh, dh, rch));
                                 pre[g][0] = y.x;
@@ -1028,11 +956,12 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                                 const bool fits =
                                     (long long)args.K_x * ax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31) &&
                                     (long long)K * ah * (long long)max(abs(qh.z), abs(qh.z + 255)) < (1LL << 31);
-                                float bias[2];
-                                int csx[2], csh[2];
+                                float bias[2], csxf[2], cshf[2];
                                 ld_vec(colb + g * CW + c2, bias);
-                                ld_vec(coli + (4 + g) * CW + c2, csx);
-                                ld_vec(coli + (8 + g) * CW + c2, csh);
+                                ld_vec(colb + (4 + g) * CW + c2, csxf);
+                                ld_vec(colb + (8 + g) * CW + c2, cshf);
+                                const int csx[2] = {__float2int_rn(csxf[0]), __float2int_rn(csxf[1])};
+                                const int csh[2] = {__float2int_rn(cshf[0]), __float2int_rn(cshf[1])};
 #pragma unroll
                                 for (int jj = 0; jj < 2; ++jj) {
                                     const int Px = f32_integer_to_s32(__uint_as_float(rx[g][jj]));
@@ -1239,6 +1168,11 @@ qnn_status make_map(CUtensorMap *map, const __half *base, int64_t rows, int64_t 
 }
 
 }  // namespace
+
+qnn_status tc_map_f16(CUtensorMap *map, const __half *base, int64_t rows, int64_t ld, int box_rows) {
+    if (ld % TBK || box_rows < 1 || box_rows > 256 || (reinterpret_cast<uintptr_t>(base) & 15)) return QNN_ERR_INVALID_ARG;
+    return make_map(map, base, rows, ld, box_rows);
+}
 
 size_t tc_scratch_bytes(int64_t M, int64_t N, int64_t K) {
     const int64_t kp = (K + 63) / 64 * 64;

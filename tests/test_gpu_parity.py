@@ -512,6 +512,35 @@ def test_tc_input_product_fused_and_batched(qnn, cfg, fuse, monkeypatch):
     _compare(got, ref, wl, params)
 
 
+# The LSTMP projection of a step as one cluster launch (lstmp_proj.cu) and as split-K partial sums
+# with a finishing row kernel, both against the oracle: a partial last 128-row block, a reduction of
+# one pipeline stage (H = 100), two exact accumulation chunks with a short second one (H = 1100),
+# column groups of 16 to 64 (P = 128 .. 512; P = 384 takes the element-wise code stores), and the
+# full 2048 x 512 shape.
+CLUSTER_PROJ_CASES = [dict(L=2, I=40, H=256, P=128, C=11, B=130, T=4, w=0.1),
+                      dict(L=1, I=24, H=100, P=256, B=64, T=3),
+                      dict(L=1, I=16, H=1100, P=384, B=70, T=3, w=0.1),
+                      dict(L=2, I=80, H=2048, P=512, C=20, B=129, T=3, w=0.05)]
+
+
+@pytest.mark.parametrize("mode", ["cluster", "split"])
+@pytest.mark.parametrize("cfg", CLUSTER_PROJ_CASES)
+def test_tc_lstmp_projection_forms(qnn, cfg, mode, monkeypatch):
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    monkeypatch.setenv("QNN_TC_PROJ", mode)
+    wl = _small(**cfg)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x, want_h_all=True)
+    qnn.profile_read()
+    qnn.profile_enable(True)
+    got = _gpu_forward(qnn, wl, params, x)
+    qnn.profile_enable(False)
+    kernels = qnn.profile_read()
+    assert ("lstmp_proj_tc" in kernels) == (mode == "cluster"), kernels
+    assert ("proj_finish" in kernels) == (mode == "split"), kernels
+    _compare(got, ref, wl, params)
+
+
 @pytest.mark.parametrize("bn,fuse", [("32", "1"), ("64", "1"), ("96", "0")])
 def test_tc_recurrence_large_weight_offsets(qnn, bn, fuse, monkeypatch):
     # every weight shifted by +20: weight ranges far from zero give offsets z of about 32000, so
@@ -638,6 +667,7 @@ def _block_scaled(params, wl, nb, seed):
 
 SUB_CASES = [("small", dict(L=2, I=40, H=96, C=12, B=2, T=10), 4), ("layerwise", dict(L=2, I=24, H=48, P=16, C=8, B=9, T=5), 2),
              ("tc", dict(L=2, I=24, H=64, P=32, C=16, B=70, T=4), 4), ("tc", dict(L=1, I=40, H=96, B=130, T=3), 3),
+             ("tc", dict(L=2, I=24, H=128, P=128, C=16, B=70, T=4), 4),
              ("layerwise", dict(L=1, I=40, H=12, B=6, T=5), 6)]
 
 
