@@ -239,16 +239,51 @@ __global__ void __launch_bounds__(256) proj_finish_kernel(const FinishArgs a) {
             for (int e = 0; e < 8; ++e)
                 if (k0 + e < a.P) Psum[e] += a.part[((int64_t)s * a.rows + r) * a.ldpart + k0 + e];
     }
+    // The usual case: the 8 columns lie in one weight unit and the sums S of eq. (1) fit in 32 bits
+    // (K max|a' + za| max|w' + zw| < 2^31: wrapping 32-bit arithmetic gives them exactly), so S =
+    // Psum + rt + (128 + za) cs, and S / (Qa Qw) is taken from the divisor's correctly rounded
+    // reciprocal (div_by_recip: the IEEE quotient while the divisor stays within 2^-60 .. 2^60).
+    // Otherwise each output the general way (64-bit S, IEEE divide).
+    const int u0 = k0 / a.rows_per_unit;
+    bool fast = rv && k0 + 8 <= a.P && (k0 + 7) / a.rows_per_unit == u0 && (reinterpret_cast<uintptr_t>(a.wp_sum) & 15) == 0;
+    qnn_qparams qw0{};
+    float d = 1.0f;
+    if (fast) {
+        qw0 = a.wp_p[u0];
+        d = __fmul_rn(Qa, qw0.Q);
+        fast = (long long)a.K * max(abs(za), abs(za + 255)) * (long long)max(abs(qw0.z), abs(qw0.z + 255)) < (1LL << 31) &&
+               d >= 0x1p-60f && d <= 0x1p60f;
+    }
+    if (fast) {
+        const float rcp = __frcp_rn(d);
+        const uint32_t rt = (uint32_t)(128 + qw0.z) * (uint32_t)ra + (uint32_t)a.K * (uint32_t)(za * qw0.z - 16384);
+        const int4 c0 = *reinterpret_cast<const int4 *>(a.wp_sum + k0), c1 = *reinterpret_cast<const int4 *>(a.wp_sum + k0 + 4);
+        const int cs[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const int n = k0 + e;
-        v[e] = 0.0f;
-        if (rv && n < a.P) {
-            const int cs = a.wp_sum[n];
-            const qnn_qparams qw = a.wp_p[n / a.rows_per_unit];
-            const int acc = Psum[e] + 128 * (ra + cs) - 16384 * a.K;  // raw code product
-            v[e] = recover_product(offset_product(acc, za, qw.z, ra, cs, a.K), Qa, qw.Q);
-            a.out[(int64_t)r * a.ldo + n] = v[e];
+        for (int e = 0; e < 8; ++e) {
+            const int S = (int)((uint32_t)Psum[e] + rt + (uint32_t)(128 + za) * (uint32_t)cs[e]);
+            v[e] = div_by_recip(__int2float_rn(S), d, rcp);
+        }
+        float *o = a.out + (int64_t)r * a.ldo + k0;
+        if ((reinterpret_cast<uintptr_t>(o) & 15) == 0) {
+            *reinterpret_cast<float4 *>(o) = make_float4(v[0], v[1], v[2], v[3]);
+            *reinterpret_cast<float4 *>(o + 4) = make_float4(v[4], v[5], v[6], v[7]);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[e] = v[e];
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int n = k0 + e;
+            v[e] = 0.0f;
+            if (rv && n < a.P) {
+                const int cs = a.wp_sum[n];
+                const qnn_qparams qw = a.wp_p[n / a.rows_per_unit];
+                const int acc = Psum[e] + 128 * (ra + cs) - 16384 * a.K;  // raw code product
+                v[e] = recover_product(offset_product(acc, za, qw.z, ra, cs, a.K), Qa, qw.Q);
+                a.out[(int64_t)r * a.ldo + n] = v[e];
+            }
         }
     }
     if (!a.quantize) return;

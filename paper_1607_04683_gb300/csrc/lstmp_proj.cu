@@ -239,6 +239,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int e = 0; e < 4; ++e)
                     if (4 * g4 < nv) run[4 * g4 + e] += f32_integer_to_s32(__uint_as_float(r4[g4][e]));
         }
+        // The usual case: the thread's columns share one weight unit and the sums S of eq. (1) fit in
+        // 32 bits (K max|a' + za| max|w' + zw| < 2^31: wrapping 32-bit arithmetic gives them exactly),
+        // so S = run + rt + (128 + za) cs and S / (Qa Qw) comes from the divisor's correctly rounded
+        // reciprocal (div_by_recip: the IEEE quotient while the divisor stays within 2^-60 .. 2^60);
+        // otherwise each output the general way (64-bit S, IEEE divide).
+        const ColConst cf = scol[c0], cl = scol[c0 + nv - 1];
+        const float d = __fmul_rn(Qa, cf.Qw);
+        const bool fast = cf.zw == cl.zw && __float_as_uint(cf.Qw) == __float_as_uint(cl.Qw) &&
+                          (long long)a.K * max(abs(za), abs(za + 255)) * (long long)max(abs(cf.zw), abs(cf.zw + 255)) <
+                              (1LL << 31) &&
+                          d >= 0x1p-60f && d <= 0x1p60f;
+        const float rcp = fast ? __frcp_rn(d) : 1.0f;
+        const uint32_t rt = (uint32_t)(128 + cf.zw) * (uint32_t)ra + (uint32_t)a.K * (uint32_t)(za * cf.zw - 16384);
         float v[16];
         float mn = FLT_MAX, mx = -FLT_MAX;
         bool bad = false;
@@ -247,8 +260,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             v[e] = 0.0f;
             if (e < nv) {
                 const ColConst cc = scol[c0 + e];
-                const int acc = run[e] + 128 * (ra + cc.cs) - 16384 * a.K;  // raw code product
-                v[e] = recover_product(offset_product(acc, za, cc.zw, ra, cc.cs, a.K), Qa, cc.Qw);
+                if (fast) {
+                    const int S = (int)((uint32_t)run[e] + rt + (uint32_t)(128 + za) * (uint32_t)cc.cs);
+                    v[e] = div_by_recip(__int2float_rn(S), d, rcp);
+                } else {
+                    const int acc = run[e] + 128 * (ra + cc.cs) - 16384 * a.K;  // raw code product
+                    v[e] = recover_product(offset_product(acc, za, cc.zw, ra, cc.cs, a.K), Qa, cc.Qw);
+                }
                 bad |= !isfinite(v[e]);
                 mn = fminf(mn, v[e]);
                 mx = fmaxf(mx, v[e]);

@@ -912,6 +912,9 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     // constants were cached take reciprocal-based quotients and 32-bit sums; the others
                     // the general way (any weight unit, 64-bit sums when needed, IEEE divides).
                     const int unit = j0 / E.cpu;
+                    // the slice's cell state in, and its new state and outputs out, as one vector each
+                    float cst[CPS], mst[CPS];
+                    if (valid) ld_vec(pxb + C_OFF / 4 + rl * CW + jt, cst);
 #pragma unroll
                     for (int c2 = 0; c2 < CPS; c2 += 2) {
                         uint32_t rx[4][2], rh[4][2];
@@ -981,12 +984,16 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                                 }
                             }
                         }
-                        float2 cv = *reinterpret_cast<const float2 *>(pxb + C_OFF / 4 + rl * CW + jt + c2);
+                        float2 cv = make_float2(cst[c2], cst[c2 + 1]);
                         const float2 mv = lstm_cell2(make_float2(pre[0][0], pre[0][1]), make_float2(pre[1][0], pre[1][1]),
                                                      make_float2(pre[2][0], pre[2][1]), make_float2(pre[3][0], pre[3][1]),
                                                      cv);
-                        *reinterpret_cast<float2 *>(E.c + b * (int64_t)H + j0 + c2) = cv;
-                        *reinterpret_cast<float2 *>(E.h + b * E.h_ld + j0 + c2) = mv;
+                        cst[c2] = cv.x, cst[c2 + 1] = cv.y;
+                        mst[c2] = mv.x, mst[c2 + 1] = mv.y;
+                    }
+                    if (valid) {
+                        st_vec(E.c + b * (int64_t)H + j0, cst);
+                        st_vec(E.h + b * E.h_ld + j0, mst);
                     }
                     continue;
                 }
