@@ -390,15 +390,11 @@ int64_t max_proj_splits(const qnn_lstm_model *m) {
 }
 
 // The projection of a step after the m_t quantizer: by default split-K partial sums and a finishing
-// row kernel (P <= 2048); QNN_TC_PROJ=cluster one cluster launch (lstmp_proj.cu) for the shapes it
-// takes; QNN_TC_PROJ=linear, and P > 2048, one tensor-core product over the whole K whose epilogue
-// writes r_t, the next step's quantizer then reading r_t.
-enum class ProjMode { kCluster, kSplit, kLinear };
-ProjMode proj_mode(int64_t H, int64_t P) {
+// row kernel (P <= 2048); with QNN_TC_PROJ=linear, and for P > 2048, one tensor-core product over
+// the whole K whose epilogue writes r_t, the next step's quantizer then reading r_t.
+bool split_proj_enabled(int64_t P) {
     const char *e = std::getenv("QNN_TC_PROJ");
-    if (e && std::strcmp(e, "linear") == 0) return ProjMode::kLinear;
-    if (e && std::strcmp(e, "cluster") == 0 && tc_proj_cluster_supported(H, P)) return ProjMode::kCluster;
-    return P <= 2048 ? ProjMode::kSplit : ProjMode::kLinear;
+    return P <= 2048 && !(e && std::strcmp(e, "linear") == 0);
 }
 
 // Programmatic dependent launches between the recurrence's kernels (QNN_PDL=0 turns them off).
@@ -548,18 +544,11 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     int bn_gates = fx ? tc_choose_bn(B, 4 * H8, gate_bn_fused, 3) : tc_choose_bn(B, 4 * H8, gate_bn, 4);
     if (fx && !std::getenv("QNN_TC_BN") && ((B + 127) / 128) * ((4 * H8 + 127) / 128) >= sm_count()) bn_gates = 128;
     QNN_TRY(tc_operands(&gates, a16, B, tl.wh16, 4 * H8, kh, bn_gates));
-    // the projection after the m_t quantizer: one cluster launch (the product, the recovery and r_t's
-    // quantization); or split-K partial sums finished (offsets, recovery, next step's quantization)
-    // by one row kernel; or one tcgen05 product with its own epilogue per step
-    const ProjMode pmode = P > 0 ? proj_mode(H, P) : ProjMode::kLinear;
-    const bool cluster_proj = P > 0 && pmode == ProjMode::kCluster;
-    const bool split_proj = P > 0 && pmode == ProjMode::kSplit;
+    // the projection after the m_t quantizer: split-K partial sums finished (offsets, recovery, next
+    // step's quantization) by one row kernel; or one tcgen05 product with its own epilogue per step
+    const bool split_proj = P > 0 && split_proj_enabled(P);
     int splits = 0;
-    CUtensorMap m_map, wp_map;
-    if (cluster_proj) {
-        QNN_TRY(tc_map_f16(&m_map, m16, B, kpj, 128));
-        QNN_TRY(tc_map_f16(&wp_map, tl.wp16, P, kpj, (int)(P / 8)));
-    } else if (P > 0) {
+    if (P > 0) {
         QNN_TRY(tc_operands(&proj, m16, B, tl.wp16, P, kpj, split_proj ? 128 : tc_pick_bn(B, P, kpj)));
         if (split_proj) splits = tc_partial_splits(proj, (int)max_proj_splits(m));
     }
@@ -578,7 +567,7 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     }
     QNN_TRY(launch_quantize_rows_f16(h0, R, B, R, kh, a16, prm, rs, status, false, st));
     for (int64_t t = 0; t < T; ++t) {
-        if (t > 0 && !split_proj && !cluster_proj)
+        if (t > 0 && !split_proj)
             QNN_TRY(launch_quantize_rows_f16(out + (t - 1) * R, T * R, B, R, kh, a16, prm, rs, status, gates.pdl, st));
         TcLstmOut o{fx ? nullptr : px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R,
                     (int)H, (int)m->S, (int)(H / m->S)};
@@ -590,14 +579,7 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
         }
         if (P > 0) {
             QNN_TRY(launch_quantize_rows_f16(mbuf, H, B, H, kpj, m16, prm_m, rs_m, status, gates.pdl, st));
-            if (cluster_proj) {
-                TcProjStep ps;
-                ps.amap = &m_map, ps.wmap = &wp_map, ps.prm_m = prm_m, ps.rs_m = rs_m;
-                ps.wp_p = ly.wp.params, ps.wp_sum = ly.wp.sums, ps.rows_per_unit = P / m->S;
-                ps.out = out + t * R, ps.ldo = T * R, ps.B = B, ps.H = H, ps.kp = kpj, ps.P = P;
-                ps.quantize = t + 1 < T, ps.kh = kh, ps.dst = a16, ps.prm = prm, ps.rsum = rs;
-                QNN_TRY(tc_lstmp_projection(ps, gates.pdl, st));
-            } else if (split_proj) {
+            if (split_proj) {
                 QNN_TRY(tc_partial(proj, splits, part, P, st));
                 FinishArgs fa{part, splits, P, prm_m, rs_m, ly.wp.params, ly.wp.sums, (int)(P / m->S), (int)H,
                               out + t * R, T * R, (int)B, (int)P, t + 1 < T, (int)kh, a16, prm, rs, status};

@@ -111,8 +111,7 @@ struct Tile {
     // warps sit on the four SM sub-partitions by index: 18 warps put 5 on one (5 x 32 x 96 <= 16384),
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : (LSTM96 ? 72 : 96);
-    static constexpr uint32_t IDESC =
-        (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TBM >> 4) << 24);
+    static constexpr uint32_t IDESC = mma_idesc_f16(TBM, BN);
     static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + EPI_BYTES + 256;
 };
 
@@ -584,7 +583,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 }
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
-                if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+                if (lane == 0) mb_arrive(drained0 + 8 * buf);
             }
             const int64_t m = m0 + 32 * q + lane;
             if (failed || m >= args.M) continue;
@@ -735,7 +734,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
-            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+            if (lane == 0) mb_arrive(drained0 + 8 * buf);
             ++gc;
         }
     } else if constexpr (EPI == kEpiPartial) {
@@ -779,7 +778,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
-            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
+            if (lane == 0) mb_arrive(drained0 + 8 * buf);
         }
     } else {
         // ---------------- epilogue: LSTM cell update ----------------
@@ -1054,8 +1053,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) {
-                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(drained0 + 8 * buf) : "memory");
-                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(pxempty0 + 8 * pbuf) : "memory");
+                mb_arrive(drained0 + 8 * buf);
+                mb_arrive(pxempty0 + 8 * pbuf);
             }
             // refill the buffer with the tile two ahead once every epilogue warp has released it
             if (issuer && tile + 2 * (int64_t)gridDim.x < tiles &&
@@ -1175,11 +1174,6 @@ qnn_status make_map(CUtensorMap *map, const __half *base, int64_t rows, int64_t 
 }
 
 }  // namespace
-
-qnn_status tc_map_f16(CUtensorMap *map, const __half *base, int64_t rows, int64_t ld, int box_rows) {
-    if (ld % TBK || box_rows < 1 || box_rows > 256 || (reinterpret_cast<uintptr_t>(base) & 15)) return QNN_ERR_INVALID_ARG;
-    return make_map(map, base, rows, ld, box_rows);
-}
 
 size_t tc_scratch_bytes(int64_t M, int64_t N, int64_t K) {
     const int64_t kp = (K + 63) / 64 * 64;

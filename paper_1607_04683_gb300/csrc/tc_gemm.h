@@ -95,36 +95,6 @@ qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int3
 int tc_partial_splits(const TcOperands &op, int max_splits);
 qnn_status tc_partial(const TcOperands &op, int splits, int32_t *part, int64_t ldpart, cudaStream_t st);
 
-// One recurrent step's LSTMP projection in one cluster launch (lstmp_proj.cu): r_t = R(Q(m_t) Wp')
-// from the centered fp16 codes of m_t (amap: [B][kp], boxes of 64 x 128 rows; their units prm_m and
-// code sums rs_m, one unit per row), written to out (row b at out + b * ldo); with `quantize`,
-// r_t's codes, units and code sums for the next step go to dst [B][kh], prm [B], rsum [B].
-// wmap: Wp' [P][kp] centered fp16, boxes of 64 x P / 8 rows (tc_map_f16). K = H (true), kp its
-// padding to 64. Supported shapes: tc_proj_cluster_supported.
-struct TcProjStep {
-    const CUtensorMap *amap = nullptr, *wmap = nullptr;
-    const qnn_qparams *prm_m = nullptr;
-    const int32_t *rs_m = nullptr;
-    const qnn_qparams *wp_p = nullptr;
-    const int32_t *wp_sum = nullptr;
-    int64_t rows_per_unit = 0;
-    float *out = nullptr;
-    int64_t ldo = 0;
-    int64_t B = 0, H = 0, kp = 0, P = 0;
-    bool quantize = false;
-    int64_t kh = 0;
-    __half *dst = nullptr;
-    qnn_qparams *prm = nullptr;
-    int32_t *rsum = nullptr;
-};
-// P a multiple of 128 up to 512 (columns per CTA a multiple of 16), H's exact chunks times P / 8
-// at most 512 tensor-memory columns.
-bool tc_proj_cluster_supported(int64_t H, int64_t P);
-qnn_status tc_lstmp_projection(const TcProjStep &s, bool pdl, cudaStream_t st);
-// TMA map of a centered fp16 matrix [rows][ld] (ld a multiple of 64), boxes of 64 x box_rows,
-// 128-byte swizzle.
-qnn_status tc_map_f16(CUtensorMap *map, const __half *base, int64_t rows, int64_t ld, int box_rows);
-
 // u8 codes [rows][ldi] -> centered fp16 [rows][ldo], zero past K.
 qnn_status launch_center_fp16(const uint8_t *in, int64_t rows, int64_t K, int64_t ldi, __half *out, int64_t ldo,
                               cudaStream_t st);

@@ -1,7 +1,5 @@
-// tc_ptx.cuh — inline-PTX building blocks of the sm_103a tensor-core kernels (qgemm_tc.cu,
-// lstmp_proj.cu): shared-memory mbarriers, TMA tile loads, tcgen05 MMA descriptors, issue and
-// commit, tensor-memory loads, and the thread-block-cluster operations (distributed shared memory,
-// the cluster barrier, bulk reduce-copies between the CTAs of a cluster).
+// tc_ptx.cuh — inline-PTX building blocks of the sm_103a tensor-core kernels: shared-memory
+// mbarriers, TMA tile loads, tcgen05 MMA descriptors, issue and commit, tensor-memory loads.
 #pragma once
 
 #include <cstdint>
@@ -58,14 +56,6 @@ __device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_
         "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate)
         : "memory");
 }
-__device__ __forceinline__ void mma_f16_rt(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                           uint32_t accumulate) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
 // Arrives on `bar` once every MMA issued so far by this thread has completed.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
@@ -94,12 +84,7 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         : "r"(taddr));
     tmem_wait_ld();
 }
-// 8, 4 or 2 consecutive fp32 columns, without the wait (the caller waits once for several loads).
-__device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[8]) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                 : "r"(taddr));
-}
+// 4 or 2 consecutive fp32 columns, without the wait (the caller waits once for several loads).
 __device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[4]) {
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
@@ -107,48 +92,6 @@ __device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[4])
 }
 __device__ __forceinline__ void tmem_ld_nowait(uint32_t taddr, uint32_t (&r)[2]) {
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(taddr));
-}
-
-// ---- thread-block clusters ----
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-// The address under which this CTA reaches the shared-memory location `addr` (a shared::cta
-// address of this CTA's layout) in CTA `rank` of its cluster.
-__device__ __forceinline__ uint32_t cluster_map(uint32_t addr, uint32_t rank) {
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-    return r;
-}
-__device__ __forceinline__ void st_cluster_u32(uint32_t addr, uint32_t v) {
-    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-__device__ __forceinline__ void st_cluster_v2(uint32_t addr, uint32_t a, uint32_t b) {
-    asm volatile("st.shared::cluster.v2.u32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
-}
-// Cluster-wide barrier of every thread of every CTA of the cluster: the arrival releases this
-// thread's earlier memory operations (shared memory of any CTA of the cluster, global memory) and
-// the wait acquires those of every arrival. Every warp executes both halves convergently.
-__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
-__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
-__device__ __forceinline__ void cluster_sync() {
-    cluster_arrive();
-    cluster_wait();
-}
-// Makes this thread's generic-proxy writes to shared memory visible to later asynchronous-proxy
-// operations (TMA, bulk copies, tensor-core operand reads).
-__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-// Element-wise 32-bit integer add of `bytes` (a multiple of 16) from this CTA's shared memory `src`
-// into shared memory `dst` of a CTA of the cluster (dst and bar: cluster addresses from
-// cluster_map); completion counted in bytes on the mbarrier `bar` of the destination CTA.
-__device__ __forceinline__ void bulk_reduce_add_u32(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t bar) {
-    asm volatile(
-        "cp.reduce.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes.add.u32 [%0], [%1], %2, [%3];" ::"r"(
-            dst),
-        "r"(src), "r"(bytes), "r"(bar)
-        : "memory");
 }
 
 }  // namespace qnn

@@ -512,19 +512,18 @@ def test_tc_input_product_fused_and_batched(qnn, cfg, fuse, monkeypatch):
     _compare(got, ref, wl, params)
 
 
-# The LSTMP projection of a step as one cluster launch (lstmp_proj.cu) and as split-K partial sums
-# with a finishing row kernel, both against the oracle: a partial last 128-row block, a reduction of
-# one pipeline stage (H = 100), two exact accumulation chunks with a short second one (H = 1100),
-# column groups of 16 to 64 (P = 128 .. 512; P = 384 takes the element-wise code stores), and the
-# full 2048 x 512 shape.
-CLUSTER_PROJ_CASES = [dict(L=2, I=40, H=256, P=128, C=11, B=130, T=4, w=0.1),
-                      dict(L=1, I=24, H=100, P=256, B=64, T=3),
-                      dict(L=1, I=16, H=1100, P=384, B=70, T=3, w=0.1),
-                      dict(L=2, I=80, H=2048, P=512, C=20, B=129, T=3, w=0.05)]
+# The LSTMP projection of a step in both of its forms, split-K partial sums with a finishing row
+# kernel (the default) and one product whose epilogue writes r_t (QNN_TC_PROJ=linear), against the
+# oracle: a partial last 128-row block, a projection wider than the cells (H = 100, P = 256), two
+# exact accumulation chunks with a short second one (H = 1100), and the full 2048 x 512 shape.
+PROJ_CASES = [dict(L=2, I=40, H=256, P=128, C=11, B=130, T=4, w=0.1),
+              dict(L=1, I=24, H=100, P=256, B=64, T=3),
+              dict(L=1, I=16, H=1100, P=384, B=70, T=3, w=0.1),
+              dict(L=2, I=80, H=2048, P=512, C=20, B=129, T=3, w=0.05)]
 
 
-@pytest.mark.parametrize("mode", ["cluster", "split"])
-@pytest.mark.parametrize("cfg", CLUSTER_PROJ_CASES)
+@pytest.mark.parametrize("mode", ["split", "linear"])
+@pytest.mark.parametrize("cfg", PROJ_CASES)
 def test_tc_lstmp_projection_forms(qnn, cfg, mode, monkeypatch):
     monkeypatch.setenv("QNN_LSTM_PATH", "tc")
     monkeypatch.setenv("QNN_TC_PROJ", mode)
@@ -536,7 +535,6 @@ def test_tc_lstmp_projection_forms(qnn, cfg, mode, monkeypatch):
     got = _gpu_forward(qnn, wl, params, x)
     qnn.profile_enable(False)
     kernels = qnn.profile_read()
-    assert ("lstmp_proj_tc" in kernels) == (mode == "cluster"), kernels
     assert ("proj_finish" in kernels) == (mode == "split"), kernels
     _compare(got, ref, wl, params)
 
