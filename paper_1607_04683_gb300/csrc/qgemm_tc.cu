@@ -93,9 +93,10 @@ struct Tile {
     static constexpr int COL_BYTES = 12 * (BN / 4) * 4;
     static constexpr int LSTM_TX = EPI == kEpiLstmX ? PX_BOX + COL_BYTES : 5 * PX_BOX;  // bytes of one fill
     static constexpr int LSTM_BUF = (LSTM_TX + 1023) / 1024 * 1024;  // [4 px boxes +] the c box [+ constants]
-    // kEpiLstmX: per epilogue thread, the reciprocals of its row's eight divisors of eq. (3) and its
-    // eight row terms rt of eq. (1), kept in shared memory across the block's tiles ([warp][16][lane] floats)
-    static constexpr int RC_BYTES = EPI == kEpiLstmX ? EPI_WARPS * 16 * 32 * 4 : 0;
+    // kEpiLstmX: per epilogue thread, its row's per-gate constants of eq. (1)/(3), kept in shared
+    // memory across the block's tiles: per warp [4 gates][32 lanes] float4 (1/dx, 1/dh, rt_x, rt_h),
+    // then [4 gates][32 lanes] float2 (dx, dh)
+    static constexpr int RC_BYTES = EPI == kEpiLstmX ? EPI_WARPS * 24 * 32 * 4 : 0;
     static constexpr int EPI_BYTES = IS_LSTM              ? 2 * LSTM_BUF + RC_BYTES
                                      : EPI == kEpiPartial ? 0
                                                           : 2 * BN * (int)(sizeof(ColConst) + sizeof(ColUnit));
@@ -260,11 +261,6 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             tma_load_2d(dst, &mapW, bar, (kb - (LX ? args.KB_x : 0)) * TBK, n0);
     };
     __shared__ int s_abort;
-    // kEpiLstmX with one weight unit per gate matrix: the eight weight units (Wx then Wh, gates i f g
-    // o), read by every epilogue thread for every slice
-    __shared__ qnn_qparams s_pw[8];
-    if (LX && threadIdx.x < 8 && args.lstm.ups == 1)
-        s_pw[threadIdx.x] = threadIdx.x < 4 ? args.pw_x[threadIdx.x] : args.pw[threadIdx.x - 4];
 
     if (threadIdx.x == 0) {
         s_abort = 0;
@@ -827,9 +823,15 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         // terms are cheap to re-form
         int64_t cm0 = -1;
         bool fastrow = false;
-        float *const rcs = pxs0 + 2 * (TL::LSTM_BUF / 4) + (warp - 2) * 16 * 32 + lane;  // [16][32] per warp
+        float *const rcw = pxs0 + 2 * (TL::LSTM_BUF / 4) + (warp - 2) * 24 * 32;  // this warp's constants
+        float4 *const rq = reinterpret_cast<float4 *>(rcw) + lane;                 // rq[32 g]
+        float2 *const rd = reinterpret_cast<float2 *>(rcw + 16 * 32) + lane;       // rd[32 g]
         int64_t gc = 0;
         bool ok = true;
+        // row b's units and code sums: za, Qa, rs of h_{t-1}; zx, Qx, rsx of x_t (kEpiLstmX)
+        int64_t lm0 = -1;
+        int za = 0, rs = 0, zx = 0, rsx = 0;
+        float Qa = 1.0f, Qx = 1.0f;
         for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
             int64_t m0, n0;
             tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
@@ -838,24 +840,24 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             const int rl = 32 * q + lane;    // row within the tile
             const int64_t b = m0 + 32 * q + lane;
             const bool bv = b < args.M;
-            int za = 0, rs = 0;
-            float Qa = 1.0f;
-            if (bv) {
-                const qnn_qparams qa = args.pa[b];
-                za = qa.z;
-                Qa = qa.Q;
-                rs = args.rsA[b];
+            if (m0 != lm0) {  // the row's units and code sums (kept while the block stays on this row tile)
+                lm0 = m0;
+                za = 0, rs = 0, Qa = 1.0f, zx = 0, rsx = 0, Qx = 1.0f;
+                if (bv) {
+                    const qnn_qparams qa = args.pa[b];
+                    za = qa.z;
+                    Qa = qa.Q;
+                    rs = args.rsA[b];
+                }
+                if (LX && bv) {
+                    const qnn_qparams qa = args.pa_x[b * args.x_stride];
+                    zx = qa.z;
+                    Qx = qa.Q;
+                    rsx = args.rsA_x[b * args.x_stride];
+                }
             }
             const int za128 = 128 + za;
             const float za128f = (float)za128;
-            int zx = 0, rsx = 0;  // kEpiLstmX: the unit and code sum of row b of x_t
-            float Qx = 1.0f;
-            if (LX && bv) {
-                const qnn_qparams qa = args.pa_x[b * args.x_stride];
-                zx = qa.z;
-                Qx = qa.Q;
-                rsx = args.rsA_x[b * args.x_stride];
-            }
             const float zx128f = (float)(128 + zx);
             if (LX && E.ups == 1 && m0 != cm0) {
                 // The fast path forms S = P + rt_g + (128 + z_row) cs of eq. (1) in fp32: the tensor-core
@@ -875,10 +877,9 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                     const float dx = __fmul_rn(Qx, qw.Q), dh = __fmul_rn(Qa, qh.Q);
                     const long long rtx = (long long)(128 + qw.z) * rsx + (long long)args.K_x * ((long long)zx * qw.z - 16384);
                     const long long rth = (long long)(128 + qh.z) * rs + (long long)K * ((long long)za * qh.z - 16384);
-                    rcs[g * 32] = __frcp_rn(dx);
-                    rcs[(4 + g) * 32] = __frcp_rn(dh);
-                    rcs[(8 + g) * 32] = (float)rtx;  // exact when the bound below holds
-                    rcs[(12 + g) * 32] = (float)rth;
+                    // (rt_x, rt_h exact when the bound below holds)
+                    rq[32 * g] = make_float4(__frcp_rn(dx), __frcp_rn(dh), (float)rtx, (float)rth);
+                    rd[32 * g] = make_float2(dx, dh);
                     f &= (long long)args.K_x * ax * (long long)max(abs(qw.z), abs(qw.z + 255)) < (1LL << 31) &&
                          (long long)K * ah * (long long)max(abs(qh.z), abs(qh.z + 255)) < (1LL << 31) &&
                          llabs(rtx) + (long long)abs(128 + zx) * 255 * args.K_x < (1LL << 24) &&
@@ -932,12 +933,12 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                                 ld_vec(colb + g * CW + c2, bias);
                                 ld_vec(colb + (4 + g) * CW + c2, csx);
                                 ld_vec(colb + (8 + g) * CW + c2, csh);
-                                const qnn_qparams qw = s_pw[g], qh = s_pw[4 + g];
-                                const float dx = __fmul_rn(Qx, qw.Q), dh = __fmul_rn(Qa, qh.Q);
-                                const float rcx = rcs[g * 32], rch = rcs[(4 + g) * 32];
+                                const float4 rr = rq[32 * g];  // 1/dx, 1/dh, rt_x, rt_h
+                                const float2 dd = rd[32 * g];  // dx, dh
+                                const float dx = dd.x, dh = dd.y, rcx = rr.x, rch = rr.y;
                                 // S = P + (rt + (128 + z) cs): the offset term exact, then one rounding
-                                const float2 ox = ffma2_rn(f2(zx128f), make_float2(csx[0], csx[1]), f2(rcs[(8 + g) * 32]));
-                                const float2 oh = ffma2_rn(f2(za128f), make_float2(csh[0], csh[1]), f2(rcs[(12 + g) * 32]));
+                                const float2 ox = ffma2_rn(f2(zx128f), make_float2(csx[0], csx[1]), f2(rr.z));
+                                const float2 oh = ffma2_rn(f2(za128f), make_float2(csh[0], csh[1]), f2(rr.w));
                                 const float2 vx = fadd2_rn(make_float2(__uint_as_float(rx[g][0]), __uint_as_float(rx[g][1])), ox);
                                 const float2 vh = fadd2_rn(make_float2(__uint_as_float(rh[g][0]), __uint_as_float(rh[g][1])), oh);
                                 const float2 yx = fadd2_rn(div_by_recip2(vx, dx, rcx), make_float2(bias[0], bias[1]));
