@@ -22,6 +22,7 @@
 
 #include <cstdio>
 #include <cstdlib>
+#include <cstring>
 #include <algorithm>
 #include <mutex>
 
@@ -113,6 +114,7 @@ struct Tile {
     // 26 warps put 7 on one (7 x 32 x 72 <= 16384)
     static constexpr int MAX_REGS = EPI == kEpiLinear ? 168 : (LSTM96 ? 72 : 96);
     static constexpr uint32_t IDESC = mma_idesc_f16(TBM, BN);
+    static constexpr uint32_t IDESC_HALF = mma_idesc_f16(TBM, BN / 2 >= 16 ? BN / 2 : 16);  // half-width items
     static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + EPI_BYTES + 256;
 };
 
@@ -149,6 +151,9 @@ struct TcArgs {
     const int32_t *csW_x;
     const float *bias_x;
     int K_x, KB_x;
+    // LSTM epilogues: tiles from full_tiles on (the last, partial wave of the persistent grid) run as
+    // two half-width items each, so that the blocks of that wave finish together (0: none)
+    int64_t full_tiles;
 };
 
 __device__ __forceinline__ unsigned long long gtime() { return global_timer_ns(); }
@@ -244,9 +249,25 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
     const int tiles_n = (int)((args.N + BN - 1) / BN);
     const int64_t tiles_m = (args.M + TBM - 1) / TBM;
     const int64_t tiles = tiles_m * tiles_n;
-    // work items: (tile, K range); one K range per tile except for split-K
+    // work items: (tile, K range); one K range per tile except for split-K. LSTM epilogues may split
+    // the tiles of the last wave into half-width items (the first BN / 2 columns of the tile's W box
+    // feed an MMA of N = BN / 2; the px, c and constant boxes are loaded whole)
     const int splits = args.splits;
-    const int64_t items = tiles * splits;
+    const int64_t full_tiles =
+        (TL::IS_LSTM && args.full_tiles > 0 && args.full_tiles < tiles) ? args.full_tiles : tiles;
+    const int64_t work = full_tiles + 2 * (tiles - full_tiles);  // tile items
+    const int64_t items = work * splits;
+    // origin of tile item w; true for a half-width item
+    auto item_origin = [&](int64_t w, int64_t &m0, int64_t &n0) -> bool {
+        if (w < full_tiles) {
+            tile_origin(w, tiles_m, tiles_n, BN, m0, n0);
+            return false;
+        }
+        const int64_t j = w - full_tiles;
+        tile_origin(full_tiles + j / 2, tiles_m, tiles_n, BN, m0, n0);
+        n0 += (j & 1) * (BN / 2);
+        return true;
+    };
     // the A and W tiles of k-block kb (kEpiLstmX: x_t and Wx for kb < KB_x, then h_{t-1} and Wh)
     auto load_a = [&](uint32_t dst, uint32_t bar, int kb, int m0) {
         if (LX && kb < args.KB_x)
@@ -303,7 +324,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         }
         if (args.w_static && blockIdx.x < items) {
             int64_t m0, n0;
-            tile_origin(blockIdx.x / splits, tiles_m, tiles_n, BN, m0, n0);
+            item_origin(blockIdx.x / splits, m0, n0);
             const int kb0 = (int)(blockIdx.x % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
             if constexpr (TL::KPS == 1) {
                 w_early = min(STAGES, kb1 - kb0);
@@ -350,7 +371,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 int64_t g = 0;  // k-blocks issued by this block
                 for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
                     int64_t m0, n0;
-                    tile_origin(item / splits, tiles_m, tiles_n, BN, m0, n0);
+                    item_origin(item / splits, m0, n0);
                     const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
                     for (int kb = kb0; kb < kb1; ++kb, ++g) {
                         const int s = (int)(g % STAGES);
@@ -381,7 +402,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 uint32_t st_addr = ring0, bar_full = full0, bar_empty = empty0;
                 for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
                     int64_t m0l, n0l;
-                    tile_origin(item / splits, tiles_m, tiles_n, BN, m0l, n0l);
+                    item_origin(item / splits, m0l, n0l);
                     const int m0 = (int)m0l, n0 = (int)n0l;
                     const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
                     for (int kb = kb0; kb < kb1; kb += TL::KPS) {
@@ -420,6 +441,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 int64_t g = 0, gc = 0;  // k-blocks and chunks consumed by this block
                 for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
                     const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                    const uint32_t idesc = item / splits < full_tiles ? TL::IDESC : TL::IDESC_HALF;
                     for (int kb = kb0; kb < kb1; ++kb, ++g) {
                         const int s = (int)(g % STAGES);
                         const int kc = (kb - kb0) % kpc;
@@ -442,8 +464,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
 #pragma unroll
                         for (int k = 0; k < TBK / 16; ++k) {
                             // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
-                            mma_f16<TL::IDESC>(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k),
-                                               (fresh && k == 0) ? 0u : 1u);
+                            mma_f16(tmem_d, smem_desc(sa + 32 * k), smem_desc(sb + 32 * k), idesc,
+                                    (fresh && k == 0) ? 0u : 1u);
                         }
                         mma_commit(empty0 + 8 * s);  // frees the stage when these MMAs have read it
                         if (kc == kpc - 1 || kb == kb1 - 1) {
@@ -466,6 +488,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 int64_t gc = 0;  // chunks accumulated by this block
                 for (int64_t item = blockIdx.x; item < items && !s_abort; item += gridDim.x) {
                     const int kb0 = (int)(item % splits) * args.kbs, kb1 = min(KB, kb0 + args.kbs);
+                    const uint32_t idesc = item / splits < full_tiles ? TL::IDESC : TL::IDESC_HALF;
                     int kc = 0;  // position of the stage in its K chunk (chunks hold whole stages)
                     for (int kb = kb0; kb < kb1; kb += TL::KPS) {
                         const int nv = min(TL::KPS, kb1 - kb);
@@ -491,9 +514,9 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
 #pragma unroll
                             for (int k = 0; k < TBK / 16; ++k) {
                                 // advance 16 fp16 = 32 bytes along K inside the swizzled 128-byte rows
-                                mma_f16<TL::IDESC>(tmem_d, da + (uint64_t)((v * A_BYTES + 32 * k) >> 4),
-                                                   db + (uint64_t)((v * TL::B_BYTES + 32 * k) >> 4),
-                                                   (fresh && k == 0) ? 0u : 1u);
+                                mma_f16(tmem_d, da + (uint64_t)((v * A_BYTES + 32 * k) >> 4),
+                                        db + (uint64_t)((v * TL::B_BYTES + 32 * k) >> 4), idesc,
+                                        (fresh && k == 0) ? 0u : 1u);
                             }
                         }
                         mma_commit(bar_empty);  // frees the stage when these MMAs have read it
@@ -744,7 +767,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         const bool vec = args.ldpart % 4 == 0;
         for (int64_t item = blockIdx.x; item < items && ok; item += gridDim.x, ++gc) {
             int64_t m0, n0;
-            tile_origin(item / splits, tiles_m, tiles_n, BN, m0, n0);
+            item_origin(item / splits, m0, n0);
             int32_t *dst = args.part + (item % splits) * args.M * args.ldpart;
             const int64_t m = m0 + 32 * q + lane;
             const int buf = (int)(gc & 1);
@@ -799,7 +822,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         const bool issuer = warp == 2 && lane == 0;
         auto issue_px = [&](int64_t t_issue, int pbuf) {
             int64_t m1, n1;
-            tile_origin(t_issue, tiles_m, tiles_n, BN, m1, n1);
+            item_origin(t_issue, m1, n1);
             const uint32_t bar = pxfull0 + 8 * pbuf;
             const uint32_t dst = su32(pxs0) + (uint32_t)(pbuf * TL::LSTM_BUF);
             mb_expect(bar, (uint32_t)TL::LSTM_TX);
@@ -814,8 +837,8 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             tma_load_2d(dst + C_OFF, &mapC, bar, (int)(n1 / 4), (int)m1);
         };
         if (issuer) {
-            if (blockIdx.x < tiles) issue_px(blockIdx.x, 0);
-            if (blockIdx.x + gridDim.x < tiles) issue_px(blockIdx.x + gridDim.x, 1);
+            if (blockIdx.x < work) issue_px(blockIdx.x, 0);
+            if (blockIdx.x + gridDim.x < work) issue_px(blockIdx.x + gridDim.x, 1);
         }
         // kEpiLstmX with one weight unit per gate matrix: the correctly rounded reciprocals of the
         // per-row, per-gate divisors Qa Qw of eq. (3) are computed once for the block's row tile and
@@ -832,9 +855,9 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
         int64_t lm0 = -1;
         int za = 0, rs = 0, zx = 0, rsx = 0;
         float Qa = 1.0f, Qx = 1.0f;
-        for (int64_t tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+        for (int64_t tile = blockIdx.x; tile < work && ok; tile += gridDim.x) {
             int64_t m0, n0;
-            tile_origin(tile, tiles_m, tiles_n, BN, m0, n0);
+            const int slices = item_origin(tile, m0, n0) ? SLICES / 2 : SLICES;  // half-width items: half the slices
             const int pbuf = (int)(gc & 1);  // this tile's px/c buffer (gc counts the block's tiles)
             const float *pxb = pxs0 + pbuf * (TL::LSTM_BUF / 4);
             const int rl = 32 * q + lane;    // row within the tile
@@ -894,7 +917,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll 1
-            for (int s = eh; s < SLICES; s += TL::EPI_WARPS / 4) {
+            for (int s = eh; s < slices; s += TL::EPI_WARPS / 4) {
                 const int gi = s / SPG, part = s % SPG;
                 const int j0 = (int)(n0 / 4) + gi * 8 + part * CPS;  // H is a multiple of 4: all CPS valid or none
                 if constexpr (LX) {
@@ -1058,7 +1081,7 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 mb_arrive(pxempty0 + 8 * pbuf);
             }
             // refill the buffer with the tile two ahead once every epilogue warp has released it
-            if (issuer && tile + 2 * (int64_t)gridDim.x < tiles &&
+            if (issuer && tile + 2 * (int64_t)gridDim.x < work &&
                 mb_wait(pxempty0 + 8 * pbuf, (unsigned)(gc / 2) & 1, args.status))
                 issue_px(tile + 2 * (int64_t)gridDim.x, pbuf);
             ++gc;
@@ -1211,6 +1234,16 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
     const int64_t items = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN) * a.splits;  // (tile, K range) pairs
     // persistent: one block per SM (a block holding tensor memory has its SM to itself)
     const unsigned grid = (unsigned)std::min<int64_t>(items, (int64_t)sm_count());
+    // LSTM tiles of 64 or 128 columns: when the last wave is partial and its tiles, halved, fit one
+    // wave, they run as two half-width items each (the busiest block then does half a tile less;
+    // QNN_TC_HALF=0 keeps whole tiles)
+    TcArgs args = a;
+    args.full_tiles = 0;
+    if (TL::IS_LSTM && (BN == 64 || BN == 128) && a.splits == 1 && items > grid) {
+        const char *e = std::getenv("QNN_TC_HALF");
+        const int64_t r = items % grid;
+        if (r > 0 && 2 * r <= grid && !(e && std::strcmp(e, "0") == 0)) args.full_tiles = items - r;
+    }
     ProfScope prof(name, st);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -1224,7 +1257,7 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
     cfg.numAttrs = op.pdl ? 1 : 0;
     // the px, c, x and Wx maps are read by the LSTM kernels only (the others get A's map, unused)
     QNN_CUDA_TRY(cudaLaunchKernelEx(&cfg, qgemm_tc_kernel<BN, EPI>, op.a, op.w, map_px ? *map_px : op.a,
-                                    map_c ? *map_c : op.a, map_ax ? *map_ax : op.a, map_wx ? *map_wx : op.w, a));
+                                    map_c ? *map_c : op.a, map_ax ? *map_ax : op.a, map_wx ? *map_wx : op.w, args));
     return QNN_OK;
 }
 

@@ -539,6 +539,22 @@ def test_tc_lstmp_projection_forms(qnn, cfg, mode, monkeypatch):
     _compare(got, ref, wl, params)
 
 
+# 192 tiles of the gate product on 152 SMs: the 40 tiles of the last wave run as 80 half-width
+# items (N = 64 or 32); the same results with whole tiles (QNN_TC_HALF=0) and from the oracle
+@pytest.mark.parametrize("half", ["1", "0"])
+@pytest.mark.parametrize("bn,cfg", [("128", dict(L=1, I=40, H=2048, P=128, B=384, T=2, w=0.05)),
+                                    ("64", dict(L=1, I=40, H=1024, B=384, T=2, w=0.05))])
+def test_tc_last_wave_half_tiles(qnn, bn, cfg, half, monkeypatch):
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    monkeypatch.setenv("QNN_TC_BN", bn)
+    monkeypatch.setenv("QNN_TC_HALF", half)
+    wl = _small(**cfg)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x, want_h_all=True)
+    got = _gpu_forward(qnn, wl, params, x)
+    _compare(got, ref, wl, params)
+
+
 @pytest.mark.parametrize("bn,fuse", [("32", "1"), ("64", "1"), ("96", "0")])
 def test_tc_recurrence_large_weight_offsets(qnn, bn, fuse, monkeypatch):
     # every weight shifted by +20: weight ranges far from zero give offsets z of about 32000, so
