@@ -81,20 +81,20 @@ __global__ void __launch_bounds__(32 * kQuantRowsPerBlock)
 }
 
 // Row-group quantizer shared by the kernels below: a group of G threads (a power of two) holds a
-// row of len values, 8 consecutive values per thread (v, starting at k0 = 8 t); writes the centered
-// fp16 codes [kp] (zero past len), the unit parameters and the code sum of the row (eq. 2).
-template <int G>
-__device__ __forceinline__ void quantize_row_group(const float (&v)[8], int len, int kp, int t, int rl, bool rv, int r,
+// row of len values, V (8 or 16) consecutive values per thread (v, starting at k0 = V t); writes the
+// centered fp16 codes [kp] (zero past len), the unit parameters and the code sum of the row (eq. 2).
+template <int G, int V = 8>
+__device__ __forceinline__ void quantize_row_group(const float (&v)[V], int len, int kp, int t, int rl, bool rv, int r,
                                                    __half *__restrict__ dst, qnn_qparams *__restrict__ prm,
                                                    int32_t *__restrict__ rsum, int *status, float *s_mn, float *s_mx,
                                                    int *s_n) {
     constexpr int W = G > 32 ? G / 32 : 1;  // warps per row
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int k0 = 8 * t;
+    const int k0 = V * t;
     float mn = FLT_MAX, mx = -FLT_MAX;
     int bad = 0;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
+    for (int e = 0; e < V; ++e) {
         if (rv && k0 + e < len) {
             bad |= !isfinite(v[e]);
             mn = fminf(mn, v[e]);
@@ -130,9 +130,9 @@ __device__ __forceinline__ void quantize_row_group(const float (&v)[8], int len,
     }
     const qnn_qparams p = params_from_range(mn, mx);
     int sum = 0;
-    __align__(16) __half h[8];
+    __align__(16) __half h[V];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
+    for (int e = 0; e < V; ++e) {
         int c = 128;  // centered zero past len
         if (k0 + e < len) {
             c = (int)quant_code(v[e], p.Q, p.z);
@@ -140,7 +140,10 @@ __device__ __forceinline__ void quantize_row_group(const float (&v)[8], int len,
         }
         h[e] = __int2half_rn(c - 128);
     }
-    if (rv && k0 < kp) *reinterpret_cast<uint4 *>(dst + (int64_t)r * kp + k0) = *reinterpret_cast<const uint4 *>(h);
+#pragma unroll
+    for (int e8 = 0; e8 < V; e8 += 8)
+        if (rv && k0 + e8 < kp)
+            *reinterpret_cast<uint4 *>(dst + (int64_t)r * kp + k0 + e8) = *reinterpret_cast<const uint4 *>(h + e8);
 #pragma unroll
     for (int o = (G < 32 ? G : 32) / 2; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
     if constexpr (W > 1) {
@@ -157,8 +160,8 @@ __device__ __forceinline__ void quantize_row_group(const float (&v)[8], int len,
 }
 
 // Rows of fp32 values (row r at src + r*ld) -> centered fp16 codes for kp <= 2048: a group of G
-// threads (8 G >= kp) per row, each holding 8 consecutive values, so the row is read once.
-template <int G>
+// threads (V G >= kp) per row, each holding V consecutive values, so the row is read once.
+template <int G, int V = 8>
 __global__ void __launch_bounds__(256)
     quantize_rows_f16_kernel(const float *__restrict__ src, int64_t ld, int rows, int len, int kp,
                              __half *__restrict__ dst, qnn_qparams *__restrict__ prm, int32_t *__restrict__ rsum,
@@ -171,13 +174,21 @@ __global__ void __launch_bounds__(256)
     const int t = threadIdx.x % G, rl = threadIdx.x / G;
     const int r = blockIdx.x * RPB + rl;
     const bool rv = r < rows;
-    const int k0 = 8 * t;
+    const int k0 = V * t;
     const float *xr = src + (int64_t)(rv ? r : 0) * ld;
-    float v[8];
+    float v[V];
+    if (rv && k0 + V <= len && (ld % 4) == 0 && (reinterpret_cast<uintptr_t>(src) & 15) == 0) {
 #pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = (rv && k0 + e < len) ? xr[k0 + e] : 0.0f;
+        for (int e4 = 0; e4 < V; e4 += 4) {
+            const float4 a = *reinterpret_cast<const float4 *>(xr + k0 + e4);
+            v[e4] = a.x, v[e4 + 1] = a.y, v[e4 + 2] = a.z, v[e4 + 3] = a.w;
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < V; ++e) v[e] = (rv && k0 + e < len) ? xr[k0 + e] : 0.0f;
+    }
     const int ro = tm_T > 0 ? (r % tm_T) * tm_B + r / tm_T : r;  // output row (see launch_quantize_rows_f16)
-    quantize_row_group<G>(v, len, kp, t, rl, rv, ro, dst, prm, rsum, status, s_mn, s_mx, s_n);
+    quantize_row_group<G, V>(v, len, kp, t, rl, rv, ro, dst, prm, rsum, status, s_mn, s_mx, s_n);
 }
 
 // Arguments of the projection's finishing kernel (one recurrent step of an LSTMP layer).
@@ -344,7 +355,10 @@ qnn_status launch_quantize_rows_f16(const float *src, int64_t ld, int64_t rows, 
         case 32: cfg.gridDim = grid_for(8); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<32>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
         case 64: cfg.gridDim = grid_for(4); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<64>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
         case 128: cfg.gridDim = grid_for(2); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
-        case 256: cfg.gridDim = grid_for(1); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<256>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
+        case 256:  // 128 threads x 16 values a row: two rows a block
+            cfg.gridDim = grid_for(2);
+            e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128, 16>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB);
+            break;
         default:
             cfg.gridDim = grid_for(kQuantRowsPerBlock);
             e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_warp_kernel, src, ld, ir, il, ik, dst, prm, rsum, status, tmT,
