@@ -452,7 +452,7 @@ def run_ours(args, wl, rank, world, local):
         gbs = alg / avg_s / 1e9
         flops = 2.0 * wl.batch * 4 * wl.hidden * (wl.R + (gates_input_width(wl) if gates_fused(wl) else 0))
         tfs = flops / avg_s / 1e12
-        traffic = traffic_record(kname, wl.name, ["qgemm_tc.cu", "qnn_device.cuh"])
+        traffic = traffic_record(kname, wl.name, ["qgemm_tc.cu", "qnn_device.cuh", "tc_ptx.cuh"])
         if gates_fused(wl):
             # the kernel runs inside a long step (thousands of launches per pass): the sustained peak
             tpk = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
