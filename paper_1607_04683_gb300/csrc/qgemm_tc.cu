@@ -51,6 +51,7 @@ enum Epilogue { kEpiLinear = 0, kEpiLstm = 1, kEpiRow = 2, kEpiPartial = 4, kEpi
 struct ColConst {  // per-output-column constants of kEpiRow, staged in shared memory per tile
     int cs, zw;
     float Qw, bias;
+    float csf;  // cs as an exact fp32 value (cs <= 255 K < 2^24)
 };
 struct ColUnit {  // and the weight unit of each column (-1 past N)
     int unit;
@@ -198,8 +199,33 @@ __device__ __forceinline__ void tile_origin(int64_t tile, int64_t tiles_m, int t
     n0 = (local / rows) * bn;
 }
 
-// Recovered outputs of one 16-column block of one row that lies in one weight unit (the row
-// terms rt, za + 128 and the divisor Qa Qw hoisted), stored as four 16-byte vectors.
+// Recovered outputs of one 16-column block of one row that lies in one weight unit, in fp32: the
+// tensor-core sum P is an exact integer and, when |rt| + |za + 128| 255 K < 2^24, so is the offset
+// term rt + (za + 128) cs, formed by one fused multiply-add without rounding; the one rounded add
+// P + (offset term) then equals the rounded integer sum S of eq. (1), and S / (Qa Qw) comes from the
+// divisor's correctly rounded reciprocal (div_by_recip2: the IEEE quotient while the divisor lies
+// within 2^-60 .. 2^60). Two columns at a time with paired fp32 instructions; four 16-byte stores.
+template <bool BIAS>
+__device__ __forceinline__ void row_block_f32(const uint32_t (&r)[16], const ColConst *cc, float rtf, float za128f,
+                                              float den, float rden, float *yr) {
+#pragma unroll
+    for (int v4 = 0; v4 < 4; ++v4) {
+        float y[4];
+#pragma unroll
+        for (int e2 = 0; e2 < 4; e2 += 2) {
+            const int i = 4 * v4 + e2;
+            const float2 off = ffma2_rn(f2(za128f), make_float2(cc[i].csf, cc[i + 1].csf), f2(rtf));
+            const float2 S = fadd2_rn(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), off);
+            float2 q = div_by_recip2(S, den, rden);
+            if (BIAS) q = fadd2_rn(q, make_float2(cc[i].bias, cc[i + 1].bias));
+            y[e2] = q.x, y[e2 + 1] = q.y;
+        }
+        *reinterpret_cast<float4 *>(yr + 4 * v4) = make_float4(y[0], y[1], y[2], y[3]);
+    }
+}
+
+// The same block with the integer sum formed in 64 bits and an IEEE divide (rows outside the
+// bounds above).
 template <bool BIAS>
 __device__ __forceinline__ void row_block_fast(const uint32_t (&r)[16], const ColConst *cc, long long rt, int za128,
                                                float den, float *yr) {
@@ -562,12 +588,13 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             ColUnit *cu = sunit + (it & 1) * BN;
             for (int c = ew * 32 + lane; c < BN; c += 32 * TL::EPI_WARPS) {
                 const int64_t n = n0 + c;
-                ColConst v{0, 0, 1.0f, 0.0f};
+                ColConst v{0, 0, 1.0f, 0.0f, 0.0f};
                 int unit = -1;
                 if (n < args.N) {
                     unit = (int)(n / args.rows_per_block);
                     const qnn_qparams qw = args.pw[unit];
                     v.cs = args.csW[n];
+                    v.csf = (float)v.cs;
                     v.zw = qw.z;
                     v.Qw = qw.Q;
                     v.bias = args.bias ? args.bias[n] : 0.0f;
@@ -662,12 +689,13 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
             ColUnit *cu = sunit + (gc & 1) * BN;
             for (int c = ew * 32 + lane; c < BN; c += 32 * TL::EPI_WARPS) {
                 const int64_t n = n0 + c;
-                ColConst v{0, 0, 1.0f, 0.0f};
+                ColConst v{0, 0, 1.0f, 0.0f, 0.0f};
                 int unit = -1;
                 if (n < args.N) {
                     unit = (int)(n / args.rows_per_block);
                     const qnn_qparams qw = args.pw[unit];
                     v.cs = args.csW[n];
+                    v.csf = (float)v.cs;
                     v.zw = qw.z;
                     v.Qw = qw.Q;
                     v.bias = args.bias ? args.bias[n] : 0.0f;
@@ -713,10 +741,18 @@ __global__ void __launch_bounds__((Tile<BN, EPI>::THREADS)) __maxnreg__((Tile<BN
                 float *yr = args.Y ? args.Y + m * args.ldy + nb : nullptr;
                 const bool full = vec && nb + 16 <= args.N;
                 if (one_unit && full && !args.acc_out) {  // the usual block: no per-element branches
-                    if (args.bias)
+                    if (den >= 0x1p-60f && den <= 0x1p60f &&
+                        llabs(rt) + (long long)abs(za128) * 255 * K < (1LL << 24)) {
+                        const float rden = __frcp_rn(den);
+                        if (args.bias)
+                            row_block_f32<true>(r, cc + c0, (float)rt, (float)za128, den, rden, yr);
+                        else
+                            row_block_f32<false>(r, cc + c0, (float)rt, (float)za128, den, rden, yr);
+                    } else if (args.bias) {
                         row_block_fast<true>(r, cc + c0, rt, za128, den, yr);
-                    else
+                    } else {
                         row_block_fast<false>(r, cc + c0, rt, za128, den, yr);
+                    }
                     continue;
                 }
 #pragma unroll
