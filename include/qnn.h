@@ -58,7 +58,9 @@ typedef enum { QNN_OUT_NONE = 0, QNN_OUT_QUANT = 1, QNN_OUT_FLOAT = 2 } qnn_outp
  * eq. (2). Code of v: clamp(round(Q v) - z, 0, 255). Recovery (eq. 3): (code + z) / Q.
  * Readings where the paper is silent: Q is raised by single ulps until the range maximum reaches
  * code 255; codes are clamped to [0, 255]; a unit with vmax == vmin, or with |Q vmin| or
- * |Q vmax| >= 2^22, uses Q = 255 / max(|vmin|, |vmax|) (Q = 1 if all values are 0). */
+ * |Q vmax| >= 2^22, uses Q = 255 / max(|vmin|, |vmax|) (Q = 1 if all values are 0). That rule
+ * takes the place of a range error: no call fails on a unit without a usable range (an all-zero
+ * initial state, a constant row); only non-finite values are errors (QNN_ERR_NONFINITE). */
 typedef struct {
     float vmin;
     float vmax;
