@@ -366,8 +366,14 @@ def run_ours(args, wl, rank, world, local):
     step_ms = [a.elapsed_time(b) for a, b in evs]
     # Per-kernel durations: the same K steps again with CUDA events around every launch (events
     # between back-to-back launches lengthen the step, so the step time above is taken without).
+    # The layers of a multi-layer LSTMP run as a wavefront on one stream each, where a kernel's
+    # events would also span other layers' kernels running beside it; the instrumented replay runs
+    # the layers one after the other (QNN_TC_WAVE=0: the same kernels on the same data), so each
+    # launch's events time that kernel alone.
     qnn.profile_read()
     qnn.profile_enable(True)
+    wave_env = os.environ.get("QNN_TC_WAVE")
+    os.environ["QNN_TC_WAVE"] = "0"
     prof_ms = 0.0  # the instrumented steps' own duration: a kernel's share of the step is taken from it
     for i in range(args.steps):
         flush.zero_()
@@ -379,6 +385,10 @@ def run_ours(args, wl, rank, world, local):
         prof_ms += a.elapsed_time(b)
     torch.cuda.synchronize()
     qnn.profile_enable(False)
+    if wave_env is None:
+        del os.environ["QNN_TC_WAVE"]
+    else:
+        os.environ["QNN_TC_WAVE"] = wave_env
     prof = qnn.profile_read()
     total_ms = max_over_ranks(sum(step_ms), world, dev)
     frames_per_step = wl.batch * wl.frames
@@ -478,6 +488,10 @@ def run_ours(args, wl, rank, world, local):
         "e2e": {"value": e2e_value, "unit": "frames/s", "h2d_bytes_per_step": int(x.nbytes),
                 "d2h_bytes_per_step": int(wl.batch * wl.frames * ycols * 4)},
         "clocks": clk.summary(),
+        # how the library ran the layers in the timed steps (the kernels' own durations above come
+        # from a replay with the layers in sequence)
+        "layer_schedule": ("wavefront: one stream per layer" if wl.proj > 0 and wl.num_layers >= 2 and
+                           wl.batch >= 64 and os.environ.get("QNN_TC_WAVE") != "0" else "sequential"),
     }
     if world == 1 and not args.no_extras:
         line["int8_gemm"] = gemm_metric(qnn, torch, peaks, peak_kind, flush, max(5, args.steps))

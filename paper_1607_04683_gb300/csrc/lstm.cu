@@ -575,6 +575,8 @@ extern "C" void qnn_lstm_model_destroy(qnn_lstm_model *m) {
     cudaFree(m->sws);
     cudaFree(m->tcw);
     cudaFree(m->fws);
+    for (cudaStream_t w : m->wave_st) cudaStreamDestroy(w);
+    for (cudaEvent_t e : m->wave_ev) cudaEventDestroy(e);
     cudaSetDevice(prev);
     delete m;
 }
@@ -838,6 +840,9 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     if (use_tc) QNN_TRY(tc_prepare(m));
     // the tensor-core recurrence computes each step's input product in its gate kernel (no px)
     const bool fused = use_tc && tc_input_fused(m);
+    // layers as a wavefront on one stream each (every layer's recurrence state its own; the layer
+    // outputs are kept whole only where they are read: the top layer, and every layer with h_all)
+    const bool wave = fused && tc_stack_supported(m) && (!h_all || ha_dev);
     const FwdPlan plan = plan_recurrent(m, B);
 
     // workspace layout
@@ -866,6 +871,22 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     const size_t o_lg = acct(C > 0 ? rows * C * 4 : 0);
     const size_t o_y = (y_dev || y_map) ? 0 : acct(rows * ycols * 4);
     const size_t o_tc = use_tc ? acct(tc_work_bytes(m, B)) : 0;
+    // wavefront: for layers 1 .. L - 1 (index l - 1) the input codes the previous layer writes and
+    // the recurrence state; for every layer l (index l) the step's output when the layer's outputs
+    // are not kept
+    const int64_t kxr = round_up(R, 64);
+    std::vector<size_t> o_wx16, o_wprm, o_wrs, o_wc, o_wm, o_wtc, o_wout;
+    if (wave) {
+        for (int64_t l = 1; l < L; ++l) {
+            o_wx16.push_back(acct(rows * kxr * 2));
+            o_wprm.push_back(acct(rows * sizeof(qnn_qparams)));
+            o_wrs.push_back(acct(rows * 4));
+            o_wc.push_back(acct(B * H * 4));
+            o_wm.push_back(acct(B * H * 4));
+            o_wtc.push_back(acct(tc_work_bytes(m, B)));
+        }
+        for (int64_t l = 0; l < L; ++l) o_wout.push_back(acct(B * R * 4));
+    }
     if (need > m->ws_bytes) {
         if (m->ws) {
             QNN_CUDA_TRY(cudaStreamSynchronize(st));
@@ -911,7 +932,74 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
 
     const float *in = xd;
     int64_t kin = I;
-    for (int64_t l = 0; l < L; ++l) {
+    if (wave) {
+        // streams of layers 1 .. L - 1 and the events: L - 1 layer edges, a fork, L - 1 joins
+        if ((int64_t)m->wave_st.size() != L - 1) {
+            for (cudaStream_t w : m->wave_st) cudaStreamDestroy(w);
+            for (cudaEvent_t e : m->wave_ev) cudaEventDestroy(e);
+            m->wave_st.assign((size_t)(L - 1), nullptr);
+            m->wave_ev.assign((size_t)(2 * L - 1), nullptr);
+            for (auto &w : m->wave_st) QNN_CUDA_TRY(cudaStreamCreateWithFlags(&w, cudaStreamNonBlocking));
+            for (auto &e : m->wave_ev) QNN_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+        }
+        std::vector<cudaStream_t> streams((size_t)L);
+        streams[0] = st;
+        for (int64_t l = 1; l < L; ++l) streams[(size_t)l] = m->wave_st[(size_t)(l - 1)];
+        const cudaEvent_t *edges = m->wave_ev.data(), fork = m->wave_ev[(size_t)(L - 1)];
+        const cudaEvent_t *joins = m->wave_ev.data() + L;
+        std::vector<TcStackLayer> sl((size_t)L);
+        std::vector<const float *> hsrc((size_t)L);
+        std::vector<int64_t> hsrc_ld((size_t)L);
+        for (int64_t l = 0; l < L; ++l) {
+            TcStackLayer &y = sl[(size_t)l];
+            const bool keep = ha_dev || l == L - 1;  // outputs kept whole
+            y.h0 = h0 + l * B * R;
+            y.cbuf = l == 0 ? cbuf : reinterpret_cast<float *>(ws + o_wc[(size_t)(l - 1)]);
+            y.mbuf = l == 0 ? mbuf : reinterpret_cast<float *>(ws + o_wm[(size_t)(l - 1)]);
+            y.work = l == 0 ? ws + o_tc : ws + o_wtc[(size_t)(l - 1)];
+            if (keep) {
+                y.out = ha_dev ? h_all + l * rows * R : seq[0];
+                y.out_t = R, y.out_b = T * R;
+            } else {
+                y.out = reinterpret_cast<float *>(ws + o_wout[(size_t)l]);
+                y.out_t = 0, y.out_b = R;
+            }
+            hsrc[(size_t)l] = y.out + (T - 1) * y.out_t;
+            hsrc_ld[(size_t)l] = y.out_b;
+            if (l == 0) {
+                y.fx.in = xd, y.fx.kin = I, y.fx.x16 = reinterpret_cast<__half *>(ws + o_x16), y.fx.prm = prm;
+                y.fx.rs = rs;
+            } else {
+                y.fx.in = nullptr, y.fx.kin = R;
+                y.fx.x16 = reinterpret_cast<__half *>(ws + o_wx16[(size_t)(l - 1)]);
+                y.fx.prm = reinterpret_cast<qnn_qparams *>(ws + o_wprm[(size_t)(l - 1)]);
+                y.fx.rs = reinterpret_cast<int32_t *>(ws + o_wrs[(size_t)(l - 1)]);
+            }
+            if (c_state)
+                QNN_CUDA_TRY(cudaMemcpyAsync(y.cbuf, c_state + l * B * H, B * H * 4, cudaMemcpyDefault, st));
+            else
+                QNN_CUDA_TRY(cudaMemsetAsync(y.cbuf, 0, B * H * 4, st));
+        }
+        // the layer streams follow everything queued so far on the caller's stream
+        QNN_CUDA_TRY(cudaEventRecord(fork, st));
+        for (int64_t l = 1; l < L; ++l) QNN_CUDA_TRY(cudaStreamWaitEvent(streams[(size_t)l], fork, 0));
+        QNN_TRY(tc_stack_recurrence(m, sl.data(), B, T, streams.data(), edges));
+        // ... and the caller's stream follows every layer
+        for (int64_t l = 1; l < L; ++l) {
+            QNN_CUDA_TRY(cudaEventRecord(joins[l - 1], streams[(size_t)l]));
+            QNN_CUDA_TRY(cudaStreamWaitEvent(st, joins[l - 1], 0));
+        }
+        for (int64_t l = 0; l < L; ++l) {
+            if (h_state)  // final h of the layer: its output at the last frame
+                QNN_CUDA_TRY(cudaMemcpy2DAsync(h_state + l * B * R, R * 4, hsrc[(size_t)l], hsrc_ld[(size_t)l] * 4,
+                                               R * 4, B, cudaMemcpyDefault, st));
+            if (c_state)
+                QNN_CUDA_TRY(cudaMemcpyAsync(c_state + l * B * H, sl[(size_t)l].cbuf, B * H * 4, cudaMemcpyDefault, st));
+        }
+        in = sl[(size_t)(L - 1)].out;
+        kin = R;
+    }
+    for (int64_t l = 0; l < L && !wave; ++l) {
         const LayerDev &ly = m->layers[l];
         if (!fused) {
             // 1. quantize every frame of the layer input (one unit per row)

@@ -68,6 +68,9 @@ struct qnn_lstm_model {
     uint32_t epoch = 0;
     // fp16 weight copies of the tensor-core recurrence (made on first use)
     void *tcw = nullptr;
+    // streams of layers 1 .. L - 1 and events of the layer wavefront (made on first use)
+    std::vector<cudaStream_t> wave_st;
+    std::vector<cudaEvent_t> wave_ev;
     std::vector<qnn::TcLayer> tc_layers;
     // host mirror of the unit parameters (filled at creation)
     std::vector<qnn_qparams> host_params;
@@ -123,6 +126,25 @@ size_t tc_work_bytes(const qnn_lstm_model *m, int64_t B);
 qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
                                float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st,
                                const TcFusedInput *fx = nullptr);
+// The tensor-core recurrences of all layers as a wavefront across layers (LSTMP with the split
+// projection and the fused input product, two or more layers; QNN_TC_WAVE=0 turns it off): layer l
+// runs on streams[l], its step t after step t of layer l - 1 (edges[l - 1], recorded on
+// streams[l - 1]); each layer's finishing kernel also writes the next layer's input codes of that
+// step (fx.x16 / prm / rs of layer l + 1, time-major [B T][round_up(R, 64)]), so consecutive layers
+// overlap. Layer 0's input is quantized at its start from fx.in. Per layer: h0 [B][R], cell state
+// cbuf [B][H] in/out, mbuf [B][H], workspace of tc_work_bytes, outputs: row b of step t at
+// out + t out_t + b out_b. The streams must already follow everything the buffers depend on.
+struct TcStackLayer {
+    const float *h0 = nullptr;
+    float *cbuf = nullptr, *mbuf = nullptr;
+    void *work = nullptr;
+    float *out = nullptr;
+    int64_t out_t = 0, out_b = 0;
+    TcFusedInput fx;
+};
+bool tc_stack_supported(const qnn_lstm_model *m);
+qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *layers, int64_t B, int64_t T,
+                               const cudaStream_t *streams, const cudaEvent_t *edges);
 // Whether every layer's input product can be fused into its gate kernel (input width <= 1024; the
 // environment variable QNN_TC_FUSE_X=0 turns it off), and the workspace for the layer input's codes.
 bool tc_input_fused(const qnn_lstm_model *m);

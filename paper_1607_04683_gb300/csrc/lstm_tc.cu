@@ -16,6 +16,7 @@
 #include <cfloat>
 #include <cstdlib>
 #include <cstring>
+#include <vector>
 
 #include "lstm_model.h"
 #include "qnn_device.cuh"
@@ -82,12 +83,14 @@ __global__ void __launch_bounds__(32 * kQuantRowsPerBlock)
 
 // Row-group quantizer shared by the kernels below: a group of G threads (a power of two) holds a
 // row of len values, V (8 or 16) consecutive values per thread (v, starting at k0 = V t); writes the
-// centered fp16 codes [kp] (zero past len), the unit parameters and the code sum of the row (eq. 2).
+// centered fp16 codes [kp] (zero past len), the unit parameters and the code sum of the row (eq. 2),
+// and the same again to dst2, prm2, rsum2 (row r2) when dst2 is given.
 template <int G, int V = 8>
 __device__ __forceinline__ void quantize_row_group(const float (&v)[V], int len, int kp, int t, int rl, bool rv, int r,
                                                    __half *__restrict__ dst, qnn_qparams *__restrict__ prm,
                                                    int32_t *__restrict__ rsum, int *status, float *s_mn, float *s_mx,
-                                                   int *s_n) {
+                                                   int *s_n, __half *dst2 = nullptr, qnn_qparams *prm2 = nullptr,
+                                                   int32_t *rsum2 = nullptr, int r2 = 0) {
     constexpr int W = G > 32 ? G / 32 : 1;  // warps per row
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int k0 = V * t;
@@ -142,8 +145,11 @@ __device__ __forceinline__ void quantize_row_group(const float (&v)[V], int len,
     }
 #pragma unroll
     for (int e8 = 0; e8 < V; e8 += 8)
-        if (rv && k0 + e8 < kp)
+        if (rv && k0 + e8 < kp) {
             *reinterpret_cast<uint4 *>(dst + (int64_t)r * kp + k0 + e8) = *reinterpret_cast<const uint4 *>(h + e8);
+            if (dst2)
+                *reinterpret_cast<uint4 *>(dst2 + (int64_t)r2 * kp + k0 + e8) = *reinterpret_cast<const uint4 *>(h + e8);
+        }
 #pragma unroll
     for (int o = (G < 32 ? G : 32) / 2; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
     if constexpr (W > 1) {
@@ -156,6 +162,10 @@ __device__ __forceinline__ void quantize_row_group(const float (&v)[V], int len,
     if (t == 0 && rv) {
         prm[r] = p;
         rsum[r] = sum;
+        if (dst2) {
+            prm2[r2] = p;
+            rsum2[r2] = sum;
+        }
     }
 }
 
@@ -211,6 +221,11 @@ struct FinishArgs {
     qnn_qparams *prm;
     int32_t *rsum;
     int *status;
+    // nullable: the same codes, params and sums again as the next layer's input of this step
+    // ([B][kp] rows of the next layer's time-major input codes)
+    __half *dst2;
+    qnn_qparams *prm2;
+    int32_t *rsum2;
 };
 
 // Adds the split-K slices, applies eq. (1)'s offsets and eq. (3)'s recovery (the same integer
@@ -298,7 +313,8 @@ __global__ void __launch_bounds__(256) proj_finish_kernel(const FinishArgs a) {
         }
     }
     if (!a.quantize) return;
-    quantize_row_group<G>(v, a.P, a.kp, t, rl, rv, r, a.dst, a.prm, a.rsum, a.status, s_mn, s_mx, s_n);
+    quantize_row_group<G>(v, a.P, a.kp, t, rl, rv, r, a.dst, a.prm, a.rsum, a.status, s_mn, s_mx, s_n, a.dst2, a.prm2,
+                          a.rsum2, r);
 }
 
 // The four Wh gate matrices (u8 codes, row g*H + j, ld bytes) -> centered fp16 rows in 8-cell
@@ -523,31 +539,59 @@ size_t tc_xwork_bytes(const qnn_lstm_model *m, int64_t rows) {
     return (size_t)round_up(rows * kx * 2, 256);
 }
 
-qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
-                               float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st,
-                               const TcFusedInput *fx) {
-    const LayerDev &ly = m->layers[l];
-    const TcLayer &tl = m->tc_layers[l];
-    const int64_t H = m->H, R = m->R, P = m->P, H8 = round_up(H, 8);
+namespace {
+// One layer's tensor-core recurrence, launched a step at a time: tc_layer_begin, then tc_layer_step
+// for t = 0 .. T - 1 in order, all on the run's stream.
+struct TcLayerRun {
+    const qnn_lstm_model *m = nullptr;
+    int64_t l = 0, B = 0, T = 0;
+    const float *px = nullptr;  // batched input products (unfused input), row b T + t
+    float *cbuf = nullptr, *mbuf = nullptr;
+    float *out = nullptr;       // row b of step t's output at out + t * out_t + b * out_b
+    int64_t out_t = 0, out_b = 0;
+    // nullable: the next layer's time-major input codes, unit params and code sums, which the
+    // finishing kernel writes for each step (split projection only)
+    __half *nx16 = nullptr;
+    qnn_qparams *nprm = nullptr;
+    int32_t *nrs = nullptr;
+    cudaStream_t st = nullptr;
+    // set by tc_layer_begin
+    TcOperands gates, proj;
+    bool split_proj = false, fused = false;
+    int splits = 0;
+    TcLstmInput xin;
+    const __half *x16 = nullptr;
+    const qnn_qparams *xprm = nullptr;
+    const int32_t *xrs = nullptr;
+    __half *a16 = nullptr, *m16 = nullptr;
+    qnn_qparams *prm = nullptr, *prm_m = nullptr;
+    int32_t *rs = nullptr, *rs_m = nullptr, *part = nullptr;
+    int *status = nullptr;
+};
+}  // namespace
+
+qnn_status tc_layer_begin(TcLayerRun &s, const float *h0, void *work, const TcFusedInput *fx, bool quantize_input) {
+    const qnn_lstm_model *m = s.m;
+    const LayerDev &ly = m->layers[s.l];
+    const TcLayer &tl = m->tc_layers[s.l];
+    const int64_t B = s.B, T = s.T, H = m->H, R = m->R, P = m->P, H8 = round_up(H, 8);
     const int64_t kh = tl.kh, kpj = tl.kp;
     char *w = reinterpret_cast<char *>(work);
-    __half *a16 = reinterpret_cast<__half *>(w);
+    s.a16 = reinterpret_cast<__half *>(w);
     w += round_up(B * kh * 2, 256);
-    __half *m16 = reinterpret_cast<__half *>(w);
+    s.m16 = reinterpret_cast<__half *>(w);
     w += round_up(B * kpj * 2, 256);
-    qnn_qparams *prm = reinterpret_cast<qnn_qparams *>(w);
+    s.prm = reinterpret_cast<qnn_qparams *>(w);
     w += round_up(B * (int64_t)sizeof(qnn_qparams), 256);
-    qnn_qparams *prm_m = reinterpret_cast<qnn_qparams *>(w);
+    s.prm_m = reinterpret_cast<qnn_qparams *>(w);
     w += round_up(B * (int64_t)sizeof(qnn_qparams), 256);
-    int32_t *rs = reinterpret_cast<int32_t *>(w);
+    s.rs = reinterpret_cast<int32_t *>(w);
     w += round_up(B * 4, 256);
-    int32_t *rs_m = reinterpret_cast<int32_t *>(w);
+    s.rs_m = reinterpret_cast<int32_t *>(w);
     w += round_up(B * 4, 256);
-    int32_t *part = reinterpret_cast<int32_t *>(w);
+    s.part = reinterpret_cast<int32_t *>(w);
 
-    int *status = nullptr;
-    QNN_TRY(status_word(&status));
-    TcOperands gates, proj;
+    QNN_TRY(status_word(&s.status));
     // tile widths, widest first; the fused kernel's 96-column tile (24 warps at 72 registers) spills
     // with the second recovery and measured slower than 64 columns, so it is left out there
     static const int gate_bn[] = {128, 96, 64, 32}, gate_bn_fused[] = {128, 64, 32};
@@ -557,53 +601,112 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
     // wave the tile count that fills the SMs best decides.
     int bn_gates = fx ? tc_choose_bn(B, 4 * H8, gate_bn_fused, 3) : tc_choose_bn(B, 4 * H8, gate_bn, 4);
     if (fx && !std::getenv("QNN_TC_BN") && ((B + 127) / 128) * ((4 * H8 + 127) / 128) >= sm_count()) bn_gates = 128;
-    QNN_TRY(tc_operands(&gates, a16, B, tl.wh16, 4 * H8, kh, bn_gates));
+    QNN_TRY(tc_operands(&s.gates, s.a16, B, tl.wh16, 4 * H8, kh, bn_gates));
     // the projection after the m_t quantizer: split-K partial sums finished (offsets, recovery, next
     // step's quantization) by one row kernel; or one tcgen05 product with its own epilogue per step
-    const bool split_proj = P > 0 && split_proj_enabled(P);
-    int splits = 0;
+    s.split_proj = P > 0 && split_proj_enabled(P);
+    s.splits = 0;
     if (P > 0) {
-        QNN_TRY(tc_operands(&proj, m16, B, tl.wp16, P, kpj, split_proj ? 128 : tc_pick_bn(B, P, kpj)));
-        if (split_proj) splits = tc_partial_splits(proj, (int)max_proj_splits(m));
+        QNN_TRY(tc_operands(&s.proj, s.m16, B, tl.wp16, P, kpj, s.split_proj ? 128 : tc_pick_bn(B, P, kpj)));
+        if (s.split_proj) s.splits = tc_partial_splits(s.proj, (int)max_proj_splits(m));
     }
+    if (s.nx16 && !s.split_proj) return QNN_ERR_INVALID_ARG;  // only the finishing kernel writes them
     // the steps' kernels chain by programmatic dependent launches (see tc_gemm.h); the first one of
     // the layer follows ordinary stream order
-    gates.pdl = proj.pdl = pdl_enabled();
-    // fused input product: every frame of the layer input quantized once (rows b T + t, centered fp16)
-    TcLstmInput xin;
+    s.gates.pdl = s.proj.pdl = pdl_enabled();
+    // fused input product: the layer input as centered fp16 codes, time-major (row t B + b), so a
+    // step's x_t rows of all sequences are one contiguous block; quantized here at once, or written
+    // step by step by the previous layer (quantize_input false)
+    s.fused = fx != nullptr;
     if (fx) {
         if (!tl.wx16 || tl.kx != round_up(fx->kin, 64)) return QNN_ERR_INVALID_ARG;
-        // codes time-major (row t B + b): a step's x_t rows of all sequences are one contiguous block
-        QNN_TRY(launch_quantize_rows_f16(fx->in, fx->kin, B * T, (int)fx->kin, (int)tl.kx, fx->x16, fx->prm, fx->rs,
-                                         status, false, st, T, B));
-        xin.x_pitch = tl.kx, xin.kx = tl.kx, xin.K_x = (int)fx->kin, xin.stride = 1;
-        xin.wx16 = tl.wx16, xin.pw4 = ly.wx.params, xin.cs = ly.wx.sums, xin.bias = ly.bias, xin.colc = tl.colc;
+        if (quantize_input)
+            QNN_TRY(launch_quantize_rows_f16(fx->in, fx->kin, B * T, (int)fx->kin, (int)tl.kx, fx->x16, fx->prm,
+                                             fx->rs, s.status, false, s.st, T, B));
+        s.x16 = fx->x16, s.xprm = fx->prm, s.xrs = fx->rs;
+        s.xin.x_pitch = tl.kx, s.xin.kx = tl.kx, s.xin.K_x = (int)fx->kin, s.xin.stride = 1;
+        s.xin.wx16 = tl.wx16, s.xin.pw4 = ly.wx.params, s.xin.cs = ly.wx.sums, s.xin.bias = ly.bias;
+        s.xin.colc = tl.colc;
     }
-    QNN_TRY(launch_quantize_rows_f16(h0, R, B, R, kh, a16, prm, rs, status, false, st));
-    for (int64_t t = 0; t < T; ++t) {
-        if (t > 0 && !split_proj)
-            QNN_TRY(launch_quantize_rows_f16(out + (t - 1) * R, T * R, B, R, kh, a16, prm, rs, status, gates.pdl, st));
-        TcLstmOut o{fx ? nullptr : px + t * 4 * H, T * 4 * H, cbuf, P > 0 ? mbuf : out + t * R, P > 0 ? H : T * R,
-                    (int)H, (int)m->S, (int)(H / m->S)};
-        if (fx) {
-            xin.x16 = fx->x16 + t * B * tl.kx, xin.pa = fx->prm + t * B, xin.rs = fx->rs + t * B;
-            QNN_TRY(tc_lstm_gates_x(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, xin, st));
+    QNN_TRY(launch_quantize_rows_f16(h0, R, B, R, kh, s.a16, s.prm, s.rs, s.status, false, s.st));
+    return QNN_OK;
+}
+
+qnn_status tc_layer_step(TcLayerRun &s, int64_t t) {
+    const qnn_lstm_model *m = s.m;
+    const LayerDev &ly = m->layers[s.l];
+    const TcLayer &tl = m->tc_layers[s.l];
+    const int64_t B = s.B, T = s.T, H = m->H, R = m->R, P = m->P;
+    const int64_t kh = tl.kh, kpj = tl.kp;
+    cudaStream_t st = s.st;
+    float *out_t = s.out + t * s.out_t;  // row b of this step's output at out_t + b * out_b
+    if (t > 0 && !s.split_proj)
+        QNN_TRY(launch_quantize_rows_f16(s.out + (t - 1) * s.out_t, s.out_b, B, R, kh, s.a16, s.prm, s.rs, s.status,
+                                         s.gates.pdl, st));
+    TcLstmOut o{s.fused ? nullptr : s.px + t * 4 * H, T * 4 * H, s.cbuf, P > 0 ? s.mbuf : out_t, P > 0 ? H : s.out_b,
+                (int)H, (int)m->S, (int)(H / m->S)};
+    if (s.fused) {
+        TcLstmInput xin = s.xin;
+        xin.x16 = s.x16 + t * B * tl.kx, xin.pa = s.xprm + t * B, xin.rs = s.xrs + t * B;
+        QNN_TRY(tc_lstm_gates_x(s.gates, s.prm, s.rs, R, ly.wh.params, ly.wh.sums, o, xin, st));
+    } else {
+        QNN_TRY(tc_lstm_gates(s.gates, s.prm, s.rs, R, ly.wh.params, ly.wh.sums, o, st));
+    }
+    if (P > 0) {
+        QNN_TRY(launch_quantize_rows_f16(s.mbuf, H, B, H, kpj, s.m16, s.prm_m, s.rs_m, s.status, s.gates.pdl, st));
+        if (s.split_proj) {
+            QNN_TRY(tc_partial(s.proj, s.splits, s.part, P, st));
+            FinishArgs fa{s.part, s.splits, P, s.prm_m, s.rs_m, ly.wp.params, ly.wp.sums, (int)(P / m->S), (int)H,
+                          out_t, s.out_b, (int)B, (int)P, t + 1 < T || s.nx16 != nullptr, (int)kh, s.a16, s.prm,
+                          s.rs, s.status, s.nx16 ? s.nx16 + t * B * kh : nullptr, s.nx16 ? s.nprm + t * B : nullptr,
+                          s.nx16 ? s.nrs + t * B : nullptr};
+            QNN_TRY(launch_proj_finish(fa, s.gates.pdl, st));
         } else {
-            QNN_TRY(tc_lstm_gates(gates, prm, rs, R, ly.wh.params, ly.wh.sums, o, st));
-        }
-        if (P > 0) {
-            QNN_TRY(launch_quantize_rows_f16(mbuf, H, B, H, kpj, m16, prm_m, rs_m, status, gates.pdl, st));
-            if (split_proj) {
-                QNN_TRY(tc_partial(proj, splits, part, P, st));
-                FinishArgs fa{part, splits, P, prm_m, rs_m, ly.wp.params, ly.wp.sums, (int)(P / m->S), (int)H,
-                              out + t * R, T * R, (int)B, (int)P, t + 1 < T, (int)kh, a16, prm, rs, status};
-                QNN_TRY(launch_proj_finish(fa, gates.pdl, st));
-            } else {
-                QNN_TRY(tc_linear(proj, prm_m, 1, rs_m, H, ly.wp.params, P / m->S, ly.wp.sums, nullptr, out + t * R,
-                                  T * R, nullptr, st));
-            }
+            QNN_TRY(tc_linear(s.proj, s.prm_m, 1, s.rs_m, H, ly.wp.params, P / m->S, ly.wp.sums, nullptr, out_t, s.out_b,
+                              nullptr, st));
         }
     }
+    return QNN_OK;
+}
+
+qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
+                               float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st,
+                               const TcFusedInput *fx) {
+    TcLayerRun s;
+    s.m = m, s.l = l, s.B = B, s.T = T, s.px = px, s.cbuf = cbuf, s.mbuf = mbuf;
+    s.out = out, s.out_t = m->R, s.out_b = T * m->R, s.st = st;
+    QNN_TRY(tc_layer_begin(s, h0, work, fx, true));
+    for (int64_t t = 0; t < T; ++t) QNN_TRY(tc_layer_step(s, t));
+    return QNN_OK;
+}
+
+bool tc_stack_supported(const qnn_lstm_model *m) {
+    const char *e = std::getenv("QNN_TC_WAVE");
+    if (e && std::strcmp(e, "0") == 0) return false;
+    return m->L >= 2 && m->P > 0 && split_proj_enabled(m->P) && tc_input_fused(m);
+}
+
+qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *layers, int64_t B, int64_t T,
+                               const cudaStream_t *streams, const cudaEvent_t *edges) {
+    if (!tc_stack_supported(m)) return QNN_ERR_INVALID_ARG;
+    const int64_t L = m->L;
+    std::vector<TcLayerRun> runs((size_t)L);
+    for (int64_t l = 0; l < L; ++l) {
+        TcLayerRun &r = runs[(size_t)l];
+        const TcStackLayer &sl = layers[l];
+        r.m = m, r.l = l, r.B = B, r.T = T, r.cbuf = sl.cbuf, r.mbuf = sl.mbuf;
+        r.out = sl.out, r.out_t = sl.out_t, r.out_b = sl.out_b, r.st = streams[l];
+        if (l + 1 < L) r.nx16 = layers[l + 1].fx.x16, r.nprm = layers[l + 1].fx.prm, r.nrs = layers[l + 1].fx.rs;
+        QNN_TRY(tc_layer_begin(r, sl.h0, sl.work, &sl.fx, l == 0));
+    }
+    // step t of layer l after step t of layer l - 1 (its input codes); each layer's own steps follow
+    // its stream order
+    for (int64_t t = 0; t < T; ++t)
+        for (int64_t l = 0; l < L; ++l) {
+            if (l > 0) QNN_CUDA_TRY(cudaStreamWaitEvent(streams[l], edges[l - 1], 0));
+            QNN_TRY(tc_layer_step(runs[(size_t)l], t));
+            if (l + 1 < L) QNN_CUDA_TRY(cudaEventRecord(edges[l], streams[l]));
+        }
     return QNN_OK;
 }
 

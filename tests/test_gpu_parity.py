@@ -539,6 +539,29 @@ def test_tc_lstmp_projection_forms(qnn, cfg, mode, monkeypatch):
     _compare(got, ref, wl, params)
 
 
+# The LSTMP layers as a wavefront across streams (each layer's finishing kernel writes the next
+# layer's input codes of the step; QNN_TC_WAVE=0 runs the layers one after the other): the oracle's
+# results bit for bit, with carried state in and out, with the layer outputs requested (kept whole
+# for every layer) and without (only the top layer's), and equal to the sequential schedule.
+@pytest.mark.parametrize("want_h_all", [True, False])
+def test_tc_lstmp_layer_wavefront(qnn, want_h_all, monkeypatch):
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    wl = _small(L=3, I=40, H=256, P=128, C=13, B=130, T=5, w=0.1)
+    params, x = wl.make()
+    g = rng(77)
+    h0 = g.uniform(-0.5, 0.5, (wl.num_layers, wl.batch, wl.R)).astype(np.float32)
+    c0 = g.uniform(-1.0, 1.0, (wl.num_layers, wl.batch, wl.hidden)).astype(np.float32)
+    ref = _oracle(wl, params, x, want_h_all=True, h0=h0, c0=c0)
+    outs = {}
+    for wave in ("1", "0"):
+        monkeypatch.setenv("QNN_TC_WAVE", wave)
+        got = _gpu_forward(qnn, wl, params, x, h_all=want_h_all, h0=h0, c0=c0)
+        _compare(got, ref, wl, params)  # (h_all compared when requested)
+        outs[wave] = got
+    for k in ("y", "h", "c", "logits"):
+        assert np.array_equal(outs["1"][k], outs["0"][k]), k
+
+
 # 192 tiles of the gate product on 152 SMs: the 40 tiles of the last wave run as 80 half-width
 # items (N = 64 or 32); the same results with whole tiles (QNN_TC_HALF=0) and from the oracle
 @pytest.mark.parametrize("half", ["1", "0"])
