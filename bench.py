@@ -490,8 +490,8 @@ def run_ours(args, wl, rank, world, local):
         "clocks": clk.summary(),
         # how the library ran the layers in the timed steps (the kernels' own durations above come
         # from a replay with the layers in sequence)
-        "layer_schedule": ("wavefront: one stream per layer" if wl.proj > 0 and wl.num_layers >= 2 and
-                           wl.batch >= 64 and os.environ.get("QNN_TC_WAVE") != "0" else "sequential"),
+        "layer_schedule": ("wavefront: one stream per layer" if wl.num_layers >= 2 and wl.batch >= 64 and
+                           os.environ.get("QNN_TC_WAVE") != "0" else "sequential"),
     }
     if world == 1 and not args.no_extras:
         line["int8_gemm"] = gemm_metric(qnn, torch, peaks, peak_kind, flush, max(5, args.steps))

@@ -126,12 +126,12 @@ size_t tc_work_bytes(const qnn_lstm_model *m, int64_t B);
 qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *px, const float *h0, float *cbuf,
                                float *out, float *mbuf, int64_t B, int64_t T, void *work, cudaStream_t st,
                                const TcFusedInput *fx = nullptr);
-// The tensor-core recurrences of all layers as a wavefront across layers (LSTMP with the split
-// projection and the fused input product, two or more layers; QNN_TC_WAVE=0 turns it off): layer l
-// runs on streams[l], its step t after step t of layer l - 1 (edges[l - 1], recorded on
-// streams[l - 1]); each layer's finishing kernel also writes the next layer's input codes of that
-// step (fx.x16 / prm / rs of layer l + 1, time-major [B T][round_up(R, 64)]), so consecutive layers
-// overlap. Layer 0's input is quantized at its start from fx.in. Per layer: h0 [B][R], cell state
+// The tensor-core recurrences of all layers as a wavefront across layers (fused input product, two
+// or more layers; QNN_TC_WAVE=0 turns it off): layer l runs on streams[l], its step t after step t
+// of layer l - 1 (edges[l - 1], recorded on streams[l - 1]); the kernel that quantizes a step's
+// outputs for the layer's next step (the projection's finishing kernel, else the row quantizer)
+// also writes them as the next layer's input codes of that step (fx.x16 / prm / rs of layer l + 1,
+// time-major [B T][round_up(R, 64)]), so consecutive layers overlap. Layer 0's input is quantized at its start from fx.in. Per layer: h0 [B][R], cell state
 // cbuf [B][H] in/out, mbuf [B][H], workspace of tc_work_bytes, outputs: row b of step t at
 // out + t out_t + b out_b. The streams must already follow everything the buffers depend on.
 struct TcStackLayer {

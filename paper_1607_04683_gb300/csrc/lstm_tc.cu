@@ -169,13 +169,21 @@ __device__ __forceinline__ void quantize_row_group(const float (&v)[V], int len,
     }
 }
 
+// A second destination of a row quantizer's codes, unit params and code sums (nullable dst).
+struct RowCodes {
+    __half *dst;
+    qnn_qparams *prm;
+    int32_t *rsum;
+};
+
 // Rows of fp32 values (row r at src + r*ld) -> centered fp16 codes for kp <= 2048: a group of G
-// threads (V G >= kp) per row, each holding V consecutive values, so the row is read once.
+// threads (V G >= kp) per row, each holding V consecutive values, so the row is read once; the same
+// results also to d2 when d2.dst is given.
 template <int G, int V = 8>
 __global__ void __launch_bounds__(256)
     quantize_rows_f16_kernel(const float *__restrict__ src, int64_t ld, int rows, int len, int kp,
                              __half *__restrict__ dst, qnn_qparams *__restrict__ prm, int32_t *__restrict__ rsum,
-                             int *status, int tm_T, int tm_B) {
+                             int *status, int tm_T, int tm_B, const RowCodes d2) {
     constexpr int RPB = 256 / G;  // rows per block
     __shared__ float s_mn[8], s_mx[8];
     __shared__ int s_n[8];
@@ -198,7 +206,8 @@ __global__ void __launch_bounds__(256)
         for (int e = 0; e < V; ++e) v[e] = (rv && k0 + e < len) ? xr[k0 + e] : 0.0f;
     }
     const int ro = tm_T > 0 ? (r % tm_T) * tm_B + r / tm_T : r;  // output row (see launch_quantize_rows_f16)
-    quantize_row_group<G, V>(v, len, kp, t, rl, rv, ro, dst, prm, rsum, status, s_mn, s_mx, s_n);
+    quantize_row_group<G, V>(v, len, kp, t, rl, rv, ro, dst, prm, rsum, status, s_mn, s_mx, s_n, d2.dst, d2.prm,
+                             d2.rsum, ro);
 }
 
 // Arguments of the projection's finishing kernel (one recurrent step of an LSTMP layer).
@@ -347,13 +356,15 @@ __global__ void sums_to_f32_kernel(const int32_t *__restrict__ in, float *__rest
 // Launches one of the two row quantizers; with `pdl` as a programmatic dependent launch. With
 // tm_T > 0 the source rows are b tm_T + t (sequence-major, tm_B sequences) and row b tm_T + t is
 // written to output row t tm_B + b (time-major), so that one step's rows of all sequences are
-// contiguous for the tensor-core kernel's loads.
+// contiguous for the tensor-core kernel's loads. With d2.dst the same results go there too (kp <=
+// 2048).
 qnn_status launch_quantize_rows_f16(const float *src, int64_t ld, int64_t rows, int64_t len, int64_t kp, __half *dst,
                                     qnn_qparams *prm, int32_t *rsum, int *status, bool pdl, cudaStream_t st,
-                                    int64_t tm_T = 0, int64_t tm_B = 0) {
+                                    int64_t tm_T = 0, int64_t tm_B = 0, RowCodes d2 = RowCodes{nullptr, nullptr, nullptr}) {
     ProfScope prof("quantize_rows_f16", st);
     int g = 8;
     while (g * 8 < kp) g *= 2;
+    if (d2.dst && g > 256) return QNN_ERR_INVALID_ARG;
     cudaLaunchConfig_t cfg = {};
     cfg.blockDim = dim3(256);
     cfg.stream = st;
@@ -366,14 +377,15 @@ qnn_status launch_quantize_rows_f16(const float *src, int64_t ld, int64_t rows, 
     auto grid_for = [&](int rpb) { return dim3((unsigned)((rows + rpb - 1) / rpb)); };
     cudaError_t e;
     switch (g) {
-        case 8: cfg.gridDim = grid_for(32); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<8>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
-        case 16: cfg.gridDim = grid_for(16); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<16>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
-        case 32: cfg.gridDim = grid_for(8); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<32>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
-        case 64: cfg.gridDim = grid_for(4); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<64>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
-        case 128: cfg.gridDim = grid_for(2); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB); break;
+        case 8: cfg.gridDim = grid_for(32); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<8>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB, d2); break;
+        case 16: cfg.gridDim = grid_for(16); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<16>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB, d2); break;
+        case 32: cfg.gridDim = grid_for(8); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<32>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB, d2); break;
+        case 64: cfg.gridDim = grid_for(4); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<64>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB, d2); break;
+        case 128: cfg.gridDim = grid_for(2); e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB, d2); break;
         case 256:  // 128 threads x 16 values a row: two rows a block
             cfg.gridDim = grid_for(2);
-            e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128, 16>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB);
+            e = cudaLaunchKernelEx(&cfg, quantize_rows_f16_kernel<128, 16>, src, ld, ir, il, ik, dst, prm, rsum, status, tmT, tmB,
+                                   d2);
             break;
         default:
             cfg.gridDim = grid_for(kQuantRowsPerBlock);
@@ -610,7 +622,6 @@ qnn_status tc_layer_begin(TcLayerRun &s, const float *h0, void *work, const TcFu
         QNN_TRY(tc_operands(&s.proj, s.m16, B, tl.wp16, P, kpj, s.split_proj ? 128 : tc_pick_bn(B, P, kpj)));
         if (s.split_proj) s.splits = tc_partial_splits(s.proj, (int)max_proj_splits(m));
     }
-    if (s.nx16 && !s.split_proj) return QNN_ERR_INVALID_ARG;  // only the finishing kernel writes them
     // the steps' kernels chain by programmatic dependent launches (see tc_gemm.h); the first one of
     // the layer follows ordinary stream order
     s.gates.pdl = s.proj.pdl = pdl_enabled();
@@ -640,9 +651,9 @@ qnn_status tc_layer_step(TcLayerRun &s, int64_t t) {
     const int64_t kh = tl.kh, kpj = tl.kp;
     cudaStream_t st = s.st;
     float *out_t = s.out + t * s.out_t;  // row b of this step's output at out_t + b * out_b
-    if (t > 0 && !s.split_proj)
-        QNN_TRY(launch_quantize_rows_f16(s.out + (t - 1) * s.out_t, s.out_b, B, R, kh, s.a16, s.prm, s.rs, s.status,
-                                         s.gates.pdl, st));
+    // the next layer's input codes of this step (wavefront), written with this step's own codes
+    const RowCodes next{s.nx16 ? s.nx16 + t * B * kh : nullptr, s.nx16 ? s.nprm + t * B : nullptr,
+                        s.nx16 ? s.nrs + t * B : nullptr};
     TcLstmOut o{s.fused ? nullptr : s.px + t * 4 * H, T * 4 * H, s.cbuf, P > 0 ? s.mbuf : out_t, P > 0 ? H : s.out_b,
                 (int)H, (int)m->S, (int)(H / m->S)};
     if (s.fused) {
@@ -658,14 +669,18 @@ qnn_status tc_layer_step(TcLayerRun &s, int64_t t) {
             QNN_TRY(tc_partial(s.proj, s.splits, s.part, P, st));
             FinishArgs fa{s.part, s.splits, P, s.prm_m, s.rs_m, ly.wp.params, ly.wp.sums, (int)(P / m->S), (int)H,
                           out_t, s.out_b, (int)B, (int)P, t + 1 < T || s.nx16 != nullptr, (int)kh, s.a16, s.prm,
-                          s.rs, s.status, s.nx16 ? s.nx16 + t * B * kh : nullptr, s.nx16 ? s.nprm + t * B : nullptr,
-                          s.nx16 ? s.nrs + t * B : nullptr};
+                          s.rs, s.status, next.dst, next.prm, next.rsum};
             QNN_TRY(launch_proj_finish(fa, s.gates.pdl, st));
         } else {
             QNN_TRY(tc_linear(s.proj, s.prm_m, 1, s.rs_m, H, ly.wp.params, P / m->S, ly.wp.sums, nullptr, out_t, s.out_b,
                               nullptr, st));
         }
     }
+    // without the finishing kernel: this step's outputs quantized as the next step's recurrent input
+    // (and the next layer's input)
+    if (!s.split_proj && (t + 1 < T || s.nx16))
+        QNN_TRY(launch_quantize_rows_f16(out_t, s.out_b, B, R, kh, s.a16, s.prm, s.rs, s.status, s.gates.pdl, st, 0, 0,
+                                         next));
     return QNN_OK;
 }
 
@@ -683,7 +698,7 @@ qnn_status tc_layer_recurrence(const qnn_lstm_model *m, int64_t l, const float *
 bool tc_stack_supported(const qnn_lstm_model *m) {
     const char *e = std::getenv("QNN_TC_WAVE");
     if (e && std::strcmp(e, "0") == 0) return false;
-    return m->L >= 2 && m->P > 0 && split_proj_enabled(m->P) && tc_input_fused(m);
+    return m->L >= 2 && tc_input_fused(m);
 }
 
 qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *layers, int64_t B, int64_t T,

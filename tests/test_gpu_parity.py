@@ -539,14 +539,17 @@ def test_tc_lstmp_projection_forms(qnn, cfg, mode, monkeypatch):
     _compare(got, ref, wl, params)
 
 
-# The LSTMP layers as a wavefront across streams (each layer's finishing kernel writes the next
-# layer's input codes of the step; QNN_TC_WAVE=0 runs the layers one after the other): the oracle's
-# results bit for bit, with carried state in and out, with the layer outputs requested (kept whole
-# for every layer) and without (only the top layer's), and equal to the sequential schedule.
+# The layers as a wavefront across streams (the kernel that quantizes a step's outputs for the
+# layer's next step also writes the next layer's input codes of the step; QNN_TC_WAVE=0 runs the
+# layers one after the other): the oracle's results bit for bit, with carried state in and out,
+# with the layer outputs requested (kept whole for every layer) and without (only the top layer's),
+# and equal to the sequential schedule; LSTMP with the split and the linear projection, and LSTM.
 @pytest.mark.parametrize("want_h_all", [True, False])
-def test_tc_lstmp_layer_wavefront(qnn, want_h_all, monkeypatch):
+@pytest.mark.parametrize("proj", ["split", "linear", "none"])
+def test_tc_layer_wavefront(qnn, want_h_all, proj, monkeypatch):
     monkeypatch.setenv("QNN_LSTM_PATH", "tc")
-    wl = _small(L=3, I=40, H=256, P=128, C=13, B=130, T=5, w=0.1)
+    monkeypatch.setenv("QNN_TC_PROJ", "linear" if proj == "linear" else "split")
+    wl = _small(L=3, I=40, H=256, P=0 if proj == "none" else 128, C=13, B=130, T=5, w=0.1)
     params, x = wl.make()
     g = rng(77)
     h0 = g.uniform(-0.5, 0.5, (wl.num_layers, wl.batch, wl.R)).astype(np.float32)
