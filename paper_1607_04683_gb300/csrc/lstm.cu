@@ -12,14 +12,17 @@
 //      whose waits are bounded in time.
 // Output layer: quantize the top layer's outputs, integer product with Wo', recovery + bias, then
 // softmax with the pinned exponential.
+#include <algorithm>
 #include <cfloat>
 #include <cstdlib>
 #include <cstring>
+#include <functional>
 #include <vector>
 
 #include "lstm_model.h"
 #include "qnn_device.cuh"
 #include "qnn_host.h"
+#include "tc_gemm.h"
 
 namespace qnn {
 namespace {
@@ -414,12 +417,16 @@ __global__ void __launch_bounds__(kRecThreads, 1) lstm_recurrent_kernel(RecArgs 
 }
 
 __global__ void __launch_bounds__(256) softmax_rows_kernel(const float *__restrict__ logits, int C,
-                                                           float *__restrict__ y) {
+                                                           float *__restrict__ y, int64_t tm_B, int64_t tm_T,
+                                                           int64_t tm_t0) {
     __shared__ float red[8];
     __shared__ float s_bcast;
     const int64_t row = blockIdx.x;
     const float *l = logits + row * C;
-    float *yr = y + row * C;
+    // time-major rows (tm_B > 0): row i is frame tm_t0 + i / tm_B of sequence i % tm_B, whose
+    // posteriors go to row (i % tm_B) tm_T + tm_t0 + i / tm_B of y
+    const int64_t yrow = tm_B > 0 ? (row % tm_B) * tm_T + tm_t0 + row / tm_B : row;
+    float *yr = y + yrow * C;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float mx = -FLT_MAX;
     for (int c = threadIdx.x; c < C; c += 256) mx = fmaxf(mx, l[c]);
@@ -495,10 +502,11 @@ __global__ void __launch_bounds__(256) float_linear_kernel(const float *__restri
 
 }  // namespace
 
-qnn_status launch_softmax_rows(const float *logits, int64_t rows, int64_t C, float *y, cudaStream_t st) {
+qnn_status launch_softmax_rows(const float *logits, int64_t rows, int64_t C, float *y, cudaStream_t st, int64_t tm_B,
+                               int64_t tm_T, int64_t tm_t0) {
     if (rows == 0) return QNN_OK;
     ProfScope prof("softmax_rows", st);
-    softmax_rows_kernel<<<(unsigned)rows, 256, 0, st>>>(logits, (int)C, y);
+    softmax_rows_kernel<<<(unsigned)rows, 256, 0, st>>>(logits, (int)C, y, tm_B, tm_T, tm_t0);
     QNN_CUDA_TRY(cudaGetLastError());
     return QNN_OK;
 }
@@ -577,6 +585,9 @@ extern "C" void qnn_lstm_model_destroy(qnn_lstm_model *m) {
     cudaFree(m->fws);
     for (cudaStream_t w : m->wave_st) cudaStreamDestroy(w);
     for (cudaEvent_t e : m->wave_ev) cudaEventDestroy(e);
+    if (m->out_st) cudaStreamDestroy(m->out_st);
+    for (cudaEvent_t e : m->out_ev)
+        if (e) cudaEventDestroy(e);
     cudaSetDevice(prev);
     delete m;
 }
@@ -887,6 +898,14 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
         }
         for (int64_t l = 0; l < L; ++l) o_wout.push_back(acct(B * R * 4));
     }
+    // the 8-bit output layer beside the recurrence (wavefront): its input codes, which the top
+    // layer's step kernels write time-major (row t B + b), with their units and code sums
+    const char *ov_env = std::getenv("QNN_OUT_OVERLAP");
+    const bool out_overlap = wave && C > 0 && m->d.output_mode == QNN_OUT_QUANT && m->wo16 &&
+                             !(ov_env && std::strcmp(ov_env, "0") == 0);
+    const size_t o_ox16 = out_overlap ? acct(rows * kxr * 2) : 0;
+    const size_t o_oprm = out_overlap ? acct(rows * sizeof(qnn_qparams)) : 0;
+    const size_t o_ors = out_overlap ? acct(rows * 4) : 0;
     if (need > m->ws_bytes) {
         if (m->ws) {
             QNN_CUDA_TRY(cudaStreamSynchronize(st));
@@ -933,20 +952,23 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     const float *in = xd;
     int64_t kin = I;
     if (wave) {
-        // streams of layers 1 .. L - 1 and the events: L - 1 layer edges, a fork, L - 1 joins
-        if ((int64_t)m->wave_st.size() != L - 1) {
+        // one stream per layer, at the device's highest priority (the output layer's stream, below,
+        // at the lowest: the block scheduler then favours the recurrence, whose steps are the
+        // critical path, and the output work fills the SMs it leaves), and the events: L - 1 layer
+        // edges, a fork, L joins
+        if ((int64_t)m->wave_st.size() != L) {
             for (cudaStream_t w : m->wave_st) cudaStreamDestroy(w);
             for (cudaEvent_t e : m->wave_ev) cudaEventDestroy(e);
-            m->wave_st.assign((size_t)(L - 1), nullptr);
-            m->wave_ev.assign((size_t)(2 * L - 1), nullptr);
-            for (auto &w : m->wave_st) QNN_CUDA_TRY(cudaStreamCreateWithFlags(&w, cudaStreamNonBlocking));
+            int least = 0, greatest = 0;
+            QNN_CUDA_TRY(cudaDeviceGetStreamPriorityRange(&least, &greatest));
+            m->wave_st.assign((size_t)L, nullptr);
+            m->wave_ev.assign((size_t)(2 * L), nullptr);
+            for (auto &w : m->wave_st) QNN_CUDA_TRY(cudaStreamCreateWithPriority(&w, cudaStreamNonBlocking, greatest));
             for (auto &e : m->wave_ev) QNN_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
         }
-        std::vector<cudaStream_t> streams((size_t)L);
-        streams[0] = st;
-        for (int64_t l = 1; l < L; ++l) streams[(size_t)l] = m->wave_st[(size_t)(l - 1)];
+        std::vector<cudaStream_t> streams(m->wave_st.begin(), m->wave_st.end());
         const cudaEvent_t *edges = m->wave_ev.data(), fork = m->wave_ev[(size_t)(L - 1)];
-        const cudaEvent_t *joins = m->wave_ev.data() + L;
+        const cudaEvent_t *joins = m->wave_ev.data() + L;  // L of them
         std::vector<TcStackLayer> sl((size_t)L);
         std::vector<const float *> hsrc((size_t)L);
         std::vector<int64_t> hsrc_ld((size_t)L);
@@ -982,12 +1004,55 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
         }
         // the layer streams follow everything queued so far on the caller's stream
         QNN_CUDA_TRY(cudaEventRecord(fork, st));
-        for (int64_t l = 1; l < L; ++l) QNN_CUDA_TRY(cudaStreamWaitEvent(streams[(size_t)l], fork, 0));
-        QNN_TRY(tc_stack_recurrence(m, sl.data(), B, T, streams.data(), edges));
-        // ... and the caller's stream follows every layer
-        for (int64_t l = 1; l < L; ++l) {
-            QNN_CUDA_TRY(cudaEventRecord(joins[l - 1], streams[(size_t)l]));
-            QNN_CUDA_TRY(cudaStreamWaitEvent(st, joins[l - 1], 0));
+        for (int64_t l = 0; l < L; ++l) QNN_CUDA_TRY(cudaStreamWaitEvent(streams[(size_t)l], fork, 0));
+        // The output layer on chunks of frames as the top layer completes them, on its own stream:
+        // the product on the codes the top layer's step kernels write (time-major), logits
+        // time-major in lg, then the softmax into y's sequence-major rows.
+        TcFusedInput oc;
+        std::function<qnn_status(int64_t)> after_top;
+        int64_t t0 = 0;
+        if (out_overlap) {
+            if (!m->out_st) {
+                int least = 0, greatest = 0;
+                QNN_CUDA_TRY(cudaDeviceGetStreamPriorityRange(&least, &greatest));
+                QNN_CUDA_TRY(cudaStreamCreateWithPriority(&m->out_st, cudaStreamNonBlocking, least));
+                for (auto &e : m->out_ev) QNN_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+            }
+            QNN_CUDA_TRY(cudaStreamWaitEvent(m->out_st, fork, 0));
+            oc.x16 = reinterpret_cast<__half *>(ws + o_ox16), oc.kin = R;
+            oc.prm = reinterpret_cast<qnn_qparams *>(ws + o_oprm), oc.rs = reinterpret_cast<int32_t *>(ws + o_ors);
+            // chunks of about 32768 rows (QNN_OUT_CHUNK sets the frames of a chunk)
+            const char *ce = std::getenv("QNN_OUT_CHUNK");
+            const int64_t tchunk = ce && std::atoi(ce) > 0 ? std::atoi(ce) : std::max<int64_t>(1, (32768 + B - 1) / B);
+            const cudaStream_t top = streams[(size_t)(L - 1)], os = m->out_st;
+            after_top = [&, tchunk, top, os](int64_t t) -> qnn_status {
+                if (t + 1 - t0 < tchunk && t + 1 < T) return QNN_OK;
+                const int64_t t1 = t + 1, rc = (t1 - t0) * B;
+                QNN_CUDA_TRY(cudaEventRecord(m->out_ev[0], top));
+                QNN_CUDA_TRY(cudaStreamWaitEvent(os, m->out_ev[0], 0));
+                TcOperands op;
+                QNN_TRY(tc_operands(&op, oc.x16 + t0 * B * kxr, rc, m->wo16, C, kxr, tc_pick_bn(rc, C, kxr)));
+                QNN_TRY(tc_linear(op, oc.prm + t0 * B, 1, oc.rs + t0 * B, R, m->wo.params, C / m->S, m->wo.sums, m->bo,
+                                  lg + t0 * B * C, C, nullptr, os));
+                if (logits)
+                    for (int64_t tt = t0; tt < t1; ++tt)
+                        QNN_CUDA_TRY(cudaMemcpy2DAsync(logits + tt * C, T * C * 4, lg + tt * B * C, C * 4, C * 4, B,
+                                                       cudaMemcpyDefault, os));
+                QNN_TRY(launch_softmax_rows(lg + t0 * B * C, rc, C, yd, os, B, T, t0));
+                t0 = t1;
+                return QNN_OK;
+            };
+        }
+        QNN_TRY(tc_stack_recurrence(m, sl.data(), B, T, streams.data(), edges, out_overlap ? &oc : nullptr,
+                                    after_top));
+        // ... and the caller's stream follows every layer (and the output layer's stream)
+        for (int64_t l = 0; l < L; ++l) {
+            QNN_CUDA_TRY(cudaEventRecord(joins[l], streams[(size_t)l]));
+            QNN_CUDA_TRY(cudaStreamWaitEvent(st, joins[l], 0));
+        }
+        if (out_overlap) {
+            QNN_CUDA_TRY(cudaEventRecord(m->out_ev[1], m->out_st));
+            QNN_CUDA_TRY(cudaStreamWaitEvent(st, m->out_ev[1], 0));
         }
         for (int64_t l = 0; l < L; ++l) {
             if (h_state)  // final h of the layer: its output at the last frame
@@ -1056,7 +1121,9 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
         in = outl;
         kin = R;
     }
-    if (C > 0) {
+    if (C > 0 && out_overlap) {
+        // done beside the recurrence
+    } else if (C > 0) {
         if (m->d.output_mode == QNN_OUT_QUANT) {
             QNN_TRY(launch_quantize_rows(in, rows, R, R, codes, ld_in, prm, rs, st));
             QNN_TRY(launch_qgemm(codes, ld_in, prm, QNN_PER_ROW, rs, rows, R, m->wo.codes, m->wo.ld, m->wo.params,

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstdint>
+#include <functional>
 #include <vector>
 
 #include "qnn_host.h"
@@ -71,6 +72,11 @@ struct qnn_lstm_model {
     // streams of layers 1 .. L - 1 and events of the layer wavefront (made on first use)
     std::vector<cudaStream_t> wave_st;
     std::vector<cudaEvent_t> wave_ev;
+    // the output layer's stream and events when it runs beside the recurrence (made on first use)
+    cudaStream_t out_st = nullptr;
+    cudaEvent_t out_ev[2] = {nullptr, nullptr};
+    // the 8-bit output layer's Wo as centered fp16 [C][round_up(R, 64)] (in tcw)
+    __half *wo16 = nullptr;
     std::vector<qnn::TcLayer> tc_layers;
     // host mirror of the unit parameters (filled at creation)
     std::vector<qnn_qparams> host_params;
@@ -142,9 +148,14 @@ struct TcStackLayer {
     int64_t out_t = 0, out_b = 0;
     TcFusedInput fx;
 };
+// With top_codes the top layer's step kernel also writes its outputs' codes there (the output
+// layer's input, time-major like fx.x16); after_top_step(t) is called once the top layer's step t
+// is queued on its stream (streams[L - 1]).
 bool tc_stack_supported(const qnn_lstm_model *m);
 qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *layers, int64_t B, int64_t T,
-                               const cudaStream_t *streams, const cudaEvent_t *edges);
+                               const cudaStream_t *streams, const cudaEvent_t *edges,
+                               const TcFusedInput *top_codes = nullptr,
+                               const std::function<qnn_status(int64_t)> &after_top_step = nullptr);
 // Whether every layer's input product can be fused into its gate kernel (input width <= 1024; the
 // environment variable QNN_TC_FUSE_X=0 turns it off), and the workspace for the layer input's codes.
 bool tc_input_fused(const qnn_lstm_model *m);

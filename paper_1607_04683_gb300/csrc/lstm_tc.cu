@@ -16,6 +16,7 @@
 #include <cfloat>
 #include <cstdlib>
 #include <cstring>
+#include <functional>
 #include <vector>
 
 #include "lstm_model.h"
@@ -465,6 +466,9 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
             bytes += (size_t)round_up(12 * H * 4, 256);
         }
     }
+    // the 8-bit output layer's Wo as centered fp16 [C][kh], for its product on the top layer's codes
+    const bool wo16 = m->C > 0 && m->d.output_mode == QNN_OUT_QUANT;
+    if (wo16) bytes += (size_t)round_up(m->C * kh * 2, 256);
     void *buf = nullptr;
     QNN_CUDA_TRY(cudaMalloc(&buf, bytes));
     char *p = reinterpret_cast<char *>(buf);
@@ -519,6 +523,15 @@ qnn_status tc_prepare(qnn_lstm_model *m) {
                 cudaFree(buf);
                 return s;
             }
+        }
+    }
+    if (wo16) {
+        m->wo16 = reinterpret_cast<__half *>(p);
+        p += round_up(m->C * kh * 2, 256);
+        qnn_status s = launch_center_fp16(m->wo.codes, m->C, R, m->wo.ld, m->wo16, kh, nullptr);
+        if (s != QNN_OK) {
+            cudaFree(buf);
+            return s;
         }
     }
     if (cudaDeviceSynchronize() != cudaSuccess) {
@@ -702,7 +715,8 @@ bool tc_stack_supported(const qnn_lstm_model *m) {
 }
 
 qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *layers, int64_t B, int64_t T,
-                               const cudaStream_t *streams, const cudaEvent_t *edges) {
+                               const cudaStream_t *streams, const cudaEvent_t *edges, const TcFusedInput *top_codes,
+                               const std::function<qnn_status(int64_t)> &after_top_step) {
     if (!tc_stack_supported(m)) return QNN_ERR_INVALID_ARG;
     const int64_t L = m->L;
     std::vector<TcLayerRun> runs((size_t)L);
@@ -711,7 +725,10 @@ qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *laye
         const TcStackLayer &sl = layers[l];
         r.m = m, r.l = l, r.B = B, r.T = T, r.cbuf = sl.cbuf, r.mbuf = sl.mbuf;
         r.out = sl.out, r.out_t = sl.out_t, r.out_b = sl.out_b, r.st = streams[l];
-        if (l + 1 < L) r.nx16 = layers[l + 1].fx.x16, r.nprm = layers[l + 1].fx.prm, r.nrs = layers[l + 1].fx.rs;
+        if (l + 1 < L)
+            r.nx16 = layers[l + 1].fx.x16, r.nprm = layers[l + 1].fx.prm, r.nrs = layers[l + 1].fx.rs;
+        else if (top_codes)  // the output layer's input codes
+            r.nx16 = top_codes->x16, r.nprm = top_codes->prm, r.nrs = top_codes->rs;
         QNN_TRY(tc_layer_begin(r, sl.h0, sl.work, &sl.fx, l == 0));
     }
     // step t of layer l after step t of layer l - 1 (its input codes); each layer's own steps follow
@@ -721,6 +738,7 @@ qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *laye
             if (l > 0) QNN_CUDA_TRY(cudaStreamWaitEvent(streams[l], edges[l - 1], 0));
             QNN_TRY(tc_layer_step(runs[(size_t)l], t));
             if (l + 1 < L) QNN_CUDA_TRY(cudaEventRecord(edges[l], streams[l]));
+            else if (after_top_step) QNN_TRY(after_top_step(t));
         }
     return QNN_OK;
 }

@@ -90,7 +90,11 @@ qnn_status launch_qgemm_tc(const uint8_t *A, int64_t lda, const qnn_qparams *pa,
                            const int32_t *csW, int64_t N, const float *bias, float *Y, int64_t ldy, int32_t *acc_out,
                            void *scratch, cudaStream_t st);
 size_t tc_scratch_bytes(int64_t M, int64_t N, int64_t K);
-qnn_status launch_softmax_rows(const float *logits, int64_t rows, int64_t C, float *y, cudaStream_t st);
+// Softmax of rows of logits into y. With tm_B > 0 the rows are time-major, frames tm_t0 .. of tm_B
+// sequences (row i: frame tm_t0 + i / tm_B of sequence i % tm_B), and each goes to its row of the
+// sequence-major y [tm_B][tm_T][C].
+qnn_status launch_softmax_rows(const float *logits, int64_t rows, int64_t C, float *y, cudaStream_t st,
+                               int64_t tm_B = 0, int64_t tm_T = 0, int64_t tm_t0 = 0);
 // Sec. 4 frame stacking (frontend.cu): x [B][T][I] -> out [B][ceil(T/stride)][n I], device memory.
 qnn_status launch_stack_frames(const float *x, int64_t B, int64_t T, int64_t I, int n, int stride, float *out,
                                cudaStream_t st);

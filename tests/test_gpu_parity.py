@@ -565,6 +565,29 @@ def test_tc_layer_wavefront(qnn, want_h_all, proj, monkeypatch):
         assert np.array_equal(outs["1"][k], outs["0"][k]), k
 
 
+# The 8-bit output layer beside the recurrence (wavefront): chunks of frames as the top layer
+# completes them, from the codes its step kernels write, logits time-major and the softmax into the
+# sequence-major posteriors. Chunks of 1 and 2 frames (a short last chunk) and one chunk, LSTM and
+# LSTMP; logits bit-exact, and everything equal to the output layer run after the recurrence.
+@pytest.mark.parametrize("chunk", ["1", "2", ""])
+@pytest.mark.parametrize("P", [0, 128])
+def test_tc_output_layer_beside_recurrence(qnn, chunk, P, monkeypatch):
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    if chunk:
+        monkeypatch.setenv("QNN_OUT_CHUNK", chunk)
+    wl = _small(L=2, I=40, H=256, P=P, C=37, B=130, T=5, w=0.1, wo=0.5)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x, want_h_all=True)
+    outs = {}
+    for ov in ("1", "0"):
+        monkeypatch.setenv("QNN_OUT_OVERLAP", ov)
+        got = _gpu_forward(qnn, wl, params, x)
+        _compare(got, ref, wl, params)
+        outs[ov] = got
+    for k in ("y", "logits", "h", "c"):
+        assert np.array_equal(outs["1"][k], outs["0"][k]), k
+
+
 # 192 tiles of the gate product on 152 SMs: the 40 tiles of the last wave run as 80 half-width
 # items (N = 64 or 32); the same results with whole tiles (QNN_TC_HALF=0) and from the oracle
 @pytest.mark.parametrize("half", ["1", "0"])
