@@ -586,6 +586,7 @@ extern "C" void qnn_lstm_model_destroy(qnn_lstm_model *m) {
     for (cudaStream_t w : m->wave_st) cudaStreamDestroy(w);
     for (cudaEvent_t e : m->wave_ev) cudaEventDestroy(e);
     if (m->out_st) cudaStreamDestroy(m->out_st);
+    if (m->cp_st) cudaStreamDestroy(m->cp_st);
     for (cudaEvent_t e : m->out_ev)
         if (e) cudaEventDestroy(e);
     cudaSetDevice(prev);
@@ -906,6 +907,16 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     const size_t o_ox16 = out_overlap ? acct(rows * kxr * 2) : 0;
     const size_t o_oprm = out_overlap ? acct(rows * sizeof(qnn_qparams)) : 0;
     const size_t o_ors = out_overlap ? acct(rows * 4) : 0;
+    // chunks of about 32768 rows (QNN_OUT_CHUNK sets the frames of a chunk); posteriors for pinned
+    // host memory go through two device buffers of a chunk each, so that the copy engines carry
+    // them to the host while the SMs go on with the recurrence (QNN_OUT_STAGE=0: the softmax writes
+    // them to the host itself)
+    const char *ce = std::getenv("QNN_OUT_CHUNK");
+    const int64_t tchunk = std::min<int64_t>(
+        T, ce && std::atoi(ce) > 0 ? std::atoi(ce) : std::max<int64_t>(1, (32768 + B - 1) / B));
+    const char *se = std::getenv("QNN_OUT_STAGE");
+    const bool out_stage = out_overlap && y_map && !(se && std::strcmp(se, "0") == 0);
+    const size_t o_ystage = out_stage ? acct(2 * tchunk * B * C * 4) : 0;
     if (need > m->ws_bytes) {
         if (m->ws) {
             QNN_CUDA_TRY(cudaStreamSynchronize(st));
@@ -952,18 +963,16 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     const float *in = xd;
     int64_t kin = I;
     if (wave) {
-        // one stream per layer, at the device's highest priority (the output layer's stream, below,
-        // at the lowest: the block scheduler then favours the recurrence, whose steps are the
-        // critical path, and the output work fills the SMs it leaves), and the events: L - 1 layer
-        // edges, a fork, L joins
+        // one stream per layer (all at the default priority: with the layers above the output
+        // layer's stream, the output work waited for the end of the recurrence, and with the output
+        // layer above the layers, the recurrence slowed more than the output work gained), and the
+        // events: L - 1 layer edges, a fork, L joins
         if ((int64_t)m->wave_st.size() != L) {
             for (cudaStream_t w : m->wave_st) cudaStreamDestroy(w);
             for (cudaEvent_t e : m->wave_ev) cudaEventDestroy(e);
-            int least = 0, greatest = 0;
-            QNN_CUDA_TRY(cudaDeviceGetStreamPriorityRange(&least, &greatest));
             m->wave_st.assign((size_t)L, nullptr);
             m->wave_ev.assign((size_t)(2 * L), nullptr);
-            for (auto &w : m->wave_st) QNN_CUDA_TRY(cudaStreamCreateWithPriority(&w, cudaStreamNonBlocking, greatest));
+            for (auto &w : m->wave_st) QNN_CUDA_TRY(cudaStreamCreateWithFlags(&w, cudaStreamNonBlocking));
             for (auto &e : m->wave_ev) QNN_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
         }
         std::vector<cudaStream_t> streams(m->wave_st.begin(), m->wave_st.end());
@@ -1013,19 +1022,16 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
         int64_t t0 = 0;
         if (out_overlap) {
             if (!m->out_st) {
-                int least = 0, greatest = 0;
-                QNN_CUDA_TRY(cudaDeviceGetStreamPriorityRange(&least, &greatest));
-                QNN_CUDA_TRY(cudaStreamCreateWithPriority(&m->out_st, cudaStreamNonBlocking, least));
+                QNN_CUDA_TRY(cudaStreamCreateWithFlags(&m->out_st, cudaStreamNonBlocking));
+                QNN_CUDA_TRY(cudaStreamCreateWithFlags(&m->cp_st, cudaStreamNonBlocking));
                 for (auto &e : m->out_ev) QNN_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
             }
             QNN_CUDA_TRY(cudaStreamWaitEvent(m->out_st, fork, 0));
             oc.x16 = reinterpret_cast<__half *>(ws + o_ox16), oc.kin = R;
             oc.prm = reinterpret_cast<qnn_qparams *>(ws + o_oprm), oc.rs = reinterpret_cast<int32_t *>(ws + o_ors);
-            // chunks of about 32768 rows (QNN_OUT_CHUNK sets the frames of a chunk)
-            const char *ce = std::getenv("QNN_OUT_CHUNK");
-            const int64_t tchunk = ce && std::atoi(ce) > 0 ? std::atoi(ce) : std::max<int64_t>(1, (32768 + B - 1) / B);
-            const cudaStream_t top = streams[(size_t)(L - 1)], os = m->out_st;
-            after_top = [&, tchunk, top, os](int64_t t) -> qnn_status {
+            const cudaStream_t top = streams[(size_t)(L - 1)], os = m->out_st, cs = m->cp_st;
+            float *const ystage = out_stage ? reinterpret_cast<float *>(ws + o_ystage) : nullptr;
+            after_top = [&, top, os, cs, ystage](int64_t t) -> qnn_status {
                 if (t + 1 - t0 < tchunk && t + 1 < T) return QNN_OK;
                 const int64_t t1 = t + 1, rc = (t1 - t0) * B;
                 QNN_CUDA_TRY(cudaEventRecord(m->out_ev[0], top));
@@ -1038,7 +1044,21 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
                     for (int64_t tt = t0; tt < t1; ++tt)
                         QNN_CUDA_TRY(cudaMemcpy2DAsync(logits + tt * C, T * C * 4, lg + tt * B * C, C * 4, C * 4, B,
                                                        cudaMemcpyDefault, os));
-                QNN_TRY(launch_softmax_rows(lg + t0 * B * C, rc, C, yd, os, B, T, t0));
+                if (ystage) {
+                    // softmax into the chunk's buffer (sequence-major within the chunk) once the copy
+                    // out of that buffer two chunks ago is done, then the copy into y's rows
+                    const int64_t k = t0 / tchunk, n = t1 - t0;
+                    float *const sb = ystage + (k & 1) * tchunk * B * C;
+                    if (k >= 2) QNN_CUDA_TRY(cudaStreamWaitEvent(os, m->out_ev[4 + (k & 1)], 0));
+                    QNN_TRY(launch_softmax_rows(lg + t0 * B * C, rc, C, sb, os, B, n, 0));
+                    QNN_CUDA_TRY(cudaEventRecord(m->out_ev[2 + (k & 1)], os));
+                    QNN_CUDA_TRY(cudaStreamWaitEvent(cs, m->out_ev[2 + (k & 1)], 0));
+                    QNN_CUDA_TRY(cudaMemcpy2DAsync(y + t0 * C, T * C * 4, sb, n * C * 4, n * C * 4, B,
+                                                   cudaMemcpyDeviceToHost, cs));
+                    QNN_CUDA_TRY(cudaEventRecord(m->out_ev[4 + (k & 1)], cs));
+                } else {
+                    QNN_TRY(launch_softmax_rows(lg + t0 * B * C, rc, C, yd, os, B, T, t0));
+                }
                 t0 = t1;
                 return QNN_OK;
             };
@@ -1053,6 +1073,10 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
         if (out_overlap) {
             QNN_CUDA_TRY(cudaEventRecord(m->out_ev[1], m->out_st));
             QNN_CUDA_TRY(cudaStreamWaitEvent(st, m->out_ev[1], 0));
+        }
+        if (out_stage) {
+            QNN_CUDA_TRY(cudaEventRecord(m->out_ev[6], m->cp_st));
+            QNN_CUDA_TRY(cudaStreamWaitEvent(st, m->out_ev[6], 0));
         }
         for (int64_t l = 0; l < L; ++l) {
             if (h_state)  // final h of the layer: its output at the last frame

@@ -72,9 +72,12 @@ struct qnn_lstm_model {
     // streams of layers 1 .. L - 1 and events of the layer wavefront (made on first use)
     std::vector<cudaStream_t> wave_st;
     std::vector<cudaEvent_t> wave_ev;
-    // the output layer's stream and events when it runs beside the recurrence (made on first use)
-    cudaStream_t out_st = nullptr;
-    cudaEvent_t out_ev[2] = {nullptr, nullptr};
+    // the output layer's stream, the stream of its copies to the host and their events when it runs
+    // beside the recurrence (made on first use): [0] a chunk of the top layer done, [1] output stream
+    // joined, [2, 3] posteriors staged in buffer 0 / 1, [4, 5] buffer 0 / 1 copied out, [6] copy
+    // stream joined
+    cudaStream_t out_st = nullptr, cp_st = nullptr;
+    cudaEvent_t out_ev[7] = {};
     // the 8-bit output layer's Wo as centered fp16 [C][round_up(R, 64)] (in tcw)
     __half *wo16 = nullptr;
     std::vector<qnn::TcLayer> tc_layers;

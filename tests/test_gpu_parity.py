@@ -588,6 +588,31 @@ def test_tc_output_layer_beside_recurrence(qnn, chunk, P, monkeypatch):
         assert np.array_equal(outs["1"][k], outs["0"][k]), k
 
 
+# posteriors for pinned host memory: staged in two device buffers of a chunk and copied out
+# beside the recurrence (chunks of 1, 2 and 3 frames of 5: buffers reused, a ragged last chunk), or
+# written to the host by the softmax itself; both equal the device-memory result
+@pytest.mark.parametrize("stage", ["1", "0"])
+@pytest.mark.parametrize("chunk", ["1", "2", "3"])
+def test_tc_output_posteriors_to_pinned_host(qnn, chunk, stage, monkeypatch):
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    monkeypatch.setenv("QNN_OUT_CHUNK", chunk)
+    monkeypatch.setenv("QNN_OUT_STAGE", stage)
+    wl = _small(L=2, I=40, H=256, P=64, C=37, B=130, T=5, w=0.1, wo=0.5)
+    params, x = wl.make()
+    ref = _oracle(wl, params, x)
+    d = qnn.lstm_desc(wl.num_layers, wl.input_dim, wl.hidden, wl.proj, wl.num_classes, wl.output_mode)
+    model = qnn.LstmModel(d, gpu(params))
+    y_dev = model.forward(gpu(x)).cpu().numpy()
+    x_host = torch.from_numpy(x).pin_memory()
+    y_host = torch.full((wl.batch, wl.frames, wl.num_classes), float("nan"), dtype=torch.float32).pin_memory()
+    for _ in range(2):  # the second pass reuses the staging buffers
+        model.forward(x_host, y=y_host)
+        torch.cuda.synchronize()
+        assert qnn.device_status() == qnn.QNN_OK
+        assert np.array_equal(y_host.numpy(), y_dev)
+    parity.check_posteriors(y_dev, ref["y"])
+
+
 # 192 tiles of the gate product on 152 SMs: the 40 tiles of the last wave run as 80 half-width
 # items (N = 64 or 32); the same results with whole tiles (QNN_TC_HALF=0) and from the oracle
 @pytest.mark.parametrize("half", ["1", "0"])
