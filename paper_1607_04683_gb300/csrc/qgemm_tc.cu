@@ -1275,7 +1275,7 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
     // QNN_TC_HALF=0 keeps whole tiles)
     TcArgs args = a;
     args.full_tiles = 0;
-    if (TL::IS_LSTM && (BN == 64 || BN == 128) && a.splits == 1 && items > grid) {
+    if (TL::IS_LSTM && op.half_items && (BN == 64 || BN == 128) && a.splits == 1 && items > grid) {
         const char *e = std::getenv("QNN_TC_HALF");
         const int64_t r = items % grid;
         if (r > 0 && 2 * r <= grid && !(e && std::strcmp(e, "0") == 0)) args.full_tiles = items - r;
