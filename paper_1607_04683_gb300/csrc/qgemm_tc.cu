@@ -78,9 +78,11 @@ struct Tile {
     // a pipeline stage carries KPS consecutive k-blocks (A sub-tiles first, then the W sub-tiles):
     // the operand stream advances by stages at a pace that hardly depends on their size, so short
     // reductions (K <= 1024) take several k-blocks a stage: four for narrow LSTM tiles (two stages in
-    // flight), two for row tiles and split-K items; the long-K linear tiles and the 96-column LSTM
-    // tiles keep more, smaller stages in flight (each choice measured on GB300)
-    static constexpr int KPS = IS_LSTM ? (BN <= 32 ? 4 : (BN == 64 ? 2 : 1))
+    // flight), two for row tiles, split-K items and the 128-column LSTM tiles with the input product
+    // (two 64 KB stages: 38.9 against 41.1 us a step with four of 32 KB); the long-K linear tiles and
+    // the other 96- and 128-column LSTM tiles keep more, smaller stages in flight (each choice
+    // measured on GB300)
+    static constexpr int KPS = IS_LSTM ? (BN <= 32 ? 4 : ((BN == 64 || (BN == 128 && EPI == kEpiLstmX)) ? 2 : 1))
                                                : ((EPI == kEpiPartial || EPI == kEpiRow) ? 2 : 1);
     static constexpr int SUB_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGE_BYTES = KPS * SUB_BYTES;
