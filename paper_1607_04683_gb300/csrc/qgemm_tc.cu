@@ -1271,7 +1271,8 @@ qnn_status launch_tc(const TcOperands &op, const TcArgs &a, const char *name, cu
     }
     const int64_t items = ((a.M + TBM - 1) / TBM) * ((a.N + BN - 1) / BN) * a.splits;  // (tile, K range) pairs
     // persistent: one block per SM (a block holding tensor memory has its SM to itself)
-    const unsigned grid = (unsigned)std::min<int64_t>(items, (int64_t)sm_count());
+    const int64_t blocks = op.max_blocks > 0 ? std::min(op.max_blocks, sm_count()) : sm_count();
+    const unsigned grid = (unsigned)std::min<int64_t>(items, blocks);
     // LSTM tiles of 64 or 128 columns: when the last wave is partial and its tiles, halved, fit one
     // wave, they run as two half-width items each (the busiest block then does half a tile less;
     // QNN_TC_HALF=0 keeps whole tiles)

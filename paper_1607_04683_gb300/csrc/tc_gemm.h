@@ -26,6 +26,8 @@ struct TcOperands {
     bool row_epilogue = false;  // linear products: set by tc_operands when kp <= 1024 and bn <= 128
     // LSTM epilogues: a last, partial wave of tiles may run as half-width items (QNN_TC_HALF=0: never)
     bool half_items = true;
+    // persistent grid: at most this many blocks (0: one per SM)
+    int max_blocks = 0;
 };
 qnn_status tc_operands(TcOperands *op, const __half *A16, int64_t M, const __half *W16, int64_t N, int64_t kp, int bn);
 // Default tile width of a linear product (QNN_TC_BN overrides).
