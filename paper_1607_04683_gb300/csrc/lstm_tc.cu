@@ -737,6 +737,10 @@ qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *laye
         // (4.15M against 4.07M frames/s with every SM; 128 and 144 of 152 blocks: 4.11M)
         r.gates.half_items = false;
         r.gates.max_blocks = sm_count() * 9 / 10;
+        // the projection's split-K product in as few K ranges as its exact chunks allow: fewer,
+        // longer work items hold fewer SMs beside the other layers' gate kernels (4.38M against
+        // 4.09-4.13M frames/s with 2 ranges of 1024 instead of 4 of 512)
+        if (r.split_proj) r.splits = tc_partial_splits(r.proj, (int)max_proj_splits(m), false);
     }
     // step t of layer l after step t of layer l - 1 (its input codes); each layer's own steps follow
     // its stream order

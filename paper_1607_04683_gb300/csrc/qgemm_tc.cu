@@ -1432,11 +1432,12 @@ qnn_status tc_lstm_gates_x(const TcOperands &op, const qnn_qparams *pa, const in
     }
 }
 
-int tc_partial_splits(const TcOperands &op, int max_splits) {
+int tc_partial_splits(const TcOperands &op, int max_splits, bool fill_sms) {
     const int KB = (int)(op.kp / TBK), kpc = KCHUNK / TBK;
     const int64_t tiles = ((op.M + TBM - 1) / TBM) * ((op.N + op.bn - 1) / op.bn);
-    // as many K ranges as keep the work items within one wave, but at least one exact chunk each
-    int splits = (int)std::max<int64_t>((KB + kpc - 1) / kpc, sm_count() / tiles);
+    // as many K ranges as keep the work items within one wave (without fill_sms: as few as the
+    // exact chunks allow), but at least one exact chunk each
+    int splits = (int)std::max<int64_t>((KB + kpc - 1) / kpc, fill_sms ? sm_count() / tiles : 1);
     splits = std::max(1, std::min({splits, KB, std::max(max_splits, (KB + kpc - 1) / kpc)}));
     const int kbs = (KB + splits - 1) / splits;  // equal ranges (the last one shorter)
     return (KB + kbs - 1) / kbs;

@@ -95,8 +95,8 @@ qnn_status tc_lstm_gates(const TcOperands &op, const qnn_qparams *pa, const int3
 // (a - 128)(w - 128), int32, ranges of at most 1024 so that each is exact in one accumulator;
 // the slices add up to P = acc - 128 (rsA + csW) + 128^2 K. ldpart >= N (elements).
 // K ranges giving at most one wave of work items (each range one exact chunk; at most
-// max(max_splits, the chunks K needs) ranges).
-int tc_partial_splits(const TcOperands &op, int max_splits);
+// max(max_splits, the chunks K needs) ranges); without fill_sms, the fewest exact chunks.
+int tc_partial_splits(const TcOperands &op, int max_splits, bool fill_sms = true);
 qnn_status tc_partial(const TcOperands &op, int splits, int32_t *part, int64_t ldpart, cudaStream_t st);
 
 // u8 codes [rows][ldi] -> centered fp16 [rows][ldo], zero past K.
