@@ -580,6 +580,7 @@ struct TcLayerRun {
     qnn_qparams *nprm = nullptr;
     int32_t *nrs = nullptr;
     cudaStream_t st = nullptr;
+    bool wave = false;  // one layer of a wavefront (other layers' kernels run beside this one's)
     // set by tc_layer_begin
     TcOperands gates, proj;
     bool split_proj = false, fused = false;
@@ -623,9 +624,13 @@ qnn_status tc_layer_begin(TcLayerRun &s, const float *h0, void *work, const TcFu
     // The fused kernel's operand stream (A re-read for every tile of a block) is bounded by the rate at
     // which a block's TMA ring turns over, so with at least a full wave of tiles the widest tile wins
     // (LSTMP 5x2048p512 B=1024: 128 columns 49.6 us per step against 52.0 for 64); with less than a
-    // wave the tile count that fills the SMs best decides.
+    // wave the tile count that fills the SMs best decides, except in a wavefront, where the other
+    // layers' kernels fill the SMs a narrow grid leaves: there the widest tile always wins (5 x 500
+    // B = 256: 32 blocks of 128 columns 8.9M frames/s, 64 of 64 columns 8.5M, 126 of 32 columns 6.0M).
     int bn_gates = fx ? tc_choose_bn(B, 4 * H8, gate_bn_fused, 3) : tc_choose_bn(B, 4 * H8, gate_bn, 4);
-    if (fx && !std::getenv("QNN_TC_BN") && ((B + 127) / 128) * ((4 * H8 + 127) / 128) >= sm_count()) bn_gates = 128;
+    if (fx && !std::getenv("QNN_TC_BN") &&
+        (s.wave || ((B + 127) / 128) * ((4 * H8 + 127) / 128) >= sm_count()))
+        bn_gates = 128;
     QNN_TRY(tc_operands(&s.gates, s.a16, B, tl.wh16, 4 * H8, kh, bn_gates));
     // the projection after the m_t quantizer: split-K partial sums finished (offsets, recovery, next
     // step's quantization) by one row kernel; or one tcgen05 product with its own epilogue per step
@@ -729,6 +734,7 @@ qnn_status tc_stack_recurrence(const qnn_lstm_model *m, const TcStackLayer *laye
             r.nx16 = layers[l + 1].fx.x16, r.nprm = layers[l + 1].fx.prm, r.nrs = layers[l + 1].fx.rs;
         else if (top_codes)  // the output layer's input codes
             r.nx16 = top_codes->x16, r.nprm = top_codes->prm, r.nrs = top_codes->rs;
+        r.wave = true;
         QNN_TRY(tc_layer_begin(r, sl.h0, sl.work, &sl.fx, l == 0));
         // whole tiles in the last, partial wave: the blocks that finish early free their SMs for
         // the other layers' kernels, which gains more than halving those tiles to even out the
