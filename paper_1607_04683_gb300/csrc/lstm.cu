@@ -470,6 +470,76 @@ __global__ void __launch_bounds__(256) softmax_rows_kernel(const float *__restri
     }
 }
 
+// The same softmax with the row held in registers (rows of at most 256 V values, C a multiple of 4,
+// 16-byte aligned rows): the logits are read once, each E(l - max) is computed once and kept, and
+// the quotients E / sum come from the sum's correctly rounded reciprocal r (q = RN(E r), then
+// RN(q + (E - q sum) r), the last step of Markstein's division; equal to the IEEE quotient while
+// E >= 2^-100 and 1 <= sum <= 2^24, which a CPU test checks; smaller E divide as IEEE). Thread t
+// holds the 4-value groups t, t + 256, ...
+template <int V>
+__global__ void __launch_bounds__(256) softmax_rows_reg_kernel(const float *__restrict__ logits, int C,
+                                                               float *__restrict__ y, int64_t tm_B, int64_t tm_T,
+                                                               int64_t tm_t0) {
+    __shared__ float red[8];
+    __shared__ float s_bcast;
+    const int64_t row = blockIdx.x;
+    const float4 *l4 = reinterpret_cast<const float4 *>(logits + row * C);
+    const int64_t yrow = tm_B > 0 ? (row % tm_B) * tm_T + tm_t0 + row / tm_B : row;
+    float4 *y4 = reinterpret_cast<float4 *>(y + yrow * C);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int C4 = C / 4;
+    float e[V];
+    float mx = -FLT_MAX;
+#pragma unroll
+    for (int j = 0; j < V / 4; ++j) {
+        const int v = (int)threadIdx.x + 256 * j;
+        float4 a = make_float4(-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX);
+        if (v < C4) a = l4[v];
+        e[4 * j] = a.x, e[4 * j + 1] = a.y, e[4 * j + 2] = a.z, e[4 * j + 3] = a.w;
+        mx = fmaxf(mx, fmaxf(fmaxf(a.x, a.y), fmaxf(a.z, a.w)));
+    }
+    mx = warp_max(mx);
+    if (lane == 0) red[warp] = mx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float v = red[0];
+        for (int w = 1; w < 8; ++w) v = fmaxf(v, red[w]);
+        s_bcast = v;
+    }
+    __syncthreads();
+    mx = s_bcast;
+    float s = 0.0f;
+#pragma unroll
+    for (int j = 0; j < V / 4; ++j) {
+        if ((int)threadIdx.x + 256 * j >= C4) break;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            e[4 * j + i] = pexp(__fsub_rn(e[4 * j + i], mx));
+            s = __fadd_rn(s, e[4 * j + i]);
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s = __fadd_rn(s, __shfl_xor_sync(0xffffffffu, s, o));
+    __syncthreads();
+    if (lane == 0) red[warp] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float v = red[0];
+        for (int w = 1; w < 8; ++w) v = __fadd_rn(v, red[w]);
+        s_bcast = v;
+    }
+    __syncthreads();
+    s = s_bcast;
+    const float r = __frcp_rn(s);
+    auto quot = [&](float x) { return x >= 0x1p-100f ? div_by_recip(x, s, r) : __fdiv_rn(x, s); };
+#pragma unroll
+    for (int j = 0; j < V / 4; ++j) {
+        const int v = (int)threadIdx.x + 256 * j;
+        if (v >= C4) break;
+        y4[v] = make_float4(quot(e[4 * j]), quot(e[4 * j + 1]), quot(e[4 * j + 2]), quot(e[4 * j + 3]));
+    }
+}
+
 // fp32 output layer for the "quant" variant: logits[m][c] = sum_k r[m][k] Wo[c][k] + bo[c].
 __global__ void __launch_bounds__(256) float_linear_kernel(const float *__restrict__ X, int64_t M, int K,
                                                            const float *__restrict__ Wt, int C,
@@ -506,7 +576,17 @@ qnn_status launch_softmax_rows(const float *logits, int64_t rows, int64_t C, flo
                                int64_t tm_T, int64_t tm_t0) {
     if (rows == 0) return QNN_OK;
     ProfScope prof("softmax_rows", st);
-    softmax_rows_kernel<<<(unsigned)rows, 256, 0, st>>>(logits, (int)C, y, tm_B, tm_T, tm_t0);
+    // rows in registers when they fit (1 <= sum <= C <= 8192 keeps the reciprocal quotient exact)
+    const bool reg = (C & 3) == 0 && C <= 8192 &&
+                     ((reinterpret_cast<uintptr_t>(logits) | reinterpret_cast<uintptr_t>(y)) & 15) == 0;
+    if (reg && C <= 2048)
+        softmax_rows_reg_kernel<8><<<(unsigned)rows, 256, 0, st>>>(logits, (int)C, y, tm_B, tm_T, tm_t0);
+    else if (reg && C <= 4096)
+        softmax_rows_reg_kernel<16><<<(unsigned)rows, 256, 0, st>>>(logits, (int)C, y, tm_B, tm_T, tm_t0);
+    else if (reg)
+        softmax_rows_reg_kernel<32><<<(unsigned)rows, 256, 0, st>>>(logits, (int)C, y, tm_B, tm_T, tm_t0);
+    else
+        softmax_rows_kernel<<<(unsigned)rows, 256, 0, st>>>(logits, (int)C, y, tm_B, tm_T, tm_t0);
     QNN_CUDA_TRY(cudaGetLastError());
     return QNN_OK;
 }

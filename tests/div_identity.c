@@ -1,7 +1,9 @@
 /* Test helper (compiled by tests/test_float_identities.py): checks that x / d, correctly rounded,
  * equals q + (x - q d) r with r = RN(1/d) and q = RN(x r), each step rounded once (fmaf), for every
  * 24-bit numerator significand against the given divisor significands, and for random pairs of an
- * integer numerator (|x| < 2^31) and a divisor in [2^-60, 2^60]. Prints the number of mismatches. */
+ * integer numerator (|x| < 2^31) and a divisor in [2^-60, 2^60]; and, for the softmax's quotients
+ * E / sum, for random numerators in [2^-100, 1] against divisors in [1, 2^24]. Prints the number of
+ * pairs checked and of mismatches. */
 #include <math.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -47,6 +49,21 @@ int main(int argc, char **argv)
         long long xi = (long long)((u >> 33) & ((1ull << len) - 1));
         if (u >> 63) xi = -xi;
         float x = (float)xi;
+        float r = 1.0f / d;
+        if (bits(div_by_recip(x, d, r)) != bits(x / d)) ++bad;
+        ++n;
+    }
+    long nsoft = argc > 3 ? atol(argv[3]) : 0;
+    for (long i = 0; i < nsoft; ++i) {
+        uint64_t u = next();
+        int ex = -(int)(u % 101);                         /* numerator exponent -100 .. 0 */
+        uint32_t mx = (uint32_t)((u >> 8) & 0x7FFFFFu);
+        float x = ex == 0 ? 1.0f : from_bits((uint32_t)(ex + 127) << 23 | mx);
+        int ed = (int)((u >> 32) % 25);                   /* divisor exponent 0 .. 24 */
+        uint32_t md = (uint32_t)((u >> 40) & 0x7FFFFFu);
+        if ((u & 0xF) == 0) md = 0x7FFFFFu;               /* all-ones significands now and then */
+        float d = from_bits((uint32_t)(ed + 127) << 23 | md);
+        if (d > 16777216.0f) d = 16777216.0f;
         float r = 1.0f / d;
         if (bits(div_by_recip(x, d, r)) != bits(x / d)) ++bad;
         ++n;

@@ -6,6 +6,8 @@ kernel takes that quotient from the divisor's correctly rounded reciprocal r, co
 multiply-add (the final step of Markstein's division). A C helper checks, with gcc's fmaf, that
 this equals the IEEE quotient for every 24-bit numerator significand against 64 divisor
 significands (all-ones and power-of-two neighbours among them) and on random integer/divisor pairs.
+The softmax divides each E(l - max) in [2^-100, 1] by the row's sum in [1, C] the same way; random
+pairs over those ranges (divisors up to 2^24) are checked too.
 
 The gate nonlinearities (sigma = 1/(E(-x) + 1), tanh = 1 - 2/(E(2x) + 1), Sec. 3.1 cell with the
 pinned exponential) are evaluated on the GPU from the correctly rounded reciprocal r = RN(1/d):
@@ -71,6 +73,6 @@ def test_quotient_from_the_reciprocal_is_the_ieee_quotient():
     with tempfile.TemporaryDirectory() as d:
         exe = os.path.join(d, "div_identity")
         subprocess.check_call([cc, "-O2", "-ffp-contract=off", "-fno-fast-math", "-o", exe, src, "-lm"])
-        n, bad = (int(v) for v in subprocess.check_output([exe, "64", "20000000"], text=True).split())
-    assert n == 64 * (1 << 23) + 20000000
+        n, bad = (int(v) for v in subprocess.check_output([exe, "64", "20000000", "20000000"], text=True).split())
+    assert n == 64 * (1 << 23) + 20000000 + 20000000
     assert bad == 0
