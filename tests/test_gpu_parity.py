@@ -565,6 +565,26 @@ def test_tc_layer_wavefront(qnn, want_h_all, proj, monkeypatch):
         assert np.array_equal(outs["1"][k], outs["0"][k]), k
 
 
+# The wavefront's own launch shapes (gate grid below one block per SM, whole tiles in the last wave,
+# the projection in the fewest exact K ranges) on a batch of 3 row tiles and 64 column tiles: 192
+# tiles on 136 blocks, so blocks take a second tile of another row tile (their per-row constants
+# recomputed). Equal to the layers run in sequence bit for bit, and to the oracle on one sequence
+# of each row tile.
+def test_tc_wavefront_shapes_row_tile_changes(qnn, monkeypatch):
+    monkeypatch.setenv("QNN_LSTM_PATH", "tc")
+    wl = _small(L=2, I=80, H=2048, P=256, C=37, B=384, T=4, w=0.05, wo=0.5)
+    params, x = wl.make()
+    outs = {}
+    for wave in ("1", "0"):
+        monkeypatch.setenv("QNN_TC_WAVE", wave)
+        outs[wave] = _gpu_forward(qnn, wl, params, x, h_all=False)
+    for k in ("y", "h", "c", "logits"):
+        assert np.array_equal(outs["1"][k], outs["0"][k]), k
+    seqs = (0, 200, 383)
+    for b, ref in zip(seqs, _sequences_by_oracle(wl, params, x, seqs)):
+        _check_sequence(outs["1"], ref, b)
+
+
 # The 8-bit output layer beside the recurrence (wavefront): chunks of frames as the top layer
 # completes them, from the codes its step kernels write, logits time-major and the softmax into the
 # sequence-major posteriors. Chunks of 1 and 2 frames (a short last chunk) and one chunk, LSTM and
