@@ -171,11 +171,16 @@ qnn_status qnn_lstm_model_weights(const qnn_lstm_model *m, uint8_t *codes_host, 
  * x, y, h_state, c_state and h_all may each be host or device memory: host buffers are copied
  * to or from device memory on `stream` inside the call (pinned host memory keeps the copies
  * asynchronous). Posteriors (num_classes > 0) for a y in pinned host memory are written there
- * by the softmax kernel itself, without a device copy and a second transfer. With any host
- * buffer the results are complete once `stream` has been synchronized. Activations are
- * quantized per row (one frame of one sequence), weights per
- * gate matrix. The model keeps a device workspace sized for the largest B*T seen; calls on one
- * model must not overlap in time.
+ * by the softmax kernel itself, or, when the output layer runs beside the recurrence (below),
+ * staged chunk by chunk in two device buffers of the workspace and copied by the copy engines.
+ * With any host buffer the results are complete once `stream` has been synchronized.
+ * Activations are quantized per row (one frame of one sequence), weights per gate matrix.
+ * Large batches of a multi-layer model run their layers as a wavefront: the call may place its
+ * work on streams and events the model owns (one stream per layer, one for the output layer and
+ * one for its copies to the host), which start after everything queued on `stream` before the
+ * call, and `stream` waits for all of them before anything queued after it, so the call stays
+ * ordered on `stream` as a single launch would be. The model keeps a device workspace sized for
+ * the largest B*T seen; calls on one model must not overlap in time.
  */
 qnn_status qnn_lstm_forward(qnn_lstm_model *m, const float *x, int64_t B, int64_t T, float *y, float *h_state,
                             float *c_state, float *h_all, void *stream);
