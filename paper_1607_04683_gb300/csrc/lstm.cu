@@ -935,6 +935,19 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     // layers as a wavefront on one stream each (every layer's recurrence state its own; the layer
     // outputs are kept whole only where they are read: the top layer, and every layer with h_all)
     const bool wave = fused && tc_stack_supported(m) && (!h_all || ha_dev);
+    // the 8-bit output layer beside the recurrence (wavefront)
+    const char *ov_env = std::getenv("QNN_OUT_OVERLAP");
+    const bool out_overlap = wave && C > 0 && m->d.output_mode == QNN_OUT_QUANT && m->wo16 &&
+                             !(ov_env && std::strcmp(ov_env, "0") == 0);
+    // chunks of about 32768 rows (QNN_OUT_CHUNK sets the frames of a chunk); posteriors for pinned
+    // host memory go through two device buffers of a chunk each, so that the copy engines carry
+    // them to the host while the SMs go on with the recurrence (QNN_OUT_STAGE=0: the softmax writes
+    // them to the host itself)
+    const char *ce = std::getenv("QNN_OUT_CHUNK");
+    const int64_t tchunk = std::min<int64_t>(
+        T, ce && std::atoi(ce) > 0 ? std::atoi(ce) : std::max<int64_t>(1, (32768 + B - 1) / B));
+    const char *se = std::getenv("QNN_OUT_STAGE");
+    const bool out_stage = out_overlap && y_map && !(se && std::strcmp(se, "0") == 0);
     const FwdPlan plan = plan_recurrent(m, B);
 
     // workspace layout
@@ -960,7 +973,9 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     const size_t o_qc = acct(B * ldq);
     const size_t o_qp = acct(B * sizeof(qnn_qparams));
     const size_t o_qs = acct(B * 4);
-    const size_t o_lg = acct(C > 0 ? rows * C * 4 : 0);
+    // logits: every row, or with the output layer beside the recurrence one chunk at a time (the
+    // chunks' products, copies and softmaxes run in order on one stream)
+    const size_t o_lg = acct(C > 0 ? (out_overlap ? std::min(rows, tchunk * B) : rows) * C * 4 : 0);
     const size_t o_y = (y_dev || y_map) ? 0 : acct(rows * ycols * 4);
     const size_t o_tc = use_tc ? acct(tc_work_bytes(m, B)) : 0;
     // wavefront: for layers 1 .. L - 1 (index l - 1) the input codes the previous layer writes and
@@ -979,23 +994,11 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
         }
         for (int64_t l = 0; l < L; ++l) o_wout.push_back(acct(B * R * 4));
     }
-    // the 8-bit output layer beside the recurrence (wavefront): its input codes, which the top
-    // layer's step kernels write time-major (row t B + b), with their units and code sums
-    const char *ov_env = std::getenv("QNN_OUT_OVERLAP");
-    const bool out_overlap = wave && C > 0 && m->d.output_mode == QNN_OUT_QUANT && m->wo16 &&
-                             !(ov_env && std::strcmp(ov_env, "0") == 0);
+    // the output layer's input codes, which the top layer's step kernels write time-major (row
+    // t B + b), with their units and code sums; the staged posteriors
     const size_t o_ox16 = out_overlap ? acct(rows * kxr * 2) : 0;
     const size_t o_oprm = out_overlap ? acct(rows * sizeof(qnn_qparams)) : 0;
     const size_t o_ors = out_overlap ? acct(rows * 4) : 0;
-    // chunks of about 32768 rows (QNN_OUT_CHUNK sets the frames of a chunk); posteriors for pinned
-    // host memory go through two device buffers of a chunk each, so that the copy engines carry
-    // them to the host while the SMs go on with the recurrence (QNN_OUT_STAGE=0: the softmax writes
-    // them to the host itself)
-    const char *ce = std::getenv("QNN_OUT_CHUNK");
-    const int64_t tchunk = std::min<int64_t>(
-        T, ce && std::atoi(ce) > 0 ? std::atoi(ce) : std::max<int64_t>(1, (32768 + B - 1) / B));
-    const char *se = std::getenv("QNN_OUT_STAGE");
-    const bool out_stage = out_overlap && y_map && !(se && std::strcmp(se, "0") == 0);
     const size_t o_ystage = out_stage ? acct(2 * tchunk * B * C * 4) : 0;
     if (need > m->ws_bytes) {
         if (m->ws) {
@@ -1119,10 +1122,10 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
                 TcOperands op;
                 QNN_TRY(tc_operands(&op, oc.x16 + t0 * B * kxr, rc, m->wo16, C, kxr, tc_pick_bn(rc, C, kxr)));
                 QNN_TRY(tc_linear(op, oc.prm + t0 * B, 1, oc.rs + t0 * B, R, m->wo.params, C / m->S, m->wo.sums, m->bo,
-                                  lg + t0 * B * C, C, nullptr, os));
+                                  lg, C, nullptr, os));
                 if (logits)
                     for (int64_t tt = t0; tt < t1; ++tt)
-                        QNN_CUDA_TRY(cudaMemcpy2DAsync(logits + tt * C, T * C * 4, lg + tt * B * C, C * 4, C * 4, B,
+                        QNN_CUDA_TRY(cudaMemcpy2DAsync(logits + tt * C, T * C * 4, lg + (tt - t0) * B * C, C * 4, C * 4, B,
                                                        cudaMemcpyDefault, os));
                 if (ystage) {
                     // softmax into the chunk's buffer (sequence-major within the chunk) once the copy
@@ -1130,14 +1133,14 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
                     const int64_t k = t0 / tchunk, n = t1 - t0;
                     float *const sb = ystage + (k & 1) * tchunk * B * C;
                     if (k >= 2) QNN_CUDA_TRY(cudaStreamWaitEvent(os, m->out_ev[4 + (k & 1)], 0));
-                    QNN_TRY(launch_softmax_rows(lg + t0 * B * C, rc, C, sb, os, B, n, 0));
+                    QNN_TRY(launch_softmax_rows(lg, rc, C, sb, os, B, n, 0));
                     QNN_CUDA_TRY(cudaEventRecord(m->out_ev[2 + (k & 1)], os));
                     QNN_CUDA_TRY(cudaStreamWaitEvent(cs, m->out_ev[2 + (k & 1)], 0));
                     QNN_CUDA_TRY(cudaMemcpy2DAsync(y + t0 * C, T * C * 4, sb, n * C * 4, n * C * 4, B,
                                                    cudaMemcpyDeviceToHost, cs));
                     QNN_CUDA_TRY(cudaEventRecord(m->out_ev[4 + (k & 1)], cs));
                 } else {
-                    QNN_TRY(launch_softmax_rows(lg + t0 * B * C, rc, C, yd, os, B, T, t0));
+                    QNN_TRY(launch_softmax_rows(lg, rc, C, yd, os, B, T, t0));
                 }
                 t0 = t1;
                 return QNN_OK;
