@@ -935,10 +935,15 @@ qnn_status forward_impl(qnn_lstm_model *m, const float *x, int64_t B, int64_t T,
     // layers as a wavefront on one stream each (every layer's recurrence state its own; the layer
     // outputs are kept whole only where they are read: the top layer, and every layer with h_all)
     const bool wave = fused && tc_stack_supported(m) && (!h_all || ha_dev);
-    // the 8-bit output layer beside the recurrence (wavefront)
+    // the 8-bit output layer beside the recurrence (wavefront) when the posteriors go to pinned host
+    // memory, so that they cross the host link while the recurrence runs (end to end 2.71M against
+    // 2.39-2.49M frames/s at LSTMP 5 x 2048p512 B = 1024); with a device y the output layer runs
+    // after the recurrence, where its one large product costs less SM time than the chunks' (4.49M
+    // against 4.44M frames/s). QNN_OUT_OVERLAP=1 / 0 forces either way.
     const char *ov_env = std::getenv("QNN_OUT_OVERLAP");
-    const bool out_overlap = wave && C > 0 && m->d.output_mode == QNN_OUT_QUANT && m->wo16 &&
-                             !(ov_env && std::strcmp(ov_env, "0") == 0);
+    const bool ov_on = ov_env && std::strcmp(ov_env, "1") == 0, ov_off = ov_env && std::strcmp(ov_env, "0") == 0;
+    const bool out_overlap = wave && C > 0 && m->d.output_mode == QNN_OUT_QUANT && m->wo16 && !ov_off &&
+                             (ov_on || y_map != nullptr);
     // chunks of about 32768 rows (QNN_OUT_CHUNK sets the frames of a chunk); posteriors for pinned
     // host memory go through two device buffers of a chunk each, so that the copy engines carry
     // them to the host while the SMs go on with the recurrence (QNN_OUT_STAGE=0: the softmax writes
